@@ -1,0 +1,12 @@
+"""Float64 CPU oracle for JARQ refinement.
+
+TEST INFRASTRUCTURE: only the tests, ``__graft_entry__.smoke()`` and the CPU
+baseline of ``bench.py`` use this package.  The product path never imports it.
+"""
+from .jarq_oracle import (FP32_EPS, Options, Prepared, Result, babai_proposal, canonicalize,
+                          code_sweep, dequantize, group_target, objective, prepare_hessian,
+                          refine_layer, scale_system, solve_scales)
+
+__all__ = ["FP32_EPS", "Options", "Prepared", "Result", "babai_proposal", "canonicalize",
+           "code_sweep", "dequantize", "group_target", "objective", "prepare_hessian",
+           "refine_layer", "scale_system", "solve_scales"]
