@@ -1,0 +1,337 @@
+"""Benchmark of JARQ layer refinement on one GB300 (or N, weak scaling).
+
+One step = one ``jarq_refine_layer`` call refining the Llama-2-7B q_proj
+layer (4096 x 4096, g = 128, 3-bit, RTN host, K = 10 iterations, early stop
+off) from its host state: the whole hot path (target projection, then per
+iteration Gram + rhs, joint scale solve and the 32-group Babai sweep).
+Inputs are seeded synthetic tensors resident in HBM; the working set per
+step (H, W, P = W H and the residual, 64 MB each) exceeds the 129 MB L2.
+
+``value`` is weights refined per second over all ranks; ``e2e`` is the same
+metric through the C ABI with host buffers (host-to-device and back inside
+the timed region).  ``--impl reference`` times the float64 oracle (the
+reference arm of this build) on the host cores.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "JARQ refine s/layer & weights/s at 7B shapes; % of tensor/HBM roofline"
+UNIT = "weights/s"
+WORKLOAD = "llama2_7b_q_proj_4096x4096_g128_w3"
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+SM_COUNT = 152
+FP32_LANES_PER_SM = 128
+SM_MAX_MHZ = 2070.0
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=WORKLOAD)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0,
+                    help="target CPU time of the oracle baseline sample")
+    return ap.parse_args()
+
+
+def peaks():
+    try:
+        with open(PEAKS_FILE) as fh:
+            pk = json.load(fh)
+        return pk, "measured"
+    except OSError:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+# --------------------------------------------------------------------------
+# clocks sampled during the timed region
+# --------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200", "-i", str(self.gpu)], stdout=self.fh, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.fh.close()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as fh:
+            for line in fh:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for nm, v in zip(names, parts[5:9]):
+                    if v.lower().startswith("active"):
+                        reasons.add(nm)
+        os.unlink(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# --------------------------------------------------------------------------
+# oracle timing (CPU baseline and reference arm)
+# --------------------------------------------------------------------------
+
+def oracle_rows_per_second(lay_np, K, target_s, max_rows=None):
+    """Time the float64 oracle on a growing sample of rows until ~target_s."""
+    from oracle import Options, prepare_hessian, refine_layer
+    prep = prepare_hessian(lay_np.H, lay_np.g)
+    rng = np.random.default_rng(0)
+    n = 4
+    total_t, total_rows = 0.0, 0
+    while True:
+        rows = np.sort(rng.choice(lay_np.dout, size=min(n, lay_np.dout), replace=False))
+        t0 = time.perf_counter()
+        refine_layer(prep, lay_np.W[rows], lay_np.S0[rows], lay_np.Q0[rows], lay_np.Z[rows],
+                     lay_np.bits, Options(max_iters=K, early_stop=False))
+        dt = time.perf_counter() - t0
+        total_t += dt
+        total_rows += len(rows)
+        if total_t >= target_s or (max_rows and total_rows >= max_rows) or len(rows) >= lay_np.dout:
+            break
+        n = int(min(lay_np.dout, max(n * 2, n * (target_s - total_t) / max(dt, 1e-3))))
+    return total_rows, total_t
+
+
+def layer_to_numpy(lay):
+    from synth import Layer
+    return Layer(lay.name, lay.W.cpu().numpy(), lay.H.cpu().numpy(), lay.S0.cpu().numpy(),
+                 lay.Q0.cpu().numpy(), lay.Z.cpu().numpy(), lay.bits, lay.g, lay.K)
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return 0
+    import torch
+    from synth import config_layer
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    lay = layer_to_numpy(config_layer(args.workload, device=dev))
+    K = lay.K
+    per_step_rows = 4
+    from oracle import Options, prepare_hessian, refine_layer
+    prep = prepare_hessian(lay.H, lay.g)
+    rng = np.random.default_rng(1)
+    times = []
+    for it in range(args.warmup + args.steps):
+        rows = np.sort(rng.choice(lay.dout, size=per_step_rows, replace=False))
+        t0 = time.perf_counter()
+        refine_layer(prep, lay.W[rows], lay.S0[rows], lay.Q0[rows], lay.Z[rows], lay.bits,
+                     Options(max_iters=K, early_stop=False))
+        if it >= args.warmup:
+            times.append(time.perf_counter() - t0)
+    t = float(np.mean(times))
+    value = per_step_rows * lay.din / t
+    cores = os.cpu_count()
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": t * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": config_dict(lay, note=f"oracle on {per_step_rows} sampled rows per step"),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": f"{per_step_rows} of {lay.dout} rows per step, K={K}, full din"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
+def config_dict(lay, note=None):
+    c = {"workload": lay.name, "din": lay.din, "dout": lay.dout, "group_size": lay.g,
+         "bits": lay.bits, "K": lay.K, "early_stop": False, "host": "RTN",
+         "l2": "inputs larger than L2 (H, W, P, r: 64 MB each per step)"}
+    if note:
+        c["note"] = note
+    return c
+
+
+# --------------------------------------------------------------------------
+# our arm
+# --------------------------------------------------------------------------
+
+def algorithmic_flops(kernel, lay):
+    """One MMA-equivalent of useful work per launch (App. G.7 counts)."""
+    p, d, g = lay.dout, lay.din, lay.g
+    return {"phase_hr": 2.0 * p * g * d, "gram": 2.0 * p * d * d, "hw": 2.0 * p * d * d,
+            "objective": 2.0 * p * d * d}.get(kernel)
+
+
+def run_ours(args, rank, world):
+    import torch
+    from paper_2609_38599_gb300 import jarq
+    from synth import config_layer
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    lay = config_layer(args.workload, device=dev)
+    hess = jarq.prepare(lay.H, lay.g)
+    opts = jarq.default_options(max_iters=lay.K, early_stop=0)
+    S = lay.S0.clone()
+    Q = lay.Q0.clone()
+
+    def step():
+        S.copy_(lay.S0)
+        Q.copy_(lay.Q0)
+        jarq.refine(hess, lay.W, S, Q, lay.Z, lay.bits, options=opts, collect_stats=False)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES", "")
+    gpu_index = vis.split(",")[local] if vis and vis.split(",")[0].isdigit() else local
+    sampler = ClockSampler(gpu_index)
+    jarq.profile_reset()
+    jarq.profile_enable(True)
+    n0 = jarq.launch_count()
+    sampler.start()
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.steps):
+        step()
+    e1.record()
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    clocks = sampler.stop()
+    jarq.profile_enable(False)
+    launches = jarq.launch_count() - n0
+    ms = e0.elapsed_time(e1) / args.steps
+    if dist:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    weights = lay.din * lay.dout
+    value = world * weights / (ms / 1e3)
+    kernels = {}
+    for k in jarq.KERNELS:
+        n, tot = jarq.profile_read(k)
+        if n:
+            kernels[k] = {"launches": n, "total_ms": tot, "avg_us": 1e3 * tot / n,
+                          "share": None}
+    tot_all = sum(v["total_ms"] for v in kernels.values()) or 1.0
+    for v in kernels.values():
+        v["share"] = v["total_ms"] / tot_all
+    # dominant contraction kernel and its roofline
+    cand = [k for k in kernels if algorithmic_flops(k, lay)]
+    dom = max(cand, key=lambda k: kernels[k]["total_ms"]) if cand else None
+    roof = None
+    if dom:
+        avg_s = kernels[dom]["total_ms"] / kernels[dom]["launches"] / 1e3
+        achieved = algorithmic_flops(dom, lay) / avg_s / 1e12
+        peak = SM_COUNT * FP32_LANES_PER_SM * 2 * SM_MAX_MHZ * 1e6 / 1e12
+        roof = {"kernel": dom, "bound": "alu", "achieved": achieved, "peak": peak,
+                "unit": "TFLOP/s", "frac": achieved / peak, "traffic": None,
+                "peak_note": "fp32 FMA: 152 SMs x 128 lanes x 2 flop x 2070 MHz (CUDA-core contraction)"}
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "s_per_layer": ms / 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic (seeded Llama-2-7B-shaped layer, RTN host)",
+        "config": config_dict(lay), "roofline": roof, "gpu_launches": launches,
+        "launches_per_step": launches / args.steps, "clocks": clocks, "kernels": kernels,
+    }
+    # end to end through the C ABI with pinned host buffers
+    if rank == 0 or True:
+        pin = lambda t: t.cpu().pin_memory().numpy()
+        Wh, S0h, Q0h, Zh = pin(lay.W), pin(lay.S0), pin(lay.Q0), pin(lay.Z)
+        Sh = torch.empty_like(lay.S0, device="cpu").pin_memory().numpy()
+        Qh = torch.empty_like(lay.Q0, device="cpu").pin_memory().numpy()
+        times = []
+        for it in range(args.warmup + args.steps):
+            Sh[...] = S0h
+            Qh[...] = Q0h
+            t0 = time.perf_counter()
+            jarq.refine(hess, Wh, Sh, Qh, Zh, lay.bits, options=opts, collect_stats=False)
+            dt = time.perf_counter() - t0
+            if it >= args.warmup:
+                times.append(dt)
+        e2e_s = float(np.mean(times))
+        if dist:
+            t = torch.tensor([e2e_s], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_s = float(t.item())
+        line["e2e"] = {"value": world * weights / e2e_s, "unit": UNIT,
+                       "h2d_bytes_per_step": int(Wh.nbytes + S0h.nbytes + Q0h.nbytes + Zh.nbytes),
+                       "d2h_bytes_per_step": int(Sh.nbytes + Qh.nbytes),
+                       "ms_per_step": e2e_s * 1e3}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        lay_np = layer_to_numpy(lay)
+        rows, t = oracle_rows_per_second(lay_np, lay.K, args.cpu_seconds)
+        line["cpu_baseline"] = {"value": rows * lay.din / t, "unit": UNIT,
+                                "cores": os.cpu_count(), "kind": "oracle",
+                                "sample": f"{rows} of {lay.dout} rows, K={lay.K}, full din, "
+                                          f"{t:.1f} s"}
+    hess.close()
+    if rank == 0:
+        print(json.dumps(line))
+    if dist:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse_args()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if args.impl == "reference":
+        return run_reference(args, rank, world)
+    return run_ours(args, rank, world)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,167 @@
+/*
+ * jarq.h -- C ABI of the GB300 (sm_103a) JARQ layer-refinement library.
+ *
+ * JARQ (Joint Alternating Refinement for Quantization) refines a group-wise
+ * uniformly quantized linear layer.  Given the layer's weights W, the
+ * calibration Hessian H = A^T A (A = [X; nu I], Sec. 3.2, Eq. strict_target)
+ * and a host quantizer's scales S, integer codes Q and zero points Z
+ * (Sec. 3.1, Eq. quantized_group), it minimises the per-row objective
+ *
+ *     F_j = (w_j - what_j)^T H (w_j - what_j),  what_j = D_{s_j}(q_j - z_j)
+ *
+ * (Eq. bbmils_columns with the main target Y = A W) by alternating
+ *   (a) a joint least-squares fit of all G scales of a row, solved by
+ *       Cholesky on the G x G normal equations (Sec. 3.3.1, Eqs.
+ *       scale_design / scale_normal_equations, with the ridge safeguard of
+ *       App. E "Solving for scales"), and
+ *   (b) one Gauss-Seidel sweep of bounded Babai nearest-plane proposals over
+ *       the groups, each kept only if it strictly lowers the objective
+ *       (Sec. 3.3.2, Eqs. conditional_residual, group_qr, babai_update).
+ * Bit width, groups and zero points never change.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - Layout: W is float32 [dout][din] row-major (row j is the paper's column
+ *   w_j); S is float32 [dout][G]; Q is uint8 [dout][din]; Z is int32
+ *   [dout][G]; H is float32 [din][din]; G = din / group_size.
+ * - Pointers may be device memory or host memory (pageable or pinned).
+ *   Host buffers are staged through library-owned device buffers; device
+ *   buffers are used in place.  The caller owns every buffer it passes.
+ * - `stream` is a cudaStream_t passed as void* (NULL = the legacy default
+ *   stream).  Work is enqueued on it in order.  Calls return after the work
+ *   they enqueued has finished and its status has been read back.
+ * - Errors are reported as jarq_status values; no exception or abort crosses
+ *   the ABI.  On JARQ_ERR_ARG nothing is enqueued and no buffer is touched.
+ * - A handle is not thread-safe: do not use one handle from two host threads
+ *   or on two streams at the same time.  Different handles are independent.
+ */
+#ifndef JARQ_H_
+#define JARQ_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum jarq_status {
+    JARQ_OK = 0,
+    JARQ_ERR_ARG = 1,        /* invalid argument (size, pointer, range)        */
+    JARQ_ERR_NOT_SPD = 2,    /* a diagonal block H_ii is not positive definite */
+    JARQ_ERR_NUMERICAL = 3,  /* a scale system failed even with the ridge      */
+    JARQ_ERR_CUDA = 4,       /* a CUDA runtime or driver call failed           */
+    JARQ_ERR_TIMEOUT = 5,    /* reserved: a bounded device wait gave up        */
+    JARQ_ERR_NOMEM = 6       /* device allocation failed                       */
+} jarq_status;
+
+/* Opaque prepared Hessian: symmetrised H, its split-precision copy for the
+ * tensor cores and the per-group Cholesky factors R_i (H_ii = R_i^T R_i) with
+ * their inverses.  Sec. 3.3.2 (Eq. group_qr) precomputes these once and
+ * reuses them for every output row and iteration; R_i equals the paper's
+ * thin-QR factor up to row signs, to which Babai is invariant.  Library-owned;
+ * also caches the refinement workspaces, sized by the largest dout seen. */
+typedef struct jarq_hessian jarq_hessian;
+
+/* Solver settings (App. E "Numerical Updates and Stopping").  Fill with
+ * jarq_default_options() and override fields. */
+typedef struct jarq_options {
+    int   max_iters;     /* K, the iteration budget (paper: 3).  0 returns the host state. */
+    int   early_stop;    /* 1: per-row stop of Eq. strict_stopping for k >= 2; 0: run K iterations */
+    float tau_rel;       /* relative stop threshold tau (1e-5)                    */
+    float tau_abs;       /* absolute stop threshold tau (1e-5)                    */
+    float ridge;         /* lambda added when the Gram matrix is nearly singular (1e-4) */
+    float rcond;         /* r_cond of the near-singularity test (1e-10)           */
+    float eps;           /* eps_fp: FP32 machine epsilon; small-scale skip threshold */
+} jarq_options;
+
+/* Per-row statistics.  Every pointer may be NULL (not collected) and may be
+ * host or device memory; arrays have dout entries.
+ *   L_host     : objective F_j of the input state (S, Q)            [double]
+ *   L_final    : objective F_j of the returned state                 [double]
+ *   iters      : scale updates performed (<= max_iters)              [int32]
+ *   accepted   : Babai proposals accepted                            [int32]
+ *   ridge_hits : scale solves that needed the ridge                  [int32]
+ *   row_status : JARQ_OK or JARQ_ERR_NUMERICAL for that row          [int32]  */
+typedef struct jarq_stats {
+    double  *L_host;
+    double  *L_final;
+    int32_t *iters;
+    int32_t *accepted;
+    int32_t *ridge_hits;
+    int32_t *row_status;
+} jarq_stats;
+
+/* Default options: K = 3, early stop on, tau = 1e-5, ridge 1e-4,
+ * rcond 1e-10, eps = FLT_EPSILON (App. E). */
+jarq_options jarq_default_options(void);
+
+/* Prepare a Hessian for refinement (Sec. 3.3.2, Eq. group_qr; App. G.7
+ * "Shared preprocessing").
+ *   H          : float32 [din][din], host or device; symmetrised as (H+H^T)/2.
+ *   din        : input width, > 0, multiple of group_size.
+ *   group_size : g, 1 <= g <= 128.
+ *   nu2        : added to the diagonal (the paper's nu^2, Eq. strict_target);
+ *                pass 0 when H already contains its damping.
+ *   out        : receives the new handle (unchanged on error).
+ * Returns JARQ_ERR_NOT_SPD if some H_ii is not positive definite,
+ * JARQ_ERR_ARG for bad sizes or a NULL pointer. */
+jarq_status jarq_prepare_hessian(const float *H, int din, int group_size, float nu2,
+                                 jarq_hessian **out, void *stream);
+
+/* Refine one layer in place: K iterations of joint scale fit + Babai sweep
+ * (Sec. 3.3; App. E "Order of updates", "Early stopping", "Small scales").
+ *   h      : prepared Hessian for this layer's input (din, group size).
+ *   W      : float32 [dout][din], original weights (read only).
+ *   S      : float32 [dout][G], host scales in, refined signed scales out.
+ *   Q      : uint8 [dout][din], codes in [0, 2^bits - 1]; refined in place.
+ *   Z      : int32 [dout][G], zero points in [0, 2^bits - 1]; read only.
+ *   dout   : output rows, >= 0 (0 is a no-op).
+ *   bits   : b, 1 <= b <= 8.
+ *   opt    : solver settings (NULL = jarq_default_options()).
+ *   stats  : optional per-row statistics (NULL = none).
+ * Rows are independent; a row whose scale system fails even with the ridge
+ * keeps its last state and is marked JARQ_ERR_NUMERICAL in row_status, the
+ * other rows finish, and the call returns JARQ_ERR_NUMERICAL.  Codes or zero
+ * points outside [0, 2^bits - 1] return JARQ_ERR_ARG before any update. */
+jarq_status jarq_refine_layer(jarq_hessian *h, const float *W, float *S, uint8_t *Q,
+                              const int32_t *Z, int dout, int bits,
+                              const jarq_options *opt, jarq_stats *stats, void *stream);
+
+/* Per-row objective F_j = r_j^T H r_j, r_j = w_j - D_{s_j}(q_j - z_j)
+ * (Sec. 3.2, Eq. bbmils_columns), written as double to F_per_row[dout]
+ * (host or device).  Same layouts and checks as jarq_refine_layer. */
+jarq_status jarq_objective(jarq_hessian *h, const float *W, const float *S, const uint8_t *Q,
+                           const int32_t *Z, int dout, int bits, double *F_per_row,
+                           void *stream);
+
+/* Input width and group size of a prepared handle (0 for NULL). */
+int jarq_hessian_din(const jarq_hessian *h);
+int jarq_hessian_group_size(const jarq_hessian *h);
+
+/* Release a handle and its workspaces (NULL is a no-op).  Synchronises the
+ * device first so no enqueued work still uses them. */
+void jarq_hessian_destroy(jarq_hessian *h);
+
+/* Static, human-readable name of a status. */
+const char *jarq_status_string(jarq_status s);
+
+/* ---- Instrumentation (no counterpart in the paper) -------------------------
+ * Used by the benchmark to time individual kernels on the stream they run
+ * on.  When enabled, the library records a CUDA event pair around every
+ * kernel launch it makes; durations are accumulated per kernel name when the
+ * enclosing call synchronises.  Names: "validate", "residual", "init_rows",
+ * "hw", "gram", "scale_solve", "phase_hr", "babai", "objective",
+ * "symmetrize", "group_factor".  Not thread-safe. */
+void jarq_profile_enable(int on);
+void jarq_profile_reset(void);
+/* Accumulated launches and total device milliseconds of one kernel name since
+ * the last reset; returns 0 on success, -1 for an unknown name. */
+int jarq_profile_read(const char *kernel, long long *launches, double *total_ms);
+/* Number of kernels this library has launched since it was loaded. */
+long long jarq_launch_count(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* JARQ_H_ */

@@ -1,0 +1,366 @@
+// C ABI entry points: handle lifecycle, argument checks, staging of host
+// buffers and the refinement loop (Sec. 3.3; App. E "Order of updates").
+//
+// Per layer: residual r and target projection P = W H once, then for
+// k = 1..K: Gram + rhs from the current codes, the joint scale solve with
+// the early-stop bookkeeping, and one Gauss-Seidel sweep over the groups,
+// each group being a residual-product phase followed by a Babai phase.
+#include <float.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <new>
+
+#include "jarq_internal.cuh"
+
+using namespace jarq;
+
+namespace {
+
+jarq_status cuda_fail(cudaError_t e) {
+    return e == cudaErrorMemoryAllocation ? JARQ_ERR_NOMEM : JARQ_ERR_CUDA;
+}
+
+#define CK(x)                                  \
+    do {                                       \
+        cudaError_t e_ = (x);                  \
+        if (e_ != cudaSuccess) {               \
+            (void)cudaGetLastError();          \
+            return cuda_fail(e_);              \
+        }                                      \
+    } while (0)
+
+// Launch `call` (which enqueues `n` kernels) under the profiling scope `name`.
+#define RUN(name, n, call)              \
+    do {                                \
+        ProfScope ps_(name, st);        \
+        CK(call);                       \
+        ps_.done();                     \
+        count_launches(n);              \
+    } while (0)
+
+template <class T>
+cudaError_t dalloc(T **p, size_t n) {
+    *p = nullptr;
+    if (n == 0) n = 1;
+    return cudaMalloc((void **)p, n * sizeof(T));
+}
+
+bool is_device_ptr(const void *ptr) {
+    cudaPointerAttributes at;
+    if (cudaPointerGetAttributes(&at, ptr) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return false;
+    }
+    return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
+}
+
+void free_ws(Workspace &w) {
+    cudaFree(w.P);
+    cudaFree(w.r);
+    cudaFree(w.gram);
+    cudaFree(w.rhs);
+    cudaFree(w.hr);
+    cudaFree(w.fpart);
+    cudaFree(w.wHw);
+    cudaFree(w.L_prev);
+    cudaFree(w.dF_sweep);
+    cudaFree(w.L_host);
+    cudaFree(w.L_final);
+    cudaFree(w.active);
+    cudaFree(w.iters);
+    cudaFree(w.accepted);
+    cudaFree(w.ridge);
+    cudaFree(w.rstat);
+    cudaFree(w.sW);
+    cudaFree(w.sS);
+    cudaFree(w.sQ);
+    cudaFree(w.sZ);
+    w = Workspace{};
+}
+
+cudaError_t ensure_ws(jarq_hessian *h, int p) {
+    Workspace &w = h->ws;
+    if (p <= w.cap_rows) return cudaSuccess;
+    free_ws(w);
+    const size_t d = h->din, G = h->G, g = h->g;
+    const size_t nt = (d + 127) / 128;
+    cudaError_t e;
+    if ((e = dalloc(&w.P, (size_t)p * d)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.r, (size_t)p * d)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.gram, (size_t)p * G * G)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.rhs, (size_t)p * G)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.hr, (size_t)kSplitK * p * g)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.fpart, (size_t)p * nt)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.wHw, (size_t)p)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.L_prev, (size_t)p)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.dF_sweep, (size_t)p)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.L_host, (size_t)p)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.L_final, (size_t)p)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.active, (size_t)p)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.iters, (size_t)p)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.accepted, (size_t)p)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.ridge, (size_t)p)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.rstat, (size_t)p)) != cudaSuccess) return e;
+    w.cap_rows = p;
+    return cudaSuccess;
+}
+
+// Device views of the four layer arguments, staging host buffers.
+struct LayerArgs {
+    const float *W;
+    float *S;
+    uint8_t *Q;
+    const int32_t *Z;
+    bool hS = false, hQ = false;  // S / Q came from host memory
+};
+
+cudaError_t stage_layer(jarq_hessian *h, const float *W, const float *S, const uint8_t *Q,
+                        const int32_t *Z, int p, LayerArgs &out, cudaStream_t st) {
+    Workspace &w = h->ws;
+    const size_t d = h->din, G = h->G;
+    const bool dW = is_device_ptr(W), dS = is_device_ptr(S), dQ = is_device_ptr(Q),
+               dZ = is_device_ptr(Z);
+    if ((!dW || !dS || !dQ || !dZ) && w.stage_rows < p) {
+        cudaFree(w.sW);
+        cudaFree(w.sS);
+        cudaFree(w.sQ);
+        cudaFree(w.sZ);
+        w.sW = nullptr;
+        w.sS = nullptr;
+        w.sQ = nullptr;
+        w.sZ = nullptr;
+        w.stage_rows = 0;
+        cudaError_t e;
+        if ((e = dalloc(&w.sW, (size_t)p * d)) != cudaSuccess) return e;
+        if ((e = dalloc(&w.sS, (size_t)p * G)) != cudaSuccess) return e;
+        if ((e = dalloc(&w.sQ, (size_t)p * d)) != cudaSuccess) return e;
+        if ((e = dalloc(&w.sZ, (size_t)p * G)) != cudaSuccess) return e;
+        w.stage_rows = p;
+    }
+    out.W = W;
+    out.S = const_cast<float *>(S);
+    out.Q = const_cast<uint8_t *>(Q);
+    out.Z = Z;
+    cudaError_t e = cudaSuccess;
+    if (!dW) {
+        e = cudaMemcpyAsync(w.sW, W, (size_t)p * d * sizeof(float), cudaMemcpyHostToDevice, st);
+        out.W = w.sW;
+    }
+    if (e == cudaSuccess && !dS) {
+        e = cudaMemcpyAsync(w.sS, S, (size_t)p * G * sizeof(float), cudaMemcpyHostToDevice, st);
+        out.S = w.sS;
+        out.hS = true;
+    }
+    if (e == cudaSuccess && !dQ) {
+        e = cudaMemcpyAsync(w.sQ, Q, (size_t)p * d, cudaMemcpyHostToDevice, st);
+        out.Q = w.sQ;
+        out.hQ = true;
+    }
+    if (e == cudaSuccess && !dZ) {
+        e = cudaMemcpyAsync(w.sZ, Z, (size_t)p * G * sizeof(int32_t), cudaMemcpyHostToDevice,
+                            st);
+        out.Z = w.sZ;
+    }
+    return e;
+}
+
+jarq_status status_from_bits(int bits) {
+    if (bits & ST_NOT_SPD) return JARQ_ERR_NOT_SPD;
+    if (bits & (ST_BAD_CODE | ST_BAD_ZERO)) return JARQ_ERR_ARG;
+    if (bits & ST_NUMERICAL) return JARQ_ERR_NUMERICAL;
+    return JARQ_OK;
+}
+
+cudaError_t read_status(jarq_hessian *h, cudaStream_t st, int *bits) {
+    cudaError_t e = cudaMemcpyAsync(h->hstatus, h->dstatus, sizeof(int), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    *bits = (e == cudaSuccess) ? *h->hstatus : 0;
+    if (e == cudaSuccess) prof_collect();
+    return e;
+}
+
+// Common front half of refine/objective: stage, validate, residual.
+jarq_status layer_front(jarq_hessian *h, const float *W, const float *S, const uint8_t *Q,
+                        const int32_t *Z, int dout, int bits, LayerArgs &la, cudaStream_t st) {
+    CK(cudaSetDevice(h->device));
+    CK(ensure_ws(h, dout));
+    CK(stage_layer(h, W, S, Q, Z, dout, la, st));
+    CK(cudaMemsetAsync(h->dstatus, 0, sizeof(int), st));
+    RUN("validate", 1, launch_validate(la.Q, la.Z, dout, h->din, h->G, (1 << bits) - 1, h->dstatus, st));
+    int sb = 0;
+    CK(read_status(h, st, &sb));
+    if (sb) return status_from_bits(sb);
+    RUN("residual", 1, launch_residual(la.W, la.S, la.Q, la.Z, h->ws.r, dout, h->din, h->g, st));
+    return JARQ_OK;
+}
+
+bool layer_args_ok(const jarq_hessian *h, const void *W, const void *S, const void *Q,
+                   const void *Z, int dout, int bits) {
+    if (!h || dout < 0 || bits < 1 || bits > 8) return false;
+    if (dout > 0 && (!W || !S || !Q || !Z)) return false;
+    return true;
+}
+
+}  // namespace
+
+extern "C" {
+
+jarq_options jarq_default_options(void) {
+    jarq_options o;
+    o.max_iters = 3;
+    o.early_stop = 1;
+    o.tau_rel = 1e-5f;
+    o.tau_abs = 1e-5f;
+    o.ridge = 1e-4f;
+    o.rcond = 1e-10f;
+    o.eps = FLT_EPSILON;
+    return o;
+}
+
+const char *jarq_status_string(jarq_status s) {
+    switch (s) {
+        case JARQ_OK: return "ok";
+        case JARQ_ERR_ARG: return "invalid argument";
+        case JARQ_ERR_NOT_SPD: return "Hessian diagonal block not positive definite";
+        case JARQ_ERR_NUMERICAL: return "scale system failed even with the ridge";
+        case JARQ_ERR_CUDA: return "CUDA error";
+        case JARQ_ERR_TIMEOUT: return "device wait timed out";
+        case JARQ_ERR_NOMEM: return "device allocation failed";
+    }
+    return "unknown status";
+}
+
+int jarq_hessian_din(const jarq_hessian *h) { return h ? h->din : 0; }
+int jarq_hessian_group_size(const jarq_hessian *h) { return h ? h->g : 0; }
+
+void jarq_hessian_destroy(jarq_hessian *h) {
+    if (!h) return;
+    cudaSetDevice(h->device);
+    cudaDeviceSynchronize();
+    free_ws(h->ws);
+    cudaFree(h->Hs);
+    cudaFree(h->Lf);
+    cudaFree(h->Rinv);
+    cudaFree(h->dstatus);
+    cudaFreeHost(h->hstatus);
+    (void)cudaGetLastError();
+    delete h;
+}
+
+jarq_status jarq_prepare_hessian(const float *H, int din, int group_size, float nu2,
+                                 jarq_hessian **out, void *stream) {
+    if (!H || !out || din <= 0 || group_size < 1 || group_size > kMaxGroup ||
+        din % group_size != 0 || din / group_size > kMaxGroups || !isfinite(nu2))
+        return JARQ_ERR_ARG;
+    cudaStream_t st = (cudaStream_t)stream;
+    jarq_hessian *h = new (std::nothrow) jarq_hessian();
+    if (!h) return JARQ_ERR_NOMEM;
+    h->din = din;
+    h->g = group_size;
+    h->G = din / group_size;
+    jarq_status rc = JARQ_OK;
+    float *Hdev = nullptr;
+    do {
+        if (cudaGetDevice(&h->device) != cudaSuccess) { rc = JARQ_ERR_CUDA; break; }
+        const size_t dd = (size_t)din * din;
+        cudaError_t e;
+        if ((e = dalloc(&h->Hs, dd)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = dalloc(&h->Lf, (size_t)h->G * group_size * group_size)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = dalloc(&h->Rinv, (size_t)h->G * group_size * group_size)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = dalloc(&h->dstatus, 1)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = cudaMallocHost((void **)&h->hstatus, sizeof(int))) != cudaSuccess) { rc = cuda_fail(e); break; }
+        const float *Hsrc = H;
+        if (!is_device_ptr(H)) {
+            if ((e = dalloc(&Hdev, dd)) != cudaSuccess) { rc = cuda_fail(e); break; }
+            if ((e = cudaMemcpyAsync(Hdev, H, dd * sizeof(float), cudaMemcpyHostToDevice, st)) != cudaSuccess) { rc = cuda_fail(e); break; }
+            Hsrc = Hdev;
+        }
+        if ((e = cudaMemsetAsync(h->dstatus, 0, sizeof(int), st)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        { ProfScope ps("symmetrize", st); e = launch_symmetrize(Hsrc, h->Hs, din, nu2, st); ps.done(); count_launches(1); }
+        if (e != cudaSuccess) { rc = cuda_fail(e); break; }
+        { ProfScope ps("group_factor", st); e = launch_group_factor(h->Hs, h->Lf, h->Rinv, din, group_size, h->dstatus, st); ps.done(); count_launches(1); }
+        if (e != cudaSuccess) { rc = cuda_fail(e); break; }
+        int sb = 0;
+        if ((e = read_status(h, st, &sb)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        rc = status_from_bits(sb);
+    } while (0);
+    if (Hdev) {
+        cudaStreamSynchronize(st);
+        cudaFree(Hdev);
+    }
+    if (rc != JARQ_OK) {
+        jarq_hessian_destroy(h);
+        return rc;
+    }
+    *out = h;
+    return JARQ_OK;
+}
+
+jarq_status jarq_objective(jarq_hessian *h, const float *W, const float *S, const uint8_t *Q,
+                           const int32_t *Z, int dout, int bits, double *F_per_row,
+                           void *stream) {
+    if (!layer_args_ok(h, W, S, Q, Z, dout, bits) || (dout > 0 && !F_per_row))
+        return JARQ_ERR_ARG;
+    if (dout == 0) return JARQ_OK;
+    cudaStream_t st = (cudaStream_t)stream;
+    LayerArgs la;
+    jarq_status rc = layer_front(h, W, S, Q, Z, dout, bits, la, st);
+    if (rc != JARQ_OK) return rc;
+    Workspace &w = h->ws;
+    RUN("objective", 2, launch_objective(w.r, h->Hs, w.fpart, w.L_final, dout, h->din, st));
+    CK(cudaMemcpyAsync(F_per_row, w.L_final, (size_t)dout * sizeof(double), cudaMemcpyDefault, st));
+    CK(cudaStreamSynchronize(st));
+    prof_collect();
+    return JARQ_OK;
+}
+
+jarq_status jarq_refine_layer(jarq_hessian *h, const float *W, float *S, uint8_t *Q,
+                              const int32_t *Z, int dout, int bits, const jarq_options *opt,
+                              jarq_stats *stats, void *stream) {
+    if (!layer_args_ok(h, W, S, Q, Z, dout, bits)) return JARQ_ERR_ARG;
+    jarq_options o = opt ? *opt : jarq_default_options();
+    if (o.max_iters < 0 || !(o.ridge >= 0.f) || !(o.rcond >= 0.f) || !(o.eps >= 0.f))
+        return JARQ_ERR_ARG;
+    if (dout == 0) return JARQ_OK;
+    cudaStream_t st = (cudaStream_t)stream;
+    LayerArgs la;
+    jarq_status rc = layer_front(h, W, S, Q, Z, dout, bits, la, st);
+    if (rc != JARQ_OK) return rc;
+    Workspace &w = h->ws;
+    const int p = dout, d = h->din, g = h->g, G = h->G, qmax = (1 << bits) - 1;
+    RUN("init_rows", 1, launch_init_rows(w.active, w.iters, w.accepted, w.ridge, w.rstat, w.dF_sweep, p, st));
+    if (stats && stats->L_host)
+        RUN("objective", 2, launch_objective(w.r, h->Hs, w.fpart, w.L_host, p, d, st));
+    if (o.max_iters > 0) {
+        RUN("hw", 2, launch_hw(la.W, h->Hs, w.P, w.wHw, p, d, st));
+        for (int k = 1; k <= o.max_iters; ++k) {
+            RUN("gram", 1, launch_gram(la.Q, la.Z, h->Hs, w.P, w.active, w.gram, w.rhs, p, d, g, st));
+            RUN("scale_solve", 1, launch_scale_solve(w.gram, w.rhs, la.W, la.Q, la.Z, w.wHw, la.S, w.r, w.L_prev,
+                                  w.dF_sweep, w.active, w.iters, w.ridge, w.rstat, h->dstatus, p,
+                                  d, g, k, o, st));
+            for (int i = 0; i < G; ++i) {
+                RUN("phase_hr", 1, launch_phase_hr(w.r, h->Hs, w.active, w.hr, p, d, g, i, st));
+                RUN("babai", 1, launch_babai(w.hr, h->Lf, h->Rinv, la.W, la.S, la.Q, la.Z, w.r, w.active,
+                                w.dF_sweep, w.accepted, p, d, g, i, qmax, o.eps, st));
+            }
+        }
+    }
+    if (stats && stats->L_final)
+        RUN("objective", 2, launch_objective(w.r, h->Hs, w.fpart, w.L_final, p, d, st));
+    if (la.hS) CK(cudaMemcpyAsync(S, la.S, (size_t)p * G * sizeof(float), cudaMemcpyDeviceToHost, st));
+    if (la.hQ) CK(cudaMemcpyAsync(Q, la.Q, (size_t)p * d, cudaMemcpyDeviceToHost, st));
+    if (stats) {
+        if (stats->L_host) CK(cudaMemcpyAsync(stats->L_host, w.L_host, p * sizeof(double), cudaMemcpyDefault, st));
+        if (stats->L_final) CK(cudaMemcpyAsync(stats->L_final, w.L_final, p * sizeof(double), cudaMemcpyDefault, st));
+        if (stats->iters) CK(cudaMemcpyAsync(stats->iters, w.iters, p * sizeof(int), cudaMemcpyDefault, st));
+        if (stats->accepted) CK(cudaMemcpyAsync(stats->accepted, w.accepted, p * sizeof(int), cudaMemcpyDefault, st));
+        if (stats->ridge_hits) CK(cudaMemcpyAsync(stats->ridge_hits, w.ridge, p * sizeof(int), cudaMemcpyDefault, st));
+        if (stats->row_status) CK(cudaMemcpyAsync(stats->row_status, w.rstat, p * sizeof(int), cudaMemcpyDefault, st));
+    }
+    int sb = 0;
+    CK(read_status(h, st, &sb));
+    return status_from_bits(sb);
+}
+
+}  // extern "C"

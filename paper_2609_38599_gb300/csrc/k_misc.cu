@@ -1,0 +1,93 @@
+// Elementwise and bookkeeping kernels of the refinement path.
+#include "jarq_internal.cuh"
+
+namespace jarq {
+namespace {
+
+// Codes and zero points must lie in [0, qmax] (Sec. 3.1: q in B^{d_i};
+// integer zero points kept from the host).
+__global__ void validate_kernel(const uint8_t *__restrict__ Q, const int32_t *__restrict__ Z,
+                                size_t nq, size_t nz, int qmax, int *status) {
+    __shared__ int flag;
+    if (threadIdx.x == 0) flag = 0;
+    __syncthreads();
+    int local = 0;
+    const size_t stride = (size_t)gridDim.x * blockDim.x;
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < nq; i += stride)
+        if (Q[i] > qmax) local |= ST_BAD_CODE;
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < nz; i += stride)
+        if (Z[i] < 0 || Z[i] > qmax) local |= ST_BAD_ZERO;
+    if (local) atomicOr(&flag, local);
+    __syncthreads();
+    if (threadIdx.x == 0 && flag) atomicOr(status, flag);
+}
+
+// r = w - s (q - z), one rounding (fma) per element (Eq. quantized_group).
+__global__ void residual_kernel(const float *__restrict__ W, const float *__restrict__ S,
+                                const uint8_t *__restrict__ Q, const int32_t *__restrict__ Z,
+                                float *__restrict__ r, int p, int d, int g) {
+    const int G = d / g;
+    const size_t n = (size_t)p * d;
+    const size_t stride = (size_t)gridDim.x * blockDim.x;
+    for (size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x; idx < n; idx += stride) {
+        const size_t j = idx / d;
+        const int grp = (int)(idx - j * d) / g;
+        const float c = (float)((int)Q[idx] - Z[j * G + grp]);
+        r[idx] = fmaf(-S[j * G + grp], c, W[idx]);
+    }
+}
+
+__global__ void init_rows_kernel(int *active, int *iters, int *accepted, int *ridge, int *rstat,
+                                 double *dF_sweep, int p) {
+    int j = blockIdx.x * blockDim.x + threadIdx.x;
+    if (j < p) {
+        active[j] = 1;
+        iters[j] = 0;
+        accepted[j] = 0;
+        ridge[j] = 0;
+        rstat[j] = 0;
+        dF_sweep[j] = 0.0;
+    }
+}
+
+}  // namespace
+
+int num_sms() {
+    static int n = 0;
+    if (!n) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+        if (n <= 0) n = 1;
+    }
+    return n;
+}
+
+cudaError_t launch_validate(const uint8_t *Q, const int32_t *Z, int p, int d, int G, int qmax,
+                            int *status, cudaStream_t s) {
+    size_t nq = (size_t)p * d, nz = (size_t)p * G;
+    int blocks = (int)((nq + 255) / 256);
+    if (blocks > 4 * num_sms()) blocks = 4 * num_sms();
+    if (blocks < 1) blocks = 1;
+    validate_kernel<<<blocks, 256, 0, s>>>(Q, Z, nq, nz, qmax, status);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_residual(const float *W, const float *S, const uint8_t *Q, const int32_t *Z,
+                            float *r, int p, int d, int g, cudaStream_t s) {
+    size_t n = (size_t)p * d;
+    int blocks = (int)((n + 255) / 256);
+    if (blocks > 8 * num_sms()) blocks = 8 * num_sms();
+    if (blocks < 1) blocks = 1;
+    residual_kernel<<<blocks, 256, 0, s>>>(W, S, Q, Z, r, p, d, g);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_init_rows(int *active, int *iters, int *accepted, int *ridge, int *rstat,
+                             double *dF_sweep, int p, cudaStream_t s) {
+    init_rows_kernel<<<(p + 255) / 256, 256, 0, s>>>(active, iters, accepted, ridge, rstat,
+                                                      dF_sweep, p);
+    return cudaGetLastError();
+}
+
+}  // namespace jarq

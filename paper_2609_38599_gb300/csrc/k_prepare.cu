@@ -1,0 +1,128 @@
+// Hessian preparation: symmetrisation and per-group Cholesky factors.
+//
+// Sec. 3.3.2, Eq. group_qr: each group's factor R_i (A_i = U_i R_i) is
+// computed once per layer and reused for every output row and iteration.
+// With H = A^T A, R_i^T R_i = H_ii, so R_i is taken as the upper Cholesky
+// factor of H_ii (equal to the QR factor up to row signs, to which the
+// Babai recursion is invariant).  The factor and its inverse are computed in
+// float64 in shared memory and stored as float32:
+//   Lf[i]   = L_i = R_i^T          (lower, row-major: Lf[l][m] = R_i[m][l])
+//   Rinv[i] = R_i^{-1}             (upper, row-major)
+#include "jarq_internal.cuh"
+
+namespace jarq {
+namespace {
+
+// out = (H + H^T)/2 + nu2 I, through 32x32 shared-memory tiles.
+__global__ void symmetrize_kernel(const float *__restrict__ H, float *__restrict__ Hs, int d,
+                                  float nu2) {
+    __shared__ float tile[32][33];
+    const int bx = blockIdx.x * 32, by = blockIdx.y * 32;
+    const int tx = threadIdx.x, ty = threadIdx.y;  // 32 x 8
+    for (int yy = ty; yy < 32; yy += 8) {
+        int row = bx + yy, col = by + tx;  // transposed block
+        tile[yy][tx] = (row < d && col < d) ? H[(size_t)row * d + col] : 0.f;
+    }
+    __syncthreads();
+    for (int yy = ty; yy < 32; yy += 8) {
+        int row = by + yy, col = bx + tx;
+        if (row < d && col < d) {
+            float v = 0.5f * (H[(size_t)row * d + col] + tile[tx][yy]);
+            if (row == col) v += nu2;
+            Hs[(size_t)row * d + col] = v;
+        }
+    }
+}
+
+// One block per group: float64 Cholesky of H_ii in shared memory, then an
+// in-place inverse of the lower factor.
+__global__ void group_factor_kernel(const float *__restrict__ Hs, float *__restrict__ Lf,
+                                    float *__restrict__ Rinv, int d, int g, int *status) {
+    extern __shared__ double smem[];
+    const int ld = g + 1;
+    double *A = smem;               // [g][g+1]
+    double *tmp = smem + g * ld;    // [g]
+    __shared__ int failed;
+    const int grp = blockIdx.x;
+    const int base = grp * g;
+    const int tid = threadIdx.x, nt = blockDim.x;
+    if (tid == 0) failed = 0;
+    for (int idx = tid; idx < g * g; idx += nt) {
+        int a = idx / g, b = idx % g;
+        A[a * ld + b] = (double)Hs[(size_t)(base + a) * d + base + b];
+    }
+    __syncthreads();
+    // right-looking Cholesky, lower triangle
+    for (int k = 0; k < g; ++k) {
+        if (tid == 0) {
+            double piv = A[k * ld + k];
+            if (!(piv > 0.0) || !isfinite(piv)) {
+                failed = 1;
+            } else {
+                A[k * ld + k] = sqrt(piv);
+            }
+        }
+        __syncthreads();
+        if (failed) break;
+        const double lkk = A[k * ld + k];
+        for (int a = k + 1 + tid; a < g; a += nt) A[a * ld + k] /= lkk;
+        __syncthreads();
+        const int n = g - k - 1;
+        for (int idx = tid; idx < n * n; idx += nt) {
+            int a = k + 1 + idx / n, b = k + 1 + idx % n;
+            if (b <= a) A[a * ld + b] -= A[a * ld + k] * A[b * ld + k];
+        }
+        __syncthreads();
+    }
+    if (failed) {
+        if (tid == 0) atomicOr(status, ST_NOT_SPD);
+        return;
+    }
+    float *Lo = Lf + (size_t)grp * g * g;
+    for (int idx = tid; idx < g * g; idx += nt) {
+        int a = idx / g, b = idx % g;
+        Lo[idx] = (b <= a) ? (float)A[a * ld + b] : 0.f;
+    }
+    __syncthreads();
+    // in-place inverse of the lower factor, columns from last to first:
+    // Linv[j][j] = 1/L[j][j]; Linv[j+1:, j] = -Linv[j][j] * Linv[j+1:, j+1:] L[j+1:, j]
+    for (int j = g - 1; j >= 0; --j) {
+        for (int a = j + 1 + tid; a < g; a += nt) tmp[a] = A[a * ld + j];
+        __syncthreads();
+        const double inv_jj = 1.0 / A[j * ld + j];
+        for (int a = j + 1 + tid; a < g; a += nt) {
+            double acc = 0.0;
+            for (int b = j + 1; b <= a; ++b) acc += A[a * ld + b] * tmp[b];
+            A[a * ld + j] = -acc * inv_jj;
+        }
+        __syncthreads();
+        if (tid == 0) A[j * ld + j] = inv_jj;
+        __syncthreads();
+    }
+    // Rinv = (L^{-1})^T : Rinv[m][l] = Linv[l][m]
+    float *Ri = Rinv + (size_t)grp * g * g;
+    for (int idx = tid; idx < g * g; idx += nt) {
+        int m = idx / g, l = idx % g;
+        Ri[idx] = (l >= m) ? (float)A[l * ld + m] : 0.f;
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_symmetrize(const float *H, float *Hs, int d, float nu2, cudaStream_t s) {
+    dim3 grid((d + 31) / 32, (d + 31) / 32), block(32, 8);
+    symmetrize_kernel<<<grid, block, 0, s>>>(H, Hs, d, nu2);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_group_factor(const float *Hs, float *Lf, float *Rinv, int d, int g,
+                                int *status, cudaStream_t s) {
+    size_t smem = (size_t)(g * (g + 1) + g) * sizeof(double);
+    cudaError_t e = cudaFuncSetAttribute(group_factor_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    group_factor_kernel<<<d / g, 256, smem, s>>>(Hs, Lf, Rinv, d, g, status);
+    return cudaGetLastError();
+}
+
+}  // namespace jarq

@@ -1,0 +1,254 @@
+"""Python binding of the JARQ C ABI (``include/jarq.h``).
+
+Argument marshalling only: every step of the refinement runs in the CUDA
+library ``libjarq.so``.  Tensors are passed as raw pointers on torch's
+current CUDA stream; NumPy arrays are passed as host pointers and staged by
+the library.  There is no CPU fallback: importing this module raises if the
+library has not been built.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libjarq.so")
+
+JARQ_OK = 0
+JARQ_ERR_ARG = 1
+JARQ_ERR_NOT_SPD = 2
+JARQ_ERR_NUMERICAL = 3
+JARQ_ERR_CUDA = 4
+JARQ_ERR_TIMEOUT = 5
+JARQ_ERR_NOMEM = 6
+
+# Names declared in include/jarq.h (checked by the test-suite).
+EXPORTS = ("jarq_default_options", "jarq_prepare_hessian", "jarq_refine_layer",
+           "jarq_objective", "jarq_hessian_din", "jarq_hessian_group_size",
+           "jarq_hessian_destroy", "jarq_status_string", "jarq_profile_enable",
+           "jarq_profile_reset", "jarq_profile_read", "jarq_launch_count")
+
+
+class JarqError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)} (status {status})")
+
+
+class Options(ctypes.Structure):
+    _fields_ = [("max_iters", ctypes.c_int), ("early_stop", ctypes.c_int),
+                ("tau_rel", ctypes.c_float), ("tau_abs", ctypes.c_float),
+                ("ridge", ctypes.c_float), ("rcond", ctypes.c_float),
+                ("eps", ctypes.c_float)]
+
+
+class Stats(ctypes.Structure):
+    _fields_ = [("L_host", ctypes.c_void_p), ("L_final", ctypes.c_void_p),
+                ("iters", ctypes.c_void_p), ("accepted", ctypes.c_void_p),
+                ("ridge_hits", ctypes.c_void_p), ("row_status", ctypes.c_void_p)]
+
+
+def _load():
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"JARQ CUDA library not built: {LIB_PATH} is missing "
+                          "(run __graft_entry__.build())")
+    lib = ctypes.CDLL(LIB_PATH)
+    vp, ci, cf = ctypes.c_void_p, ctypes.c_int, ctypes.c_float
+    lib.jarq_default_options.restype = Options
+    lib.jarq_default_options.argtypes = []
+    lib.jarq_prepare_hessian.restype = ci
+    lib.jarq_prepare_hessian.argtypes = [vp, ci, ci, cf, ctypes.POINTER(vp), vp]
+    lib.jarq_refine_layer.restype = ci
+    lib.jarq_refine_layer.argtypes = [vp, vp, vp, vp, vp, ci, ci, ctypes.POINTER(Options),
+                                      ctypes.POINTER(Stats), vp]
+    lib.jarq_objective.restype = ci
+    lib.jarq_objective.argtypes = [vp, vp, vp, vp, vp, ci, ci, vp, vp]
+    lib.jarq_hessian_din.restype = ci
+    lib.jarq_hessian_din.argtypes = [vp]
+    lib.jarq_hessian_group_size.restype = ci
+    lib.jarq_hessian_group_size.argtypes = [vp]
+    lib.jarq_hessian_destroy.restype = None
+    lib.jarq_hessian_destroy.argtypes = [vp]
+    lib.jarq_status_string.restype = ctypes.c_char_p
+    lib.jarq_status_string.argtypes = [ci]
+    lib.jarq_profile_enable.restype = None
+    lib.jarq_profile_enable.argtypes = [ci]
+    lib.jarq_profile_reset.restype = None
+    lib.jarq_profile_reset.argtypes = []
+    lib.jarq_profile_read.restype = ci
+    lib.jarq_profile_read.argtypes = [ctypes.c_char_p, ctypes.POINTER(ctypes.c_longlong),
+                                      ctypes.POINTER(ctypes.c_double)]
+    lib.jarq_launch_count.restype = ctypes.c_longlong
+    lib.jarq_launch_count.argtypes = []
+    return lib
+
+
+_lib = _load()
+
+
+def library():
+    """The loaded ctypes library (for tests that call the C ABI directly)."""
+    return _lib
+
+
+KERNELS = ("validate", "residual", "init_rows", "hw", "gram", "scale_solve", "phase_hr",
+           "babai", "objective", "symmetrize", "group_factor")
+
+
+def profile_enable(on: bool = True):
+    """Record CUDA events around each library kernel launch (instrumentation)."""
+    _lib.jarq_profile_enable(1 if on else 0)
+
+
+def profile_reset():
+    _lib.jarq_profile_reset()
+
+
+def profile_read(kernel: str):
+    """(launches, total device ms) accumulated for one kernel name."""
+    n = ctypes.c_longlong()
+    ms = ctypes.c_double()
+    if _lib.jarq_profile_read(kernel.encode(), ctypes.byref(n), ctypes.byref(ms)) != 0:
+        raise KeyError(kernel)
+    return int(n.value), float(ms.value)
+
+
+def launch_count() -> int:
+    """Kernels launched by the library since it was loaded."""
+    return int(_lib.jarq_launch_count())
+
+
+def status_string(status: int) -> str:
+    return _lib.jarq_status_string(int(status)).decode()
+
+
+def default_options(**overrides) -> Options:
+    o = _lib.jarq_default_options()
+    for k, v in overrides.items():
+        if not hasattr(o, k):
+            raise KeyError(f"unknown option {k}")
+        setattr(o, k, type(getattr(o, k))(v))
+    return o
+
+
+def _is_torch(x):
+    return type(x).__module__.startswith("torch")
+
+
+def _ptr(x, dtype_np):
+    """Raw pointer of a contiguous torch tensor or NumPy array of the given dtype."""
+    if x is None:
+        return None
+    if _is_torch(x):
+        import torch
+        want = {np.float32: torch.float32, np.uint8: torch.uint8, np.int32: torch.int32,
+                np.float64: torch.float64}[dtype_np]
+        if x.dtype != want or not x.is_contiguous():
+            raise TypeError(f"expected a contiguous {want} tensor, got {x.dtype}")
+        return x.data_ptr()
+    if not isinstance(x, np.ndarray) or x.dtype != dtype_np or not x.flags.c_contiguous:
+        raise TypeError(f"expected a C-contiguous {np.dtype(dtype_np)} array")
+    return x.ctypes.data
+
+
+def _stream(*tensors):
+    for t in tensors:
+        if _is_torch(t) and t.is_cuda:
+            import torch
+            return ctypes.c_void_p(torch.cuda.current_stream(t.device).cuda_stream)
+    return ctypes.c_void_p(None)
+
+
+class Hessian:
+    """A prepared Hessian (``jarq_prepare_hessian``); freed on ``close``."""
+
+    def __init__(self, H, group_size: int, nu2: float = 0.0):
+        d = int(H.shape[0])
+        if tuple(H.shape) != (d, d):
+            raise ValueError("H must be square")
+        handle = ctypes.c_void_p()
+        st = _lib.jarq_prepare_hessian(_ptr(H, np.float32), d, int(group_size), float(nu2),
+                                       ctypes.byref(handle), _stream(H))
+        if st != JARQ_OK:
+            raise JarqError(st, "jarq_prepare_hessian")
+        self._h = handle
+        self.din = d
+        self.group_size = int(group_size)
+
+    @property
+    def handle(self):
+        return self._h
+
+    def close(self):
+        if self._h is not None and self._h.value:
+            _lib.jarq_hessian_destroy(self._h)
+        self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def prepare(H, group_size: int, nu2: float = 0.0) -> Hessian:
+    return Hessian(H, group_size, nu2)
+
+
+@dataclass
+class RefineStats:
+    L_host: object
+    L_final: object
+    iters: object
+    accepted: object
+    ridge_hits: object
+    row_status: object
+    status: int
+
+
+def _alloc_like(ref, n, dtype_np):
+    if _is_torch(ref):
+        import torch
+        tdt = {np.float64: torch.float64, np.int32: torch.int32}[dtype_np]
+        return torch.empty(n, dtype=tdt, device=ref.device)
+    return np.empty(n, dtype=dtype_np)
+
+
+def refine(hess: Hessian, W, S, Q, Z, bits: int, options: Options = None,
+           collect_stats: bool = True, raise_on_error: bool = True, **opt):
+    """``jarq_refine_layer``: refine S and Q in place; returns RefineStats."""
+    o = options if options is not None else default_options(**opt)
+    dout = int(W.shape[0])
+    st = None
+    stats = None
+    if collect_stats:
+        st = RefineStats(*(_alloc_like(W, dout, t) for t in
+                           (np.float64, np.float64, np.int32, np.int32, np.int32, np.int32)),
+                         status=0)
+        stats = Stats(*(_ptr(x, t) for x, t in zip(
+            (st.L_host, st.L_final, st.iters, st.accepted, st.ridge_hits, st.row_status),
+            (np.float64, np.float64, np.int32, np.int32, np.int32, np.int32))))
+    status = _lib.jarq_refine_layer(hess.handle, _ptr(W, np.float32), _ptr(S, np.float32),
+                                    _ptr(Q, np.uint8), _ptr(Z, np.int32), dout, int(bits),
+                                    ctypes.byref(o), ctypes.byref(stats) if stats else None,
+                                    _stream(W, S, Q, Z))
+    if st is not None:
+        st.status = status
+    if raise_on_error and status not in (JARQ_OK,):
+        raise JarqError(status, "jarq_refine_layer")
+    return st if st is not None else status
+
+
+def objective(hess: Hessian, W, S, Q, Z, bits: int, out=None):
+    """``jarq_objective``: per-row F_j as float64."""
+    dout = int(W.shape[0])
+    F = out if out is not None else _alloc_like(W, dout, np.float64)
+    status = _lib.jarq_objective(hess.handle, _ptr(W, np.float32), _ptr(S, np.float32),
+                                 _ptr(Q, np.uint8), _ptr(Z, np.int32), dout, int(bits),
+                                 _ptr(F, np.float64), _stream(W, S, Q, Z))
+    if status != JARQ_OK:
+        raise JarqError(status, "jarq_objective")
+    return F
