@@ -2,10 +2,10 @@
 
 One step = one ``jarq_refine_layer`` call refining the Llama-2-7B q_proj
 layer (4096 x 4096, g = 128, 3-bit, RTN host, K = 10 iterations, early stop
-off) from its host state: the whole hot path (target projection, then per
-iteration Gram + rhs, joint scale solve and the 32-group Babai sweep).
+off) from its host state: the whole hot path (per iteration the residual
+product H r, Gram matrices, joint scale solve and the 32-group Babai sweep).
 Inputs are seeded synthetic tensors resident in HBM; the working set per
-step (H, W, P = W H and the residual, 64 MB each) exceeds the 129 MB L2.
+step (H, W, H r and the residual, 64 MB each) exceeds the 129 MB L2.
 
 ``value`` is weights refined per second over all ranks; ``e2e`` is the same
 metric through the C ABI with host buffers (host-to-device and back inside
@@ -198,8 +198,8 @@ def config_dict(lay, note=None):
 def algorithmic_flops(kernel, lay):
     """One MMA-equivalent of useful work per launch (App. G.7 counts)."""
     p, d, g = lay.dout, lay.din, lay.g
-    return {"phase_hr": 2.0 * p * g * d, "gram": 2.0 * p * d * d, "hw": 2.0 * p * d * d,
-            "objective": 2.0 * p * d * d}.get(kernel)
+    return {"phase_hr": 2.0 * p * g * d, "gram": 2.0 * p * d * d,
+            "hr_full": 2.0 * p * d * d}.get(kernel)
 
 
 def run_ours(args, rank, world):

@@ -150,7 +150,7 @@ const char *jarq_status_string(jarq_status s);
  * on.  When enabled, the library records a CUDA event pair around every
  * kernel launch it makes; durations are accumulated per kernel name when the
  * enclosing call synchronises.  Names: "validate", "residual", "init_rows",
- * "hw", "gram", "scale_solve", "phase_hr", "babai", "objective",
+ * "hr_full", "grad", "gram", "scale_solve", "phase_hr", "babai",
  * "symmetrize", "group_factor".  Not thread-safe. */
 void jarq_profile_enable(int on);
 void jarq_profile_reset(void);

@@ -1,10 +1,11 @@
 // C ABI entry points: handle lifecycle, argument checks, staging of host
 // buffers and the refinement loop (Sec. 3.3; App. E "Order of updates").
 //
-// Per layer: residual r and target projection P = W H once, then for
-// k = 1..K: Gram + rhs from the current codes, the joint scale solve with
-// the early-stop bookkeeping, and one Gauss-Seidel sweep over the groups,
-// each group being a residual-product phase followed by a Babai phase.
+// Per iteration k = 1..K: the product H r of the current residual (giving
+// the objective and the scale gradient g_i = c_i^T (H r)_i), the Gram
+// matrices of the current codes, the joint scale solve with the early-stop
+// bookkeeping, and one Gauss-Seidel sweep over the groups, each group being
+// a residual-product phase followed by a Babai phase.
 #include <float.h>
 #include <stdlib.h>
 #include <string.h>
@@ -56,13 +57,12 @@ bool is_device_ptr(const void *ptr) {
 }
 
 void free_ws(Workspace &w) {
-    cudaFree(w.P);
+    cudaFree(w.Hr);
     cudaFree(w.r);
     cudaFree(w.gram);
-    cudaFree(w.rhs);
+    cudaFree(w.gvec);
     cudaFree(w.hr);
-    cudaFree(w.fpart);
-    cudaFree(w.wHw);
+    cudaFree(w.F_start);
     cudaFree(w.L_prev);
     cudaFree(w.dF_sweep);
     cudaFree(w.L_host);
@@ -84,15 +84,13 @@ cudaError_t ensure_ws(jarq_hessian *h, int p) {
     if (p <= w.cap_rows) return cudaSuccess;
     free_ws(w);
     const size_t d = h->din, G = h->G, g = h->g;
-    const size_t nt = (d + 127) / 128;
     cudaError_t e;
-    if ((e = dalloc(&w.P, (size_t)p * d)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.Hr, (size_t)p * d)) != cudaSuccess) return e;
     if ((e = dalloc(&w.r, (size_t)p * d)) != cudaSuccess) return e;
     if ((e = dalloc(&w.gram, (size_t)p * G * G)) != cudaSuccess) return e;
-    if ((e = dalloc(&w.rhs, (size_t)p * G)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.gvec, (size_t)p * G)) != cudaSuccess) return e;
     if ((e = dalloc(&w.hr, (size_t)kSplitK * p * g)) != cudaSuccess) return e;
-    if ((e = dalloc(&w.fpart, (size_t)p * nt)) != cudaSuccess) return e;
-    if ((e = dalloc(&w.wHw, (size_t)p)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.F_start, (size_t)p)) != cudaSuccess) return e;
     if ((e = dalloc(&w.L_prev, (size_t)p)) != cudaSuccess) return e;
     if ((e = dalloc(&w.dF_sweep, (size_t)p)) != cudaSuccess) return e;
     if ((e = dalloc(&w.L_host, (size_t)p)) != cudaSuccess) return e;
@@ -308,7 +306,8 @@ jarq_status jarq_objective(jarq_hessian *h, const float *W, const float *S, cons
     jarq_status rc = layer_front(h, W, S, Q, Z, dout, bits, la, st);
     if (rc != JARQ_OK) return rc;
     Workspace &w = h->ws;
-    RUN("objective", 2, launch_objective(w.r, h->Hs, w.fpart, w.L_final, dout, h->din, st));
+    RUN("hr_full", 1, launch_hr_full(w.r, h->Hs, w.Hr, dout, h->din, st));
+    RUN("grad", 1, launch_grad(la.Q, la.Z, w.r, w.Hr, nullptr, w.L_final, dout, h->din, h->g, st));
     CK(cudaMemcpyAsync(F_per_row, w.L_final, (size_t)dout * sizeof(double), cudaMemcpyDefault, st));
     CK(cudaStreamSynchronize(st));
     prof_collect();
@@ -330,24 +329,29 @@ jarq_status jarq_refine_layer(jarq_hessian *h, const float *W, float *S, uint8_t
     Workspace &w = h->ws;
     const int p = dout, d = h->din, g = h->g, G = h->G, qmax = (1 << bits) - 1;
     RUN("init_rows", 1, launch_init_rows(w.active, w.iters, w.accepted, w.ridge, w.rstat, w.dF_sweep, p, st));
-    if (stats && stats->L_host)
-        RUN("objective", 2, launch_objective(w.r, h->Hs, w.fpart, w.L_host, p, d, st));
-    if (o.max_iters > 0) {
-        RUN("hw", 2, launch_hw(la.W, h->Hs, w.P, w.wHw, p, d, st));
-        for (int k = 1; k <= o.max_iters; ++k) {
-            RUN("gram", 1, launch_gram(la.Q, la.Z, h->Hs, w.P, w.active, w.gram, w.rhs, p, d, g, st));
-            RUN("scale_solve", 1, launch_scale_solve(w.gram, w.rhs, la.W, la.Q, la.Z, w.wHw, la.S, w.r, w.L_prev,
-                                  w.dF_sweep, w.active, w.iters, w.ridge, w.rstat, h->dstatus, p,
-                                  d, g, k, o, st));
-            for (int i = 0; i < G; ++i) {
-                RUN("phase_hr", 1, launch_phase_hr(w.r, h->Hs, w.active, w.hr, p, d, g, i, st));
-                RUN("babai", 1, launch_babai(w.hr, h->Lf, h->Rinv, la.W, la.S, la.Q, la.Z, w.r, w.active,
-                                w.dF_sweep, w.accepted, p, d, g, i, qmax, o.eps, st));
-            }
+    for (int k = 1; k <= o.max_iters; ++k) {
+        RUN("hr_full", 1, launch_hr_full(w.r, h->Hs, w.Hr, p, d, st));
+        RUN("grad", 1, launch_grad(la.Q, la.Z, w.r, w.Hr, w.gvec, w.F_start, p, d, g, st));
+        if (k == 1 && stats && stats->L_host)
+            CK(cudaMemcpyAsync(w.L_host, w.F_start, p * sizeof(double), cudaMemcpyDeviceToDevice, st));
+        RUN("gram", 1, launch_gram(la.Q, la.Z, h->Hs, w.active, w.gram, p, d, g, st));
+        RUN("scale_solve", 1, launch_scale_solve(w.gram, w.gvec, la.W, la.Q, la.Z, w.F_start, la.S, w.r,
+                                                 w.L_prev, w.dF_sweep, w.active, w.iters, w.ridge, w.rstat,
+                                                 h->dstatus, p, d, g, k, o, st));
+        for (int i = 0; i < G; ++i) {
+            RUN("phase_hr", 1, launch_phase_hr(w.r, h->Hs, w.active, w.hr, p, d, g, i, st));
+            RUN("babai", 1, launch_babai(w.hr, h->Lf, h->Rinv, la.W, la.S, la.Q, la.Z, w.r, w.active,
+                                         w.dF_sweep, w.accepted, p, d, g, i, qmax, o.eps, st));
         }
     }
-    if (stats && stats->L_final)
-        RUN("objective", 2, launch_objective(w.r, h->Hs, w.fpart, w.L_final, p, d, st));
+    const bool want_final = stats && stats->L_final;
+    const bool want_host0 = stats && stats->L_host && o.max_iters == 0;
+    if (want_final || want_host0) {
+        RUN("hr_full", 1, launch_hr_full(w.r, h->Hs, w.Hr, p, d, st));
+        RUN("grad", 1, launch_grad(la.Q, la.Z, w.r, w.Hr, nullptr, w.L_final, p, d, g, st));
+        if (want_host0)
+            CK(cudaMemcpyAsync(w.L_host, w.L_final, p * sizeof(double), cudaMemcpyDeviceToDevice, st));
+    }
     if (la.hS) CK(cudaMemcpyAsync(S, la.S, (size_t)p * G * sizeof(float), cudaMemcpyDeviceToHost, st));
     if (la.hQ) CK(cudaMemcpyAsync(Q, la.Q, (size_t)p * d, cudaMemcpyDeviceToHost, st));
     if (stats) {

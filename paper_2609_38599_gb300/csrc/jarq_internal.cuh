@@ -24,14 +24,13 @@ constexpr int kSplitK = 4;         // split-K factor of the phase residual produ
 // Library-owned refinement workspace, sized for `cap_rows` output rows.
 struct Workspace {
     int cap_rows = 0;
-    float *P = nullptr;          // [p][d]  P = W H (target projection)
+    float *Hr = nullptr;         // [p][d]  H r for every row (start of an iteration)
     float *r = nullptr;          // [p][d]  residual r = w - D_s (q - z)
     float *gram = nullptr;       // [p][G][G]
-    float *rhs = nullptr;        // [p][G]
+    float *gvec = nullptr;       // [p][G]  scale gradient g_i = c_i^T (H r)_i
     float *hr = nullptr;         // [kSplitK][p][g]  split-K partials of (H r)_i
-    double *fpart = nullptr;     // [p][ceil(d/128)] objective partials
-    double *wHw = nullptr;       // [p]
-    double *L_prev = nullptr;    // [p]  L^{(k-1)} (Gram form, stop denominator)
+    double *F_start = nullptr;   // [p]  objective at the start of the iteration
+    double *L_prev = nullptr;    // [p]  L^{(k-1)} (stop denominator)
     double *dF_sweep = nullptr;  // [p]  sum of accepted Babai dF in the current sweep
     double *L_host = nullptr;    // [p]
     double *L_final = nullptr;   // [p]
@@ -72,15 +71,14 @@ cudaError_t launch_validate(const uint8_t *Q, const int32_t *Z, int p, int d, in
                             int *status, cudaStream_t s);
 cudaError_t launch_residual(const float *W, const float *S, const uint8_t *Q, const int32_t *Z,
                             float *r, int p, int d, int g, cudaStream_t s);
-cudaError_t launch_hw(const float *W, const float *Hs, float *P, double *wHw, int p, int d,
-                      cudaStream_t s);
-cudaError_t launch_objective(const float *r, const float *Hs, double *fpart, double *F, int p,
-                             int d, cudaStream_t s);
-cudaError_t launch_gram(const uint8_t *Q, const int32_t *Z, const float *Hs, const float *P,
-                        const int *active, float *gram, float *rhs, int p, int d, int g,
-                        cudaStream_t s);
-cudaError_t launch_scale_solve(const float *gram, const float *rhs, const float *W,
-                               const uint8_t *Q, const int32_t *Z, const double *wHw, float *S,
+cudaError_t launch_hr_full(const float *r, const float *Hs, float *Hr, int p, int d,
+                          cudaStream_t s);
+cudaError_t launch_grad(const uint8_t *Q, const int32_t *Z, const float *r, const float *Hr,
+                        float *gvec, double *F, int p, int d, int g, cudaStream_t s);
+cudaError_t launch_gram(const uint8_t *Q, const int32_t *Z, const float *Hs, const int *active,
+                        float *gram, int p, int d, int g, cudaStream_t s);
+cudaError_t launch_scale_solve(const float *gram, const float *gvec, const float *W,
+                               const uint8_t *Q, const int32_t *Z, const double *F_start, float *S,
                                float *r, double *L_prev, double *dF_sweep, int *active,
                                int *iters, int *ridge, int *rstat, int *status, int p, int d,
                                int g, int k, const jarq_options &o, cudaStream_t s);

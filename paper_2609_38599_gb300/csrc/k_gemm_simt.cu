@@ -1,13 +1,16 @@
 // CUDA-core contractions of the refinement path (float32, register tiled).
 //
-// All four products read the symmetrised Hessian H (ldb = d) as the right
+// All products read the symmetrised Hessian H (ldb = d) as the right
 // operand with a 64 x 128 output tile per block:
-//   hw        P = W H and wHw_j = w_j^T P_j       (App. G.7 target projection)
-//   gram      Gram_j[i,h] = c_i^T H_ih c_h, rhs_j[i] = c_i^T P_j[grp i]
-//             (Sec. 3.3.1, Eqs. scale_design / scale_normal_equations)
+//   hr_full   H r_j for every row (objective of Eq. bbmils_columns and the
+//             scale gradient g_j[i] = c_i^T (H r_j)_i, i.e. the right-hand side
+//             of the normal equations of Eq. scale_normal_equations written
+//             for the increment of the scales)
+//   gram      Gram_j[i,h] = c_i^T H_ih c_h      (Sec. 3.3.1, Eq. scale_design)
 //   phase_hr  (H r_j)_i for one group i, split over K  (Eq. conditional_residual)
-//   objective F_j = r_j^T H r_j                    (Eq. bbmils_columns)
-// Long K loops accumulate in 128-term chunks to bound float32 error growth.
+// The residual r = w - D_s (q - z) enters directly (no W H - H What
+// cancellation).  Long K loops accumulate in 128-term chunks to bound float32
+// error growth.
 #include "jarq_internal.cuh"
 
 namespace jarq {
@@ -130,14 +133,15 @@ __device__ __forceinline__ bool tile_has_active(const int *active, int p, int ro
     return __syncthreads_or(mine) != 0;
 }
 
-__global__ void __launch_bounds__(NT) hw_kernel(const float *__restrict__ W,
-                                                const float *__restrict__ Hs,
-                                                float *__restrict__ P, int p, int d) {
+// C = A H for a float32 row-major A [p][d] (used with A = r).
+__global__ void __launch_bounds__(NT) product_kernel(const float *__restrict__ A,
+                                                     const float *__restrict__ Hs,
+                                                     float *__restrict__ C, int p, int d) {
     __shared__ SmemTile sm;
     const int row0 = blockIdx.x * BM, n0 = blockIdx.y * BN;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
     float tot[4][8];
-    long_product(tot, DenseA{W, d}, p, row0, Hs, d, n0, d, 0, d, sm);
+    long_product(tot, DenseA{A, d}, p, row0, Hs, d, n0, d, 0, d, sm);
 #pragma unroll
     for (int x = 0; x < 4; ++x) {
         int j = row0 + ty * 4 + x;
@@ -145,55 +149,36 @@ __global__ void __launch_bounds__(NT) hw_kernel(const float *__restrict__ W,
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
             int col = n0 + col_of(tx, e);
-            if (col < d) P[(size_t)j * d + col] = tot[x][e];
+            if (col < d) C[(size_t)j * d + col] = tot[x][e];
         }
     }
 }
 
-// wHw_j = w_j . P_j in float64, one warp per row.
-__global__ void rowdot_kernel(const float *__restrict__ A, const float *__restrict__ B,
-                              double *__restrict__ out, int p, int d) {
+// Per row (one warp): F_j = r_j . (H r_j) in float64 and the scale gradient
+// g_j[i] = c_i . (H r_j)_i, c = q - z.
+__global__ void grad_kernel(const uint8_t *__restrict__ Q, const int32_t *__restrict__ Z,
+                            const float *__restrict__ r, const float *__restrict__ Hr,
+                            float *__restrict__ gvec, double *__restrict__ F, int p, int d,
+                            int g) {
     const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
     if (warp >= p) return;
-    double acc = 0.0;
-    for (int k = lane; k < d; k += 32)
-        acc += (double)A[(size_t)warp * d + k] * (double)B[(size_t)warp * d + k];
-    for (int o = 16; o; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    if (lane == 0) out[warp] = acc;
-}
-
-__global__ void __launch_bounds__(NT) objective_kernel(const float *__restrict__ r,
-                                                       const float *__restrict__ Hs,
-                                                       double *__restrict__ fpart, int p, int d) {
-    __shared__ SmemTile sm;
-    const int row0 = blockIdx.x * BM, n0 = blockIdx.y * BN;
-    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
-    float tot[4][8];
-    long_product(tot, DenseA{r, d}, p, row0, Hs, d, n0, d, 0, d, sm);
-    const int ntile = gridDim.y;
-#pragma unroll
-    for (int x = 0; x < 4; ++x) {
-        int j = row0 + ty * 4 + x;
-        float part = 0.f;
-        if (j < p) {
-#pragma unroll
-            for (int e = 0; e < 8; ++e) {
-                int col = n0 + col_of(tx, e);
-                if (col < d) part = fmaf(r[(size_t)j * d + col], tot[x][e], part);
-            }
+    const int G = d / g;
+    const size_t off = (size_t)warp * d;
+    double fs = 0.0;
+    for (int i = 0; i < G; ++i) {
+        double gi = 0.0;
+        const int z = Z[(size_t)warp * G + i];
+        for (int m = lane; m < g; m += 32) {
+            const size_t idx = off + (size_t)i * g + m;
+            const double hv = (double)Hr[idx];
+            gi += (double)((int)Q[idx] - z) * hv;
+            fs += (double)r[idx] * hv;
         }
-        part = reduce16(part);
-        if (tx == 0 && j < p) fpart[(size_t)j * ntile + blockIdx.y] = (double)part;
+        for (int o = 16; o; o >>= 1) gi += __shfl_xor_sync(0xffffffffu, gi, o);
+        if (lane == 0 && gvec) gvec[(size_t)warp * G + i] = (float)gi;
     }
-}
-
-__global__ void sum_parts_kernel(const double *__restrict__ fpart, double *__restrict__ F, int p,
-                                 int nt) {
-    int j = blockIdx.x * blockDim.x + threadIdx.x;
-    if (j >= p) return;
-    double s = 0.0;
-    for (int t = 0; t < nt; ++t) s += fpart[(size_t)j * nt + t];
-    F[j] = s;
+    for (int o = 16; o; o >>= 1) fs += __shfl_xor_sync(0xffffffffu, fs, o);
+    if (lane == 0) F[warp] = fs;
 }
 
 __global__ void __launch_bounds__(NT) phase_hr_kernel(const float *__restrict__ r,
@@ -227,10 +212,8 @@ __global__ void __launch_bounds__(NT) phase_hr_kernel(const float *__restrict__ 
 __global__ void __launch_bounds__(NT) gram_kernel(const uint8_t *__restrict__ Q,
                                                   const int32_t *__restrict__ Z,
                                                   const float *__restrict__ Hs,
-                                                  const float *__restrict__ P,
                                                   const int *__restrict__ active,
-                                                  float *__restrict__ gram,
-                                                  float *__restrict__ rhs, int p, int d, int g) {
+                                                  float *__restrict__ gram, int p, int d, int g) {
     __shared__ SmemTile sm;
     __shared__ float Ci[BM][BN + 4];
     const int G = d / g;
@@ -243,21 +226,6 @@ __global__ void __launch_bounds__(NT) gram_kernel(const uint8_t *__restrict__ Q,
         Ci[row][m] = (j < p && m < g) ? code(j, i * g + m) : 0.f;
     }
     __syncthreads();
-    // rhs_j[i] = c_i^T P_j[grp i]
-#pragma unroll
-    for (int x = 0; x < 4; ++x) {
-        int row = ty * 4 + x, j = row0 + row;
-        float part = 0.f;
-        if (j < p) {
-#pragma unroll
-            for (int e = 0; e < 8; ++e) {
-                int m = col_of(tx, e);
-                if (m < g) part = fmaf(Ci[row][m], P[(size_t)j * d + i * g + m], part);
-            }
-        }
-        part = reduce16(part);
-        if (tx == 0 && j < p) rhs[(size_t)j * G + i] = part;
-    }
     for (int h = 0; h < G; ++h) {
         float acc[4][8];
 #pragma unroll
@@ -280,24 +248,16 @@ __global__ void __launch_bounds__(NT) gram_kernel(const uint8_t *__restrict__ Q,
 
 }  // namespace
 
-cudaError_t launch_hw(const float *W, const float *Hs, float *P, double *wHw, int p, int d,
-                      cudaStream_t s) {
+cudaError_t launch_hr_full(const float *r, const float *Hs, float *Hr, int p, int d,
+                          cudaStream_t s) {
     dim3 grid((p + BM - 1) / BM, (d + BN - 1) / BN);
-    hw_kernel<<<grid, NT, 0, s>>>(W, Hs, P, p, d);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    rowdot_kernel<<<(p * 32 + 255) / 256, 256, 0, s>>>(W, P, wHw, p, d);
+    product_kernel<<<grid, NT, 0, s>>>(r, Hs, Hr, p, d);
     return cudaGetLastError();
 }
 
-cudaError_t launch_objective(const float *r, const float *Hs, double *fpart, double *F, int p,
-                             int d, cudaStream_t s) {
-    const int nt = (d + BN - 1) / BN;
-    dim3 grid((p + BM - 1) / BM, nt);
-    objective_kernel<<<grid, NT, 0, s>>>(r, Hs, fpart, p, d);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    sum_parts_kernel<<<(p + 255) / 256, 256, 0, s>>>(fpart, F, p, nt);
+cudaError_t launch_grad(const uint8_t *Q, const int32_t *Z, const float *r, const float *Hr,
+                        float *gvec, double *F, int p, int d, int g, cudaStream_t s) {
+    grad_kernel<<<(p * 32 + 255) / 256, 256, 0, s>>>(Q, Z, r, Hr, gvec, F, p, d, g);
     return cudaGetLastError();
 }
 
@@ -308,11 +268,10 @@ cudaError_t launch_phase_hr(const float *r, const float *Hs, const int *active, 
     return cudaGetLastError();
 }
 
-cudaError_t launch_gram(const uint8_t *Q, const int32_t *Z, const float *Hs, const float *P,
-                        const int *active, float *gram, float *rhs, int p, int d, int g,
-                        cudaStream_t s) {
+cudaError_t launch_gram(const uint8_t *Q, const int32_t *Z, const float *Hs, const int *active,
+                        float *gram, int p, int d, int g, cudaStream_t s) {
     dim3 grid((p + BM - 1) / BM, d / g);
-    gram_kernel<<<grid, NT, 0, s>>>(Q, Z, Hs, P, active, gram, rhs, p, d, g);
+    gram_kernel<<<grid, NT, 0, s>>>(Q, Z, Hs, active, gram, p, d, g);
     return cudaGetLastError();
 }
 

@@ -6,13 +6,18 @@
 //     FP32).  A pivot at or below rcond * max(max diag, eps), a nonfinite
 //     entry or a failed factorisation adds ridge * I and retries once; a
 //     second failure marks the row numerical and keeps its state;
-//  3. solves for s_j^{(k)} and writes it;
-//  4. updates the bookkeeping for the early stop of Eq. strict_stopping.
-//     With delta = s_new - s_old the change of the objective at fixed codes
-//     is dF_scale = -2 delta^T (rhs - Gram s_old) + delta^T Gram delta, so
-//     L^{(k-1)} - L^{(k)} = -(sum of accepted Babai dF of sweep k-1) - dF_scale
-//     is formed from small terms only.  |L^{(k-1)}| in the relative test is
-//     w^T H w - 2 s^T rhs + s^T Gram s;
+//  3. solves the normal equations of Eq. scale_normal_equations for the
+//     increment of the scales: with rhs = B^T y and the gradient
+//     g = rhs - Gram s_old, whose entries are g_i = c_i^T (H r)_i at the
+//     current state, Gram s_new = rhs  <=>  Gram (s_new - s_old) = g.  With the
+//     ridge, (Gram + lambda I) s_new = rhs  <=>  (Gram + lambda I) delta =
+//     g - lambda s_old.  g comes from a direct product with the residual, so
+//     the solve's rounding only touches the (small) increment;
+//  4. updates the bookkeeping for the early stop of Eq. strict_stopping:
+//     the objective change at fixed codes is
+//     dF_scale = -2 delta^T g + delta^T Gram delta, L^{(k)} = F(s_old) + dF_scale,
+//     and L^{(k-1)} - L^{(k)} = -(accepted Babai dF of sweep k-1) - dF_scale
+//     is formed from small terms only;
 //  5. rewrites the row's residual r = w - D_s (q - z) for the new scales.
 #include <float.h>
 
@@ -55,10 +60,10 @@ __device__ __forceinline__ float warp_max(float v) {
 }
 
 struct SolveArgs {
-    const float *gram, *rhs, *W;
+    const float *gram, *gvec, *W;
     const uint8_t *Q;
     const int32_t *Z;
-    const double *wHw;
+    const double *F_start;
     float *S, *r;
     double *L_prev, *dF_sweep;
     int *active, *iters, *ridge, *rstat, *status;
@@ -73,9 +78,9 @@ __global__ void scale_solve_kernel(SolveArgs a) {
     const int j = blockIdx.x * wpb + w;
     if (j >= a.p || !a.active[j]) return;  // warp-uniform
     float *A = smem + (size_t)w * (G * ld + 4 * G);
-    float *b = A + G * ld;       // rhs
+    float *b = A + G * ld;       // gradient g
     float *so = b + G;           // s_old
-    float *y = so + G;           // work vector, then s_new
+    float *y = so + G;           // right-hand side, then the increment
     const float *gj = a.gram + (size_t)j * G * G;
     auto load_sym = [&](float shift) -> bool {
         bool finite = true;
@@ -90,7 +95,7 @@ __global__ void scale_solve_kernel(SolveArgs a) {
         return __all_sync(0xffffffffu, finite);
     };
     for (int t = lane; t < G; t += 32) {
-        b[t] = a.rhs[(size_t)j * G + t];
+        b[t] = a.gvec[(size_t)j * G + t];
         so[t] = a.S[(size_t)j * G + t];
     }
     bool finite = load_sym(0.f);
@@ -117,8 +122,9 @@ __global__ void scale_solve_kernel(SolveArgs a) {
         }
         return;
     }
-    // forward: L y = rhs
-    for (int t = lane; t < G; t += 32) y[t] = b[t];
+    // forward: L y = g - lambda s_old
+    const float lam = used_ridge ? a.o.ridge : 0.f;
+    for (int t = lane; t < G; t += 32) y[t] = fmaf(-lam, so[t], b[t]);
     for (int k = 0; k < G; ++k) {
         __syncwarp();
         const float yk = y[k] / A[k * ld + k];
@@ -147,33 +153,27 @@ __global__ void scale_solve_kernel(SolveArgs a) {
         return;
     }
     // objective bookkeeping with the unridged symmetrised Gram matrix
-    double t1 = 0.0, t2 = 0.0, ls = 0.0, lq = 0.0;
+    double t1 = 0.0, t2 = 0.0;
     for (int r0 = lane; r0 < G; r0 += 32) {
-        float gso = 0.f, gdl = 0.f, gsn = 0.f;
-        for (int c0 = 0; c0 < G; ++c0) {
-            float gm = 0.5f * (gj[r0 * G + c0] + gj[c0 * G + r0]);
-            gso = fmaf(gm, so[c0], gso);
-            gdl = fmaf(gm, y[c0] - so[c0], gdl);
-            gsn = fmaf(gm, y[c0], gsn);
-        }
-        const double dl = (double)y[r0] - (double)so[r0];
-        t1 += dl * ((double)b[r0] - (double)gso);
-        t2 += dl * (double)gdl;
-        ls += (double)y[r0] * (double)b[r0];
-        lq += (double)y[r0] * (double)gsn;
+        float gdl = 0.f;
+        for (int c0 = 0; c0 < G; ++c0)
+            gdl = fmaf(0.5f * (gj[r0 * G + c0] + gj[c0 * G + r0]), y[c0], gdl);
+        t1 += (double)y[r0] * (double)b[r0];
+        t2 += (double)y[r0] * (double)gdl;
     }
     t1 = warp_sum(t1);
     t2 = warp_sum(t2);
-    ls = warp_sum(ls);
-    lq = warp_sum(lq);
     const double dF_scale = -2.0 * t1 + t2;
-    const double L_new = a.wHw[j] - 2.0 * ls + lq;
+    const double L_new = a.F_start[j] + dF_scale;
     bool stop = false;
     if (a.o.early_stop && a.k >= 2) {
         const double dec = -(a.dF_sweep[j] + dF_scale);
         const double den = fmax(fabs(a.L_prev[j]), (double)a.o.eps);
         stop = (dec / den <= (double)a.o.tau_rel) || (fabs(dec) <= (double)a.o.tau_abs);
     }
+    __syncwarp();
+    for (int t = lane; t < G; t += 32) y[t] = so[t] + y[t];   // s_new = s_old + delta
+    __syncwarp();
     for (int t = lane; t < G; t += 32) a.S[(size_t)j * G + t] = y[t];
     if (lane == 0) {
         a.L_prev[j] = L_new;
@@ -194,8 +194,8 @@ __global__ void scale_solve_kernel(SolveArgs a) {
 
 }  // namespace
 
-cudaError_t launch_scale_solve(const float *gram, const float *rhs, const float *W,
-                               const uint8_t *Q, const int32_t *Z, const double *wHw, float *S,
+cudaError_t launch_scale_solve(const float *gram, const float *gvec, const float *W,
+                               const uint8_t *Q, const int32_t *Z, const double *F_start, float *S,
                                float *r, double *L_prev, double *dF_sweep, int *active,
                                int *iters, int *ridge, int *rstat, int *status, int p, int d,
                                int g, int k, const jarq_options &o, cudaStream_t s) {
@@ -208,7 +208,7 @@ cudaError_t launch_scale_solve(const float *gram, const float *rhs, const float 
     cudaError_t e = cudaFuncSetAttribute(scale_solve_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    SolveArgs a{gram, rhs, W, Q, Z, wHw, S, r, L_prev, dF_sweep, active, iters, ridge, rstat,
+    SolveArgs a{gram, gvec, W, Q, Z, F_start, S, r, L_prev, dF_sweep, active, iters, ridge, rstat,
                 status, p, d, g, k, o};
     scale_solve_kernel<<<(p + wpb - 1) / wpb, 32 * wpb, smem, s>>>(a);
     return cudaGetLastError();

@@ -8,8 +8,8 @@
 namespace jarq {
 namespace {
 
-const char *const kNames[] = {"validate", "residual", "init_rows", "hw", "gram", "scale_solve",
-                              "phase_hr", "babai", "objective", "symmetrize", "group_factor"};
+const char *const kNames[] = {"validate", "residual", "init_rows", "hr_full", "grad", "gram",
+                              "scale_solve", "phase_hr", "babai", "symmetrize", "group_factor"};
 constexpr int kNumNames = sizeof(kNames) / sizeof(kNames[0]);
 
 struct Pending {

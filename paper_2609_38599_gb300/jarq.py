@@ -94,8 +94,8 @@ def library():
     return _lib
 
 
-KERNELS = ("validate", "residual", "init_rows", "hw", "gram", "scale_solve", "phase_hr",
-           "babai", "objective", "symmetrize", "group_factor")
+KERNELS = ("validate", "residual", "init_rows", "hr_full", "grad", "gram", "scale_solve",
+           "phase_hr", "babai", "symmetrize", "group_factor")
 
 
 def profile_enable(on: bool = True):
