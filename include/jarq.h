@@ -98,8 +98,10 @@ jarq_options jarq_default_options(void);
 /* Prepare a Hessian for refinement (Sec. 3.3.2, Eq. group_qr; App. G.7
  * "Shared preprocessing").
  *   H          : float32 [din][din], host or device; symmetrised as (H+H^T)/2.
- *   din        : input width, > 0, multiple of group_size.
- *   group_size : g, 1 <= g <= 128.
+ *   din        : input width, > 0, multiple of group_size, at most
+ *                128 groups.
+ *   group_size : g, 64 or 128 (the paper's group sizes that fit the
+ *                tensor-core tiles and the Babai kernel's shared memory).
  *   nu2        : added to the diagonal (the paper's nu^2, Eq. strict_target);
  *                pass 0 when H already contains its damping.
  *   out        : receives the new handle (unchanged on error).
@@ -151,7 +153,7 @@ const char *jarq_status_string(jarq_status s);
  * kernel launch it makes; durations are accumulated per kernel name when the
  * enclosing call synchronises.  Names: "validate", "residual", "init_rows",
  * "hr_full", "grad", "gram", "scale_solve", "phase_hr", "babai",
- * "symmetrize", "group_factor".  Not thread-safe. */
+ * "symmetrize", "group_factor", "slices".  Not thread-safe. */
 void jarq_profile_enable(int on);
 void jarq_profile_reset(void);
 /* Accumulated launches and total device milliseconds of one kernel name since

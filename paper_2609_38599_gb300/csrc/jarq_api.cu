@@ -47,6 +47,45 @@ cudaError_t dalloc(T **p, size_t n) {
     return cudaMalloc((void **)p, n * sizeof(T));
 }
 
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                  const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                  const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+// 2D bf16 tensor map over [rows][cols] (pitch = cols), box_rows x 64 boxes,
+// 128-byte swizzle, out-of-range elements read as zero.
+cudaError_t make_tmap_bf16(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols,
+                           uint32_t box_rows) {
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void *ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
+                                                         cudaEnableDefault, &q);
+        if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !ptr)
+            return e != cudaSuccess ? e : cudaErrorSymbolNotFound;
+        fn = (EncodeTiledFn)ptr;
+    }
+    cuuint64_t dims[2] = {cols, rows};
+    cuuint64_t strides[1] = {cols * 2};
+    cuuint32_t box[2] = {64, box_rows};
+    cuuint32_t es[2] = {1, 1};
+    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides,
+                    box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+// Split-K factor of the phase product: enough CTAs to cover the SMs.
+int phase_splits(int p_pad, int d_pad) {
+    const int tiles = p_pad / 128, chunks = d_pad / 64;
+    int n = num_sms() / tiles;
+    if (n < 1) n = 1;
+    if (n > kMaxSplit) n = kMaxSplit;
+    if (n > chunks) n = chunks;
+    return n;
+}
+
 bool is_device_ptr(const void *ptr) {
     cudaPointerAttributes at;
     if (cudaPointerGetAttributes(&at, ptr) != cudaSuccess) {
@@ -76,6 +115,8 @@ void free_ws(Workspace &w) {
     cudaFree(w.sS);
     cudaFree(w.sQ);
     cudaFree(w.sZ);
+    cudaFree(w.rplanes);
+    cudaFree(w.cplane);
     w = Workspace{};
 }
 
@@ -84,12 +125,22 @@ cudaError_t ensure_ws(jarq_hessian *h, int p) {
     if (p <= w.cap_rows) return cudaSuccess;
     free_ws(w);
     const size_t d = h->din, G = h->G, g = h->g;
+    const int p_pad = round_up(p, 128);
     cudaError_t e;
+    if ((e = dalloc(&w.rplanes, (size_t)3 * p_pad * h->d_pad)) != cudaSuccess) return e;
+    if ((e = cudaMemset(w.rplanes, 0, (size_t)3 * p_pad * h->d_pad * 2)) != cudaSuccess) return e;
+    if ((e = make_tmap_bf16(&w.mapR, w.rplanes, (uint64_t)3 * p_pad, h->d_pad, 128)) != cudaSuccess)
+        return e;
+    if ((e = dalloc(&w.cplane, (size_t)p_pad * h->d_pad)) != cudaSuccess) return e;
+    if ((e = cudaMemset(w.cplane, 0, (size_t)p_pad * h->d_pad * 2)) != cudaSuccess) return e;
+    if ((e = make_tmap_bf16(&w.mapC, w.cplane, (uint64_t)p_pad, h->d_pad, 128)) != cudaSuccess)
+        return e;
+    w.p_pad = p_pad;
     if ((e = dalloc(&w.Hr, (size_t)p * d)) != cudaSuccess) return e;
     if ((e = dalloc(&w.r, (size_t)p * d)) != cudaSuccess) return e;
     if ((e = dalloc(&w.gram, (size_t)p * G * G)) != cudaSuccess) return e;
     if ((e = dalloc(&w.gvec, (size_t)p * G)) != cudaSuccess) return e;
-    if ((e = dalloc(&w.hr, (size_t)kSplitK * p * g)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.hr, (size_t)kMaxSplit * p_pad * g)) != cudaSuccess) return e;
     if ((e = dalloc(&w.F_start, (size_t)p)) != cudaSuccess) return e;
     if ((e = dalloc(&w.L_prev, (size_t)p)) != cudaSuccess) return e;
     if ((e = dalloc(&w.dF_sweep, (size_t)p)) != cudaSuccess) return e;
@@ -166,6 +217,7 @@ cudaError_t stage_layer(jarq_hessian *h, const float *W, const float *S, const u
 jarq_status status_from_bits(int bits) {
     if (bits & ST_NOT_SPD) return JARQ_ERR_NOT_SPD;
     if (bits & (ST_BAD_CODE | ST_BAD_ZERO)) return JARQ_ERR_ARG;
+    if (bits & ST_TIMEOUT) return JARQ_ERR_TIMEOUT;
     if (bits & ST_NUMERICAL) return JARQ_ERR_NUMERICAL;
     return JARQ_OK;
 }
@@ -176,6 +228,10 @@ cudaError_t read_status(jarq_hessian *h, cudaStream_t st, int *bits) {
     *bits = (e == cudaSuccess) ? *h->hstatus : 0;
     if (e == cudaSuccess) prof_collect();
     return e;
+}
+
+ResidualView rview(jarq_hessian *h) {
+    return ResidualView{h->ws.r, h->ws.rplanes, h->ws.cplane, h->din, h->d_pad, h->ws.p_pad};
 }
 
 // Common front half of refine/objective: stage, validate, residual.
@@ -189,7 +245,7 @@ jarq_status layer_front(jarq_hessian *h, const float *W, const float *S, const u
     int sb = 0;
     CK(read_status(h, st, &sb));
     if (sb) return status_from_bits(sb);
-    RUN("residual", 1, launch_residual(la.W, la.S, la.Q, la.Z, h->ws.r, dout, h->din, h->g, st));
+    RUN("residual", 1, launch_residual(la.W, la.S, la.Q, la.Z, rview(h), dout, h->g, st));
     return JARQ_OK;
 }
 
@@ -238,6 +294,9 @@ void jarq_hessian_destroy(jarq_hessian *h) {
     cudaDeviceSynchronize();
     free_ws(h->ws);
     cudaFree(h->Hs);
+    cudaFree(h->Hplanes);
+    cudaFree(h->Hdigits);
+    cudaFree(h->expo);
     cudaFree(h->Lf);
     cudaFree(h->Rinv);
     cudaFree(h->dstatus);
@@ -248,7 +307,7 @@ void jarq_hessian_destroy(jarq_hessian *h) {
 
 jarq_status jarq_prepare_hessian(const float *H, int din, int group_size, float nu2,
                                  jarq_hessian **out, void *stream) {
-    if (!H || !out || din <= 0 || group_size < 1 || group_size > kMaxGroup ||
+    if (!H || !out || din <= 0 || (group_size != 64 && group_size != 128) ||
         din % group_size != 0 || din / group_size > kMaxGroups || !isfinite(nu2))
         return JARQ_ERR_ARG;
     cudaStream_t st = (cudaStream_t)stream;
@@ -257,6 +316,7 @@ jarq_status jarq_prepare_hessian(const float *H, int din, int group_size, float 
     h->din = din;
     h->g = group_size;
     h->G = din / group_size;
+    h->d_pad = round_up(din, 128);
     jarq_status rc = JARQ_OK;
     float *Hdev = nullptr;
     do {
@@ -264,6 +324,15 @@ jarq_status jarq_prepare_hessian(const float *H, int din, int group_size, float 
         const size_t dd = (size_t)din * din;
         cudaError_t e;
         if ((e = dalloc(&h->Hs, dd)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        const size_t pd = (size_t)h->d_pad * h->d_pad;
+        if ((e = dalloc(&h->Hplanes, 3 * pd)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = cudaMemsetAsync(h->Hplanes, 0, 3 * pd * 2, st)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = make_tmap_bf16(&h->mapH128, h->Hplanes, (uint64_t)3 * h->d_pad, h->d_pad, 128)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = make_tmap_bf16(&h->mapH64, h->Hplanes, (uint64_t)3 * h->d_pad, h->d_pad, 64)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = dalloc(&h->Hdigits, 4 * pd)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = cudaMemsetAsync(h->Hdigits, 0, 4 * pd * 2, st)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = dalloc(&h->expo, (size_t)h->G * h->G)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = make_tmap_bf16(&h->mapD, h->Hdigits, (uint64_t)4 * h->d_pad, h->d_pad, 64)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->Lf, (size_t)h->G * group_size * group_size)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->Rinv, (size_t)h->G * group_size * group_size)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->dstatus, 1)) != cudaSuccess) { rc = cuda_fail(e); break; }
@@ -275,9 +344,11 @@ jarq_status jarq_prepare_hessian(const float *H, int din, int group_size, float 
             Hsrc = Hdev;
         }
         if ((e = cudaMemsetAsync(h->dstatus, 0, sizeof(int), st)) != cudaSuccess) { rc = cuda_fail(e); break; }
-        { ProfScope ps("symmetrize", st); e = launch_symmetrize(Hsrc, h->Hs, din, nu2, st); ps.done(); count_launches(1); }
+        { ProfScope ps("symmetrize", st); e = launch_symmetrize(Hsrc, h->Hs, h->Hplanes, din, h->d_pad, nu2, st); ps.done(); count_launches(1); }
         if (e != cudaSuccess) { rc = cuda_fail(e); break; }
         { ProfScope ps("group_factor", st); e = launch_group_factor(h->Hs, h->Lf, h->Rinv, din, group_size, h->dstatus, st); ps.done(); count_launches(1); }
+        if (e != cudaSuccess) { rc = cuda_fail(e); break; }
+        { ProfScope ps("slices", st); e = launch_slices(h->Hs, h->expo, h->Hdigits, din, h->d_pad, group_size, st); ps.done(); count_launches(2); }
         if (e != cudaSuccess) { rc = cuda_fail(e); break; }
         int sb = 0;
         if ((e = read_status(h, st, &sb)) != cudaSuccess) { rc = cuda_fail(e); break; }
@@ -306,12 +377,13 @@ jarq_status jarq_objective(jarq_hessian *h, const float *W, const float *S, cons
     jarq_status rc = layer_front(h, W, S, Q, Z, dout, bits, la, st);
     if (rc != JARQ_OK) return rc;
     Workspace &w = h->ws;
-    RUN("hr_full", 1, launch_hr_full(w.r, h->Hs, w.Hr, dout, h->din, st));
+    CK(cudaMemsetAsync(h->dstatus, 0, sizeof(int), st));
+    RUN("hr_full", 1, launch_tc_hr_full(w.mapR, h->mapH128, w.Hr, h->din, dout, w.p_pad, h->din, h->d_pad, h->dstatus, st));
     RUN("grad", 1, launch_grad(la.Q, la.Z, w.r, w.Hr, nullptr, w.L_final, dout, h->din, h->g, st));
     CK(cudaMemcpyAsync(F_per_row, w.L_final, (size_t)dout * sizeof(double), cudaMemcpyDefault, st));
-    CK(cudaStreamSynchronize(st));
-    prof_collect();
-    return JARQ_OK;
+    int sb = 0;
+    CK(read_status(h, st, &sb));
+    return status_from_bits(sb);
 }
 
 jarq_status jarq_refine_layer(jarq_hessian *h, const float *W, float *S, uint8_t *Q,
@@ -329,25 +401,29 @@ jarq_status jarq_refine_layer(jarq_hessian *h, const float *W, float *S, uint8_t
     Workspace &w = h->ws;
     const int p = dout, d = h->din, g = h->g, G = h->G, qmax = (1 << bits) - 1;
     RUN("init_rows", 1, launch_init_rows(w.active, w.iters, w.accepted, w.ridge, w.rstat, w.dF_sweep, p, st));
+    const ResidualView rv = rview(h);
+    const int nsplit = phase_splits(w.p_pad, h->d_pad);
     for (int k = 1; k <= o.max_iters; ++k) {
-        RUN("hr_full", 1, launch_hr_full(w.r, h->Hs, w.Hr, p, d, st));
+        RUN("hr_full", 1, launch_tc_hr_full(w.mapR, h->mapH128, w.Hr, d, p, w.p_pad, d, h->d_pad, h->dstatus, st));
         RUN("grad", 1, launch_grad(la.Q, la.Z, w.r, w.Hr, w.gvec, w.F_start, p, d, g, st));
         if (k == 1 && stats && stats->L_host)
             CK(cudaMemcpyAsync(w.L_host, w.F_start, p * sizeof(double), cudaMemcpyDeviceToDevice, st));
-        RUN("gram", 1, launch_gram(la.Q, la.Z, h->Hs, w.active, w.gram, p, d, g, st));
-        RUN("scale_solve", 1, launch_scale_solve(w.gram, w.gvec, la.W, la.Q, la.Z, w.F_start, la.S, w.r,
+        RUN("gram", 1, launch_tc_gram(w.mapC, h->mapD, la.Q, la.Z, h->expo, w.active, w.gram, p,
+                                      w.p_pad, d, h->d_pad, g, bits, h->dstatus, st));
+        RUN("scale_solve", 1, launch_scale_solve(w.gram, w.gvec, la.W, la.Q, la.Z, w.F_start, la.S, rv,
                                                  w.L_prev, w.dF_sweep, w.active, w.iters, w.ridge, w.rstat,
                                                  h->dstatus, p, d, g, k, o, st));
         for (int i = 0; i < G; ++i) {
-            RUN("phase_hr", 1, launch_phase_hr(w.r, h->Hs, w.active, w.hr, p, d, g, i, st));
-            RUN("babai", 1, launch_babai(w.hr, h->Lf, h->Rinv, la.W, la.S, la.Q, la.Z, w.r, w.active,
-                                         w.dF_sweep, w.accepted, p, d, g, i, qmax, o.eps, st));
+            RUN("phase_hr", 1, launch_tc_hr_phase(w.mapR, h->mapH128, h->mapH64, w.hr, p, w.p_pad, h->d_pad,
+                                                  g, i, nsplit, w.active, h->dstatus, st));
+            RUN("babai", 1, launch_babai(w.hr, nsplit, h->Lf, h->Rinv, la.W, la.S, la.Q, la.Z, rv, w.active,
+                                         w.dF_sweep, w.accepted, p, g, i, qmax, o.eps, st));
         }
     }
     const bool want_final = stats && stats->L_final;
     const bool want_host0 = stats && stats->L_host && o.max_iters == 0;
     if (want_final || want_host0) {
-        RUN("hr_full", 1, launch_hr_full(w.r, h->Hs, w.Hr, p, d, st));
+        RUN("hr_full", 1, launch_tc_hr_full(w.mapR, h->mapH128, w.Hr, d, p, w.p_pad, d, h->d_pad, h->dstatus, st));
         RUN("grad", 1, launch_grad(la.Q, la.Z, w.r, w.Hr, nullptr, w.L_final, p, d, g, st));
         if (want_host0)
             CK(cudaMemcpyAsync(w.L_host, w.L_final, p * sizeof(double), cudaMemcpyDeviceToDevice, st));

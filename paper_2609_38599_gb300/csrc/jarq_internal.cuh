@@ -1,6 +1,7 @@
 // Internal declarations shared by the JARQ CUDA sources (not part of the ABI).
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 #include <stdint.h>
@@ -15,20 +16,62 @@ enum : int {
     ST_NUMERICAL = 2,    // a row's scale system failed even with the ridge
     ST_BAD_CODE = 4,     // a code is outside [0, 2^b - 1]
     ST_BAD_ZERO = 8,     // a zero point is outside [0, 2^b - 1]
+    ST_TIMEOUT = 16,     // a bounded device wait gave up
 };
 
-constexpr int kMaxGroup = 128;     // largest supported group size g
 constexpr int kMaxGroups = 128;    // largest supported G for the scale solve
-constexpr int kSplitK = 4;         // split-K factor of the phase residual product
+constexpr int kMaxSplit = 16;      // largest split-K factor of the phase product
+
+__host__ __device__ inline int round_up(int x, int m) { return (x + m - 1) / m * m; }
+
+// View of the residual r = w - D_s (q - z): float32 [p][d] plus its exact
+// three-plane bf16 split [3][p_pad][d_pad] read by the tensor cores, and the
+// integer codes c = q - z as bf16 [p_pad][d_pad] (exact for |c| <= 256).
+struct ResidualView {
+    float *r;
+    __nv_bfloat16 *planes;
+    __nv_bfloat16 *cplane;
+    int d, d_pad, p_pad;
+};
+
+// Exact split x = x1 + x2 + x3 of a float32 into bf16 values (truncation).
+__device__ __forceinline__ void split3(float x, __nv_bfloat16 &a, __nv_bfloat16 &b,
+                                       __nv_bfloat16 &c) {
+    const float x1 = __uint_as_float(__float_as_uint(x) & 0xFFFF0000u);
+    const float rem = x - x1;
+    const float x2 = __uint_as_float(__float_as_uint(rem) & 0xFFFF0000u);
+    a = __float2bfloat16_rz(x1);
+    b = __float2bfloat16_rz(x2);
+    c = __float2bfloat16_rn(rem - x2);
+}
+
+__device__ __forceinline__ void store_code(const ResidualView &v, size_t j, int col, int c) {
+    v.cplane[j * v.d_pad + col] = __int2bfloat16_rn(c);
+}
+
+__device__ __forceinline__ void store_residual(const ResidualView &v, size_t j, int col, float x) {
+    v.r[j * v.d + col] = x;
+    __nv_bfloat16 a, b, c;
+    split3(x, a, b, c);
+    const size_t plane = (size_t)v.p_pad * v.d_pad, off = j * v.d_pad + col;
+    v.planes[off] = a;
+    v.planes[plane + off] = b;
+    v.planes[2 * plane + off] = c;
+}
 
 // Library-owned refinement workspace, sized for `cap_rows` output rows.
 struct Workspace {
     int cap_rows = 0;
+    int p_pad = 0;               // rows of the bf16 residual planes (multiple of 128)
     float *Hr = nullptr;         // [p][d]  H r for every row (start of an iteration)
     float *r = nullptr;          // [p][d]  residual r = w - D_s (q - z)
-    float *gram = nullptr;       // [p][G][G]
-    float *gvec = nullptr;       // [p][G]  scale gradient g_i = c_i^T (H r)_i
-    float *hr = nullptr;         // [kSplitK][p][g]  split-K partials of (H r)_i
+    double *gram = nullptr;      // [p][G][G]  exact Gram matrices
+    double *gvec = nullptr;      // [p][G]  scale gradient g_i = c_i^T (H r)_i
+    float *hr = nullptr;         // [nsplit][p_pad][g]  split-K partials of (H r)_i
+    __nv_bfloat16 *rplanes = nullptr;  // [3][p_pad][d_pad] bf16 split of r
+    __nv_bfloat16 *cplane = nullptr;   // [p_pad][d_pad] codes c = q - z
+    CUtensorMap mapR;            // tensor map of rplanes, 128 x 64 boxes
+    CUtensorMap mapC;            // tensor map of cplane, 128 x 64 boxes
     double *F_start = nullptr;   // [p]  objective at the start of the iteration
     double *L_prev = nullptr;    // [p]  L^{(k-1)} (stop denominator)
     double *dF_sweep = nullptr;  // [p]  sum of accepted Babai dF in the current sweep
@@ -52,7 +95,13 @@ struct Workspace {
 struct jarq_hessian {
     int din = 0, g = 0, G = 0;
     int device = 0;
+    int d_pad = 0;
     float *Hs = nullptr;          // [d][d] symmetrised H (+ nu2 I), fp32
+    __nv_bfloat16 *Hplanes = nullptr;  // [3][d_pad][d_pad] exact bf16 split of Hs
+    __nv_bfloat16 *Hdigits = nullptr;  // [4][d_pad][d_pad] per-block integer digits of Hs
+    int *expo = nullptr;          // [G][G] block exponents of the digits
+    CUtensorMap mapH128, mapH64;  // tensor maps of Hplanes, 128 x 64 and 64 x 64 boxes
+    CUtensorMap mapD;             // tensor map of Hdigits, 64 x 64 boxes
     float *Lf = nullptr;          // [G][g][g] lower factor L_i = R_i^T, row-major
     float *Rinv = nullptr;        // [G][g][g] R_i^{-1} (upper), row-major
     int *dstatus = nullptr;       // device status word
@@ -63,31 +112,39 @@ struct jarq_hessian {
 namespace jarq {
 
 // ---- launchers (each returns the cudaError_t of its launch) ----
-cudaError_t launch_symmetrize(const float *H, float *Hs, int d, float nu2, cudaStream_t s);
+cudaError_t launch_symmetrize(const float *H, float *Hs, __nv_bfloat16 *Hplanes, int d, int d_pad,
+                              float nu2, cudaStream_t s);
 cudaError_t launch_group_factor(const float *Hs, float *Lf, float *Rinv, int d, int g,
                                 int *status, cudaStream_t s);
 
 cudaError_t launch_validate(const uint8_t *Q, const int32_t *Z, int p, int d, int G, int qmax,
                             int *status, cudaStream_t s);
 cudaError_t launch_residual(const float *W, const float *S, const uint8_t *Q, const int32_t *Z,
-                            float *r, int p, int d, int g, cudaStream_t s);
-cudaError_t launch_hr_full(const float *r, const float *Hs, float *Hr, int p, int d,
-                          cudaStream_t s);
+                            ResidualView rv, int p, int g, cudaStream_t s);
+cudaError_t launch_tc_hr_full(const CUtensorMap &mapA, const CUtensorMap &mapB, float *out,
+                              int ldo, int p, int p_pad, int d, int d_pad, int *status,
+                              cudaStream_t s);
+cudaError_t launch_tc_hr_phase(const CUtensorMap &mapA, const CUtensorMap &mapB128,
+                               const CUtensorMap &mapB64, float *out, int p, int p_pad, int d_pad,
+                               int g, int i, int nsplit, const int *active, int *status,
+                               cudaStream_t s);
 cudaError_t launch_grad(const uint8_t *Q, const int32_t *Z, const float *r, const float *Hr,
-                        float *gvec, double *F, int p, int d, int g, cudaStream_t s);
-cudaError_t launch_gram(const uint8_t *Q, const int32_t *Z, const float *Hs, const int *active,
-                        float *gram, int p, int d, int g, cudaStream_t s);
-cudaError_t launch_scale_solve(const float *gram, const float *gvec, const float *W,
+                        double *gvec, double *F, int p, int d, int g, cudaStream_t s);
+cudaError_t launch_slices(const float *Hs, int *expo, __nv_bfloat16 *planes, int d, int d_pad,
+                          int g, cudaStream_t s);
+cudaError_t launch_tc_gram(const CUtensorMap &mapC, const CUtensorMap &mapS, const uint8_t *Q,
+                           const int32_t *Z, const int *expo, const int *active, double *gram,
+                           int p, int p_pad, int d, int d_pad, int g, int bits, int *status,
+                           cudaStream_t s);
+cudaError_t launch_scale_solve(const double *gram, const double *gvec, const float *W,
                                const uint8_t *Q, const int32_t *Z, const double *F_start, float *S,
-                               float *r, double *L_prev, double *dF_sweep, int *active,
+                               ResidualView rv, double *L_prev, double *dF_sweep, int *active,
                                int *iters, int *ridge, int *rstat, int *status, int p, int d,
                                int g, int k, const jarq_options &o, cudaStream_t s);
-cudaError_t launch_phase_hr(const float *r, const float *Hs, const int *active, float *hr,
-                            int p, int d, int g, int i, cudaStream_t s);
-cudaError_t launch_babai(const float *hr, const float *Lf, const float *Rinv, const float *W,
-                         const float *S, uint8_t *Q, const int32_t *Z, float *r,
-                         const int *active, double *dF_sweep, int *accepted, int p, int d,
-                         int g, int i, int qmax, float eps, cudaStream_t s);
+cudaError_t launch_babai(const float *hr, int nsplit, const float *Lf, const float *Rinv,
+                         const float *W, const float *S, uint8_t *Q, const int32_t *Z,
+                         ResidualView rv, const int *active, double *dF_sweep, int *accepted,
+                         int p, int g, int i, int qmax, float eps, cudaStream_t s);
 cudaError_t launch_init_rows(int *active, int *iters, int *accepted, int *ridge, int *rstat,
                              double *dF_sweep, int p, cudaStream_t s);
 

@@ -25,15 +25,16 @@ __global__ void validate_kernel(const uint8_t *__restrict__ Q, const int32_t *__
 // r = w - s (q - z), one rounding (fma) per element (Eq. quantized_group).
 __global__ void residual_kernel(const float *__restrict__ W, const float *__restrict__ S,
                                 const uint8_t *__restrict__ Q, const int32_t *__restrict__ Z,
-                                float *__restrict__ r, int p, int d, int g) {
-    const int G = d / g;
+                                ResidualView rv, int p, int g) {
+    const int d = rv.d, G = d / g;
     const size_t n = (size_t)p * d;
     const size_t stride = (size_t)gridDim.x * blockDim.x;
     for (size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x; idx < n; idx += stride) {
         const size_t j = idx / d;
         const int grp = (int)(idx - j * d) / g;
-        const float c = (float)((int)Q[idx] - Z[j * G + grp]);
-        r[idx] = fmaf(-S[j * G + grp], c, W[idx]);
+        const int ci = (int)Q[idx] - Z[j * G + grp];
+        store_residual(rv, j, (int)(idx - j * d), fmaf(-S[j * G + grp], (float)ci, W[idx]));
+        store_code(rv, j, (int)(idx - j * d), ci);
     }
 }
 
@@ -74,12 +75,12 @@ cudaError_t launch_validate(const uint8_t *Q, const int32_t *Z, int p, int d, in
 }
 
 cudaError_t launch_residual(const float *W, const float *S, const uint8_t *Q, const int32_t *Z,
-                            float *r, int p, int d, int g, cudaStream_t s) {
-    size_t n = (size_t)p * d;
+                            ResidualView rv, int p, int g, cudaStream_t s) {
+    size_t n = (size_t)p * rv.d;
     int blocks = (int)((n + 255) / 256);
     if (blocks > 8 * num_sms()) blocks = 8 * num_sms();
     if (blocks < 1) blocks = 1;
-    residual_kernel<<<blocks, 256, 0, s>>>(W, S, Q, Z, r, p, d, g);
+    residual_kernel<<<blocks, 256, 0, s>>>(W, S, Q, Z, rv, p, g);
     return cudaGetLastError();
 }
 

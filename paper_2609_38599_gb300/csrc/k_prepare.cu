@@ -13,8 +13,10 @@
 namespace jarq {
 namespace {
 
-// out = (H + H^T)/2 + nu2 I, through 32x32 shared-memory tiles.
-__global__ void symmetrize_kernel(const float *__restrict__ H, float *__restrict__ Hs, int d,
+// out = (H + H^T)/2 + nu2 I, through 32x32 shared-memory tiles, plus its
+// exact three-plane bf16 split (planes [3][d_pad][d_pad], pitch d_pad).
+__global__ void symmetrize_kernel(const float *__restrict__ H, float *__restrict__ Hs,
+                                  __nv_bfloat16 *__restrict__ planes, int d, int d_pad,
                                   float nu2) {
     __shared__ float tile[32][33];
     const int bx = blockIdx.x * 32, by = blockIdx.y * 32;
@@ -30,6 +32,12 @@ __global__ void symmetrize_kernel(const float *__restrict__ H, float *__restrict
             float v = 0.5f * (H[(size_t)row * d + col] + tile[tx][yy]);
             if (row == col) v += nu2;
             Hs[(size_t)row * d + col] = v;
+            __nv_bfloat16 a, b, c;
+            split3(v, a, b, c);
+            const size_t plane = (size_t)d_pad * d_pad, off = (size_t)row * d_pad + col;
+            planes[off] = a;
+            planes[plane + off] = b;
+            planes[2 * plane + off] = c;
         }
     }
 }
@@ -109,9 +117,10 @@ __global__ void group_factor_kernel(const float *__restrict__ Hs, float *__restr
 
 }  // namespace
 
-cudaError_t launch_symmetrize(const float *H, float *Hs, int d, float nu2, cudaStream_t s) {
+cudaError_t launch_symmetrize(const float *H, float *Hs, __nv_bfloat16 *Hplanes, int d, int d_pad,
+                              float nu2, cudaStream_t s) {
     dim3 grid((d + 31) / 32, (d + 31) / 32), block(32, 8);
-    symmetrize_kernel<<<grid, block, 0, s>>>(H, Hs, d, nu2);
+    symmetrize_kernel<<<grid, block, 0, s>>>(H, Hs, Hplanes, d, d_pad, nu2);
     return cudaGetLastError();
 }
 

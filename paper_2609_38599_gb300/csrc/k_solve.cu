@@ -7,7 +7,9 @@
 //     entry or a failed factorisation adds ridge * I and retries once; a
 //     second failure marks the row numerical and keeps its state;
 //  3. solves the normal equations of Eq. scale_normal_equations for the
-//     increment of the scales: with rhs = B^T y and the gradient
+//     increment of the scales (float32 Cholesky, then two refinement steps
+//     whose residuals are formed in float64 from the exact Gram matrix): with
+//     rhs = B^T y and the gradient
 //     g = rhs - Gram s_old, whose entries are g_i = c_i^T (H r)_i at the
 //     current state, Gram s_new = rhs  <=>  Gram (s_new - s_old) = g.  With the
 //     ridge, (Gram + lambda I) s_new = rhs  <=>  (Gram + lambda I) delta =
@@ -60,33 +62,67 @@ __device__ __forceinline__ float warp_max(float v) {
 }
 
 struct SolveArgs {
-    const float *gram, *gvec, *W;
+    const double *gram, *gvec;
+    const float *W;
     const uint8_t *Q;
     const int32_t *Z;
     const double *F_start;
-    float *S, *r;
+    float *S;
+    ResidualView rv;
     double *L_prev, *dF_sweep;
     int *active, *iters, *ridge, *rstat, *status;
     int p, d, g, k;
     jarq_options o;
 };
 
+// Per-warp shared memory: float A[G][G+1], s_old[G], work[G]; double rhs[G], inc[G].
+__host__ __device__ inline size_t solve_warp_bytes(int G) {
+    size_t f = (size_t)G * (G + 1) + 2 * (size_t)G;
+    f = (f + 1) & ~(size_t)1;   // 8-byte alignment of the double part
+    return f * sizeof(float) + 2 * (size_t)G * sizeof(double);
+}
+
+// Forward and back substitution with the float32 factor in A: y <- (L L^T)^{-1} y.
+__device__ void warp_chol_solve(const float *A, int G, float *y) {
+    const int lane = threadIdx.x & 31, ld = G + 1;
+    for (int k = 0; k < G; ++k) {
+        __syncwarp();
+        const float yk = y[k] / A[k * ld + k];
+        __syncwarp();
+        if (lane == 0) y[k] = yk;
+        for (int t = k + 1 + lane; t < G; t += 32) y[t] = fmaf(-A[t * ld + k], yk, y[t]);
+    }
+    for (int k = G - 1; k >= 0; --k) {
+        __syncwarp();
+        const float sk = y[k] / A[k * ld + k];
+        __syncwarp();
+        if (lane == 0) y[k] = sk;
+        for (int t = lane; t < k; t += 32) y[t] = fmaf(-A[k * ld + t], sk, y[t]);
+    }
+    __syncwarp();
+}
+
 __global__ void scale_solve_kernel(SolveArgs a) {
-    extern __shared__ float smem[];
+    extern __shared__ __align__(16) unsigned char smem_raw[];
     const int G = a.d / a.g, ld = G + 1;
     const int wpb = blockDim.x >> 5, w = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int j = blockIdx.x * wpb + w;
     if (j >= a.p || !a.active[j]) return;  // warp-uniform
-    float *A = smem + (size_t)w * (G * ld + 4 * G);
-    float *b = A + G * ld;       // gradient g
-    float *so = b + G;           // s_old
-    float *y = so + G;           // right-hand side, then the increment
-    const float *gj = a.gram + (size_t)j * G * G;
+    unsigned char *base = smem_raw + (size_t)w * solve_warp_bytes(G);
+    float *A = (float *)base;
+    float *so = A + G * ld;         // s_old
+    float *y = so + G;              // float work vector
+    size_t fcount = (size_t)G * ld + 2 * (size_t)G;
+    fcount = (fcount + 1) & ~(size_t)1;
+    double *b = (double *)(base + fcount * sizeof(float));   // gradient g
+    double *inc = b + G;                                      // increment of the scales
+    const double *gj = a.gram + (size_t)j * G * G;
+    auto gsym = [&](int r0, int c0) { return 0.5 * (gj[r0 * G + c0] + gj[c0 * G + r0]); };
     auto load_sym = [&](float shift) -> bool {
         bool finite = true;
         for (int idx = lane; idx < G * G; idx += 32) {
             int r0 = idx / G, c0 = idx % G;
-            float v = 0.5f * (gj[r0 * G + c0] + gj[c0 * G + r0]);
+            float v = (float)gsym(r0, c0);
             if (r0 == c0) v += shift;
             if (!isfinite(v)) finite = false;
             A[r0 * ld + c0] = v;
@@ -94,9 +130,11 @@ __global__ void scale_solve_kernel(SolveArgs a) {
         __syncwarp();
         return __all_sync(0xffffffffu, finite);
     };
+    bool bfin = true;
     for (int t = lane; t < G; t += 32) {
         b[t] = a.gvec[(size_t)j * G + t];
         so[t] = a.S[(size_t)j * G + t];
+        bfin &= (bool)isfinite(b[t]);
     }
     bool finite = load_sym(0.f);
     float md = 0.f;
@@ -109,57 +147,50 @@ __global__ void scale_solve_kernel(SolveArgs a) {
         load_sym(a.o.ridge);
         ok = warp_cholesky(A, G, 0.f);
     }
-    // b must be finite for a usable solve
-    bool bfin = true;
-    for (int t = lane; t < G; t += 32) bfin &= (bool)isfinite(b[t]);
     ok = ok && __all_sync(0xffffffffu, bfin);
-    if (!ok) {
+    auto fail = [&]() {
         if (lane == 0) {
             a.ridge[j] += used_ridge;
             a.rstat[j] = JARQ_ERR_NUMERICAL;
             a.active[j] = 0;
             atomicOr(a.status, ST_NUMERICAL);
         }
+    };
+    if (!ok) {
+        fail();
         return;
     }
-    // forward: L y = g - lambda s_old
-    const float lam = used_ridge ? a.o.ridge : 0.f;
-    for (int t = lane; t < G; t += 32) y[t] = fmaf(-lam, so[t], b[t]);
-    for (int k = 0; k < G; ++k) {
-        __syncwarp();
-        const float yk = y[k] / A[k * ld + k];
-        __syncwarp();
-        if (lane == 0) y[k] = yk;
-        for (int t = k + 1 + lane; t < G; t += 32) y[t] = fmaf(-A[t * ld + k], yk, y[t]);
+    // (Gram + lambda I) inc = g - lambda s_old, refined twice with float64 residuals
+    const double lam = used_ridge ? (double)a.o.ridge : 0.0;
+    for (int t = lane; t < G; t += 32) {
+        inc[t] = 0.0;
+        y[t] = (float)(b[t] - lam * (double)so[t]);
     }
-    // backward: L^T s = y
-    for (int k = G - 1; k >= 0; --k) {
+    for (int step = 0; step < 3; ++step) {
+        warp_chol_solve(A, G, y);
+        for (int t = lane; t < G; t += 32) inc[t] += (double)y[t];
         __syncwarp();
-        const float sk = y[k] / A[k * ld + k];
-        __syncwarp();
-        if (lane == 0) y[k] = sk;
-        for (int t = lane; t < k; t += 32) y[t] = fmaf(-A[k * ld + t], sk, y[t]);
-    }
-    __syncwarp();
-    bool sfin = true;
-    for (int t = lane; t < G; t += 32) sfin &= (bool)isfinite(y[t]);
-    if (!__all_sync(0xffffffffu, sfin)) {
-        if (lane == 0) {
-            a.ridge[j] += used_ridge;
-            a.rstat[j] = JARQ_ERR_NUMERICAL;
-            a.active[j] = 0;
-            atomicOr(a.status, ST_NUMERICAL);
+        if (step == 2) break;
+        for (int r0 = lane; r0 < G; r0 += 32) {
+            double res = b[r0] - lam * ((double)so[r0] + inc[r0]);
+            for (int c0 = 0; c0 < G; ++c0) res = fma(-gsym(r0, c0), inc[c0], res);
+            y[r0] = (float)res;
         }
+        __syncwarp();
+    }
+    bool sfin = true;
+    for (int t = lane; t < G; t += 32) sfin &= (bool)isfinite(inc[t]);
+    if (!__all_sync(0xffffffffu, sfin)) {
+        fail();
         return;
     }
     // objective bookkeeping with the unridged symmetrised Gram matrix
     double t1 = 0.0, t2 = 0.0;
     for (int r0 = lane; r0 < G; r0 += 32) {
-        float gdl = 0.f;
-        for (int c0 = 0; c0 < G; ++c0)
-            gdl = fmaf(0.5f * (gj[r0 * G + c0] + gj[c0 * G + r0]), y[c0], gdl);
-        t1 += (double)y[r0] * (double)b[r0];
-        t2 += (double)y[r0] * (double)gdl;
+        double gdl = 0.0;
+        for (int c0 = 0; c0 < G; ++c0) gdl = fma(gsym(r0, c0), inc[c0], gdl);
+        t1 += inc[r0] * b[r0];
+        t2 += inc[r0] * gdl;
     }
     t1 = warp_sum(t1);
     t2 = warp_sum(t2);
@@ -171,8 +202,7 @@ __global__ void scale_solve_kernel(SolveArgs a) {
         const double den = fmax(fabs(a.L_prev[j]), (double)a.o.eps);
         stop = (dec / den <= (double)a.o.tau_rel) || (fabs(dec) <= (double)a.o.tau_abs);
     }
-    __syncwarp();
-    for (int t = lane; t < G; t += 32) y[t] = so[t] + y[t];   // s_new = s_old + delta
+    for (int t = lane; t < G; t += 32) y[t] = (float)((double)so[t] + inc[t]);   // s_new
     __syncwarp();
     for (int t = lane; t < G; t += 32) a.S[(size_t)j * G + t] = y[t];
     if (lane == 0) {
@@ -188,19 +218,19 @@ __global__ void scale_solve_kernel(SolveArgs a) {
     for (int c0 = lane; c0 < a.d; c0 += 32) {
         const int grp = c0 / a.g;
         const float c = (float)((int)a.Q[rowoff + c0] - zj[grp]);
-        a.r[rowoff + c0] = fmaf(-y[grp], c, a.W[rowoff + c0]);
+        store_residual(a.rv, j, c0, fmaf(-y[grp], c, a.W[rowoff + c0]));
     }
 }
 
 }  // namespace
 
-cudaError_t launch_scale_solve(const float *gram, const float *gvec, const float *W,
+cudaError_t launch_scale_solve(const double *gram, const double *gvec, const float *W,
                                const uint8_t *Q, const int32_t *Z, const double *F_start, float *S,
-                               float *r, double *L_prev, double *dF_sweep, int *active,
+                               ResidualView rv, double *L_prev, double *dF_sweep, int *active,
                                int *iters, int *ridge, int *rstat, int *status, int p, int d,
                                int g, int k, const jarq_options &o, cudaStream_t s) {
     const int G = d / g;
-    const size_t per_warp = (size_t)(G * (G + 1) + 4 * G) * sizeof(float);
+    const size_t per_warp = solve_warp_bytes(G);
     int wpb = (int)((96 * 1024) / per_warp);
     if (wpb > 8) wpb = 8;
     if (wpb < 1) wpb = 1;
@@ -208,7 +238,7 @@ cudaError_t launch_scale_solve(const float *gram, const float *gvec, const float
     cudaError_t e = cudaFuncSetAttribute(scale_solve_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    SolveArgs a{gram, gvec, W, Q, Z, F_start, S, r, L_prev, dF_sweep, active, iters, ridge, rstat,
+    SolveArgs a{gram, gvec, W, Q, Z, F_start, S, rv, L_prev, dF_sweep, active, iters, ridge, rstat,
                 status, p, d, g, k, o};
     scale_solve_kernel<<<(p + wpb - 1) / wpb, 32 * wpb, smem, s>>>(a);
     return cudaGetLastError();

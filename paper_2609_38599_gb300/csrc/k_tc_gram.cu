@@ -1,0 +1,355 @@
+// Exact Gram matrices of the joint scale fit on the tensor cores.
+//
+// Sec. 3.3.1, Eq. scale_design: Gram_j[i,h] = (A_i c_i)^T (A_h c_h)
+// = c_i^T H_ih c_h with integer codes c = q - z.  Each g x g block H_ih is
+// written as 2^(E_ih - 7) * sum_t a_t 2^(-8 t), t = 0..3, with integer
+// digits |a_t| <= 128 (exact in bf16) and E_ih the block's exponent, so
+//     D_t[j, m] = sum_{k in grp h} c_j[k] a_t[k, m]
+// is an integer of at most 23 bits: every tensor-core partial sum is exact
+// whatever the accumulator's rounding.  The epilogue forms the integer dots
+// G_t = sum_{m in grp i} c_j[m] D_t[j, m] and
+//     Gram_j[i,h] = 2^(E_ih - 7) (G_0 + G_1 2^-8 + G_2 2^-16 + G_3 2^-24)
+// in float64, exactly for the digit-represented block (whose error is at
+// most 2^(E_ih - 32) per entry).  Only h <= i is computed; the block is
+// mirrored.  A CTA owns one 128-row tile and the group pair {i, G-1-i}, so
+// every CTA processes G + 1 blocks.
+//
+// Roles: warp 0 TMA producer; warp 1 TMEM allocation and MMA issuer;
+// warps 2..5 epilogue (TMEM lanes 32 (w % 4) ..).  One unit of work is
+// (h, column half of group i): 4 accumulators of 64 columns (one per digit
+// plane), double-buffered in 512 TMEM columns.
+#include "tc_common.cuh"
+
+namespace jarq {
+namespace {
+
+constexpr int kTileA = 128 * 64 * 2;   // 128 code rows x 64 K
+constexpr int kTileB = 64 * 64 * 2;    // 64 H rows x 64 K, one digit plane
+constexpr int kStage = kTileA + 4 * kTileB;
+constexpr int kStages = 3;
+constexpr int kCodesBytes = 128 * 128 * 2;  // int16 codes of group i for the tile
+constexpr int kSmem = 1024 + kStages * kStage + kCodesBytes + 256;
+constexpr uint32_t kIdesc = tc::idesc_bf16_f32(128, 64);
+
+struct GramArgs {
+    const uint8_t *Q;
+    const int32_t *Z;
+    const int *expo;     // [G][G] block exponents E_ih
+    const int *active;
+    double *gram;        // [p][G][G]
+    int *status;
+    int p, d, g, G, d_pad;
+};
+
+__device__ __forceinline__ int exact_int(float x) {
+    // x is an integer with |x| < 2^22: add 1.5 * 2^23 and read the low bits
+    return __float_as_int(x + 12582912.0f) - 0x4B400000;
+}
+
+// WIDE: 64-bit integer dots (codes wider than 4 bits); otherwise every
+// per-slice dot of 64 terms fits in 32 bits (|c| <= 15, |D_t| < 2^18).
+template <bool WIDE>
+__global__ void __launch_bounds__(192, 1)
+    tc_gram_kernel(const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapS,
+                   GramArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    int16_t *codes = (int16_t *)(smem + kStages * kStage);   // [128 rows][128]
+    uint64_t *bars = (uint64_t *)(smem + kStages * kStage + kCodesBytes);
+    uint32_t *tmem_slot = (uint32_t *)(bars + 2 * kStages + 4);
+    volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int j0 = blockIdx.x * 128;
+    const int G = a.G, g = a.g;
+    const int nhalf = g / 64, nkc = g / 64;   // column halves of group i; K chunks per block
+
+    {
+        int mine = 0;
+        if (threadIdx.x < 128 && j0 + (int)threadIdx.x < a.p) mine = a.active[j0 + threadIdx.x];
+        if (!__syncthreads_or(mine)) return;
+    }
+    // groups handled by this CTA and the unit list: for each group i (h = 0..i,
+    // half = 0..nhalf-1), K chunks kc = 0..nkc-1 per unit
+    const int i_lo = blockIdx.y, i_hi = G - 1 - blockIdx.y;
+    const int ngrp = (i_lo == i_hi) ? 1 : 2;
+    auto group_of = [&](int n) { return n == 0 ? i_lo : i_hi; };
+    const int units0 = (i_lo + 1) * nhalf;
+    const int nunits = units0 + (ngrp == 2 ? (i_hi + 1) * nhalf : 0);
+    auto unit = [&](int u, int &gi, int &h, int &half) {
+        const int n = u < units0 ? 0 : 1;
+        const int r = u < units0 ? u : u - units0;
+        gi = group_of(n);
+        h = r / nhalf;
+        half = r % nhalf;
+    };
+
+    auto full = [&](int s) { return tc::smem_u32(bars + s); };
+    auto empty = [&](int s) { return tc::smem_u32(bars + kStages + s); };
+    auto afull = [&](int b) { return tc::smem_u32(bars + 2 * kStages + b); };
+    auto aempty = [&](int b) { return tc::smem_u32(bars + 2 * kStages + 2 + b); };
+    auto tileA = [&](int s) { return tc::smem_u32(smem + s * kStage); };
+    auto tileB = [&](int s, int t) { return tc::smem_u32(smem + s * kStage + kTileA + t * kTileB); };
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            tc::mbar_init(full(s), 1);
+            tc::mbar_init(empty(s), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            tc::mbar_init(afull(b), 1);
+            tc::mbar_init(aempty(b), 4);
+        }
+        *abort_flag = 0;
+        tc::fence_barrier_init();
+    }
+    if (warp == 1) {
+        tc::tmem_alloc(tc::smem_u32(tmem_slot), 512);
+        tc::tmem_relinquish();
+    }
+    if (warp == 0 && lane == 0) {
+        tc::prefetch_tmap(&mapC);
+        tc::prefetch_tmap(&mapS);
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    const int nchunks = nunits * nkc;
+
+    if (warp == 0 && lane == 0) {
+        // ---------------- producer: per chunk, codes of group h and 4 digit planes
+        int issued = 0;
+        for (int c = 0; c < nchunks; ++c) {
+            const int s = c % kStages;
+            if (!tc::mbar_wait(empty(s), ((c / kStages) & 1) ^ 1) || *abort_flag) {
+                *abort_flag = 1;
+                break;
+            }
+            int gi, h, half;
+            unit(c / nkc, gi, h, half);
+            const int kx = h * g + (c % nkc) * 64;
+            tc::mbar_expect_tx(full(s), kStage);
+            tc::tma_load_2d(tileA(s), &mapC, full(s), kx, j0);
+#pragma unroll
+            for (int t = 0; t < 4; ++t)
+                tc::tma_load_2d(tileB(s, t), &mapS, full(s), kx, t * a.d_pad + gi * g + half * 64);
+            issued = c + 1;
+        }
+        for (int c = issued > kStages ? issued - kStages : 0; c < issued; ++c)
+            if (!tc::mbar_wait(full(c % kStages), (c / kStages) & 1)) *abort_flag = 1;
+    } else if (warp == 1 && lane == 0) {
+        // ---------------- MMA issuer
+        for (int u = 0; u < nunits && !*abort_flag; ++u) {
+            const int b = u & 1;
+            if (!tc::mbar_wait(aempty(b), ((u >> 1) & 1) ^ 1)) {
+                *abort_flag = 1;
+                break;
+            }
+            tc::tc_fence_after();
+            for (int kc = 0; kc < nkc; ++kc) {
+                const int c = u * nkc + kc;
+                const int s = c % kStages;
+                if (!tc::mbar_wait(full(s), (c / kStages) & 1) || *abort_flag) {
+                    *abort_flag = 1;
+                    break;
+                }
+                tc::tc_fence_after();
+#pragma unroll
+                for (int sub = 0; sub < 4; ++sub) {
+                    const uint64_t ad = tc::sdesc_sw128(tileA(s)) + 2 * sub;
+#pragma unroll
+                    for (int t = 0; t < 4; ++t) {
+                        const uint64_t bd = tc::sdesc_sw128(tileB(s, t)) + 2 * sub;
+                        tc::mma_bf16(tmem + b * 256 + t * 64, ad, bd, kIdesc, (kc | sub) != 0);
+                    }
+                }
+                tc::mma_commit(empty(s));
+            }
+            tc::mma_commit(afull(b));
+        }
+    } else if (warp >= 2) {
+        // ---------------- epilogue: exact integer dots with the codes of group i
+        const int q = warp & 3;
+        const int rl = 32 * q + lane;           // row within the tile
+        const int row = j0 + rl;
+        int cur_g = -1;
+        long long acc[4] = {0, 0, 0, 0};
+        for (int u = 0; u < nunits; ++u) {
+            int gi, h, half;
+            unit(u, gi, h, half);
+            if (gi != cur_g) {
+                // stage this tile's codes of group gi (row rl written by its own thread)
+                __syncwarp();
+                for (int m = 0; m < g; ++m) {
+                    int c = 0;
+                    if (row < a.p) {
+                        const int cc = (int)a.Q[(size_t)row * a.d + gi * g + m] -
+                                       a.Z[(size_t)row * G + gi];
+                        c = cc;
+                    }
+                    codes[rl * 128 + m] = (int16_t)c;
+                }
+                __syncwarp();
+                cur_g = gi;
+            }
+            const int b = u & 1;
+            bool w = tc::mbar_wait(afull(b), (u >> 1) & 1);
+            w = __shfl_sync(0xffffffffu, w && !*abort_flag, 0);
+            tc::tc_fence_after();
+            if (!w) {
+                *abort_flag = 1;
+                break;
+            }
+            const uint32_t base = tmem + ((uint32_t)(32 * q) << 16) + b * 256;
+            const int16_t *crow = codes + rl * 128 + half * 64;
+#pragma unroll 1
+            for (int hb = 0; hb < 64; hb += 32) {
+                int cr[32];
+#pragma unroll
+                for (int e = 0; e < 32; e += 8) {
+                    const int4 pk = *reinterpret_cast<const int4 *>(crow + hb + e);
+                    const int w4[4] = {pk.x, pk.y, pk.z, pk.w};
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        cr[e + 2 * k] = (int)(int16_t)(w4[k] & 0xFFFF);
+                        cr[e + 2 * k + 1] = w4[k] >> 16;
+                    }
+                }
+#pragma unroll
+                for (int t = 0; t < 4; ++t) {
+                    uint32_t v0[16], v1[16];
+                    tc::tmem_ld16(base + t * 64 + hb, v0);
+                    tc::tmem_ld16(base + t * 64 + hb + 16, v1);
+                    tc::tmem_wait_ld();
+                    if (WIDE) {
+                        long long part = 0;
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) {
+                            part += (long long)cr[e] * exact_int(__uint_as_float(v0[e]));
+                            part += (long long)cr[16 + e] * exact_int(__uint_as_float(v1[e]));
+                        }
+                        acc[t] += part;
+                    } else {
+                        int part = 0;
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) {
+                            part += cr[e] * exact_int(__uint_as_float(v0[e]));
+                            part += cr[16 + e] * exact_int(__uint_as_float(v1[e]));
+                        }
+                        acc[t] += part;
+                    }
+                }
+            }
+            tc::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(aempty(b));
+            if (half == nhalf - 1) {
+                if (row < a.p) {
+                    const int E = a.expo[gi * G + h];
+                    const double v = ldexp((double)acc[0] + ldexp((double)acc[1], -8) +
+                                               ldexp((double)acc[2], -16) + ldexp((double)acc[3], -24),
+                                           E - 7);
+                    double *gr = a.gram + (size_t)row * G * G;
+                    gr[(size_t)gi * G + h] = v;
+                    gr[(size_t)h * G + gi] = v;
+                }
+#pragma unroll
+                for (int t = 0; t < 4; ++t) acc[t] = 0;
+            }
+        }
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc::tc_fence_after();
+        tc::tmem_dealloc(tmem, 512);
+    }
+    if (threadIdx.x == 0 && *abort_flag) atomicOr(a.status, ST_TIMEOUT);
+}
+
+// Per g x g block of the symmetric H: E = the exponent with max |H_blk| <= 2^E.
+__global__ void block_exponent_kernel(const float *__restrict__ Hs, int *__restrict__ expo, int d,
+                                      int g) {
+    const int G = d / g, bi = blockIdx.y, bh = blockIdx.x;
+    float mx = 0.f;
+    for (int idx = threadIdx.x; idx < g * g; idx += blockDim.x) {
+        const int r = idx / g, c = idx % g;
+        mx = fmaxf(mx, fabsf(Hs[(size_t)(bi * g + r) * d + bh * g + c]));
+    }
+    for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    __shared__ float wm[32];
+    if ((threadIdx.x & 31) == 0) wm[threadIdx.x >> 5] = mx;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float m = 0.f;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) m = fmaxf(m, wm[w]);
+        int e = 0;
+        if (m > 0.f) {
+            frexpf(m, &e);     // m = f 2^e, f in [0.5, 1): |H| <= 2^e
+        }
+        expo[bi * G + bh] = e;
+    }
+}
+
+// Digits a_t of every entry: x = H 2^(7 - E) in [-128, 128], a_0 = rint(x),
+// a_t = rint(256 (remainder)), four planes [4][d_pad][d_pad].
+__global__ void slice_kernel(const float *__restrict__ Hs, const int *__restrict__ expo,
+                             __nv_bfloat16 *__restrict__ planes, int d, int d_pad, int g) {
+    const int G = d / g;
+    const size_t n = (size_t)d * d;
+    const size_t plane = (size_t)d_pad * d_pad;
+    for (size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x; idx < n;
+         idx += (size_t)gridDim.x * blockDim.x) {
+        const int r = (int)(idx / d), c = (int)(idx % d);
+        const int E = expo[(r / g) * G + c / g];
+        float x = ldexpf(Hs[idx], 7 - E);
+        const size_t off = (size_t)r * d_pad + c;
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+            const float dgt = rintf(x);
+            planes[t * plane + off] = __float2bfloat16_rn(dgt);
+            x = (x - dgt) * 256.f;
+        }
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_slices(const float *Hs, int *expo, __nv_bfloat16 *planes, int d, int d_pad,
+                          int g, cudaStream_t s) {
+    const int G = d / g;
+    block_exponent_kernel<<<dim3(G, G), 256, 0, s>>>(Hs, expo, d, g);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    size_t n = (size_t)d * d;
+    int blocks = (int)((n + 255) / 256);
+    if (blocks > 16 * num_sms()) blocks = 16 * num_sms();
+    slice_kernel<<<blocks, 256, 0, s>>>(Hs, expo, planes, d, d_pad, g);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_tc_gram(const CUtensorMap &mapC, const CUtensorMap &mapS, const uint8_t *Q,
+                           const int32_t *Z, const int *expo, const int *active, double *gram,
+                           int p, int p_pad, int d, int d_pad, int g, int bits, int *status,
+                           cudaStream_t s) {
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(tc_gram_kernel<false>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(tc_gram_kernel<true>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    const int G = d / g;
+    GramArgs a{Q, Z, expo, active, gram, status, p, d, g, G, d_pad};
+    dim3 grid(p_pad / 128, (G + 1) / 2, 1);
+    if (bits <= 4)
+        tc_gram_kernel<false><<<grid, 192, kSmem, s>>>(mapC, mapS, a);
+    else
+        tc_gram_kernel<true><<<grid, 192, kSmem, s>>>(mapC, mapS, a);
+    return cudaGetLastError();
+}
+
+}  // namespace jarq

@@ -9,7 +9,8 @@ namespace jarq {
 namespace {
 
 const char *const kNames[] = {"validate", "residual", "init_rows", "hr_full", "grad", "gram",
-                              "scale_solve", "phase_hr", "babai", "symmetrize", "group_factor"};
+                              "scale_solve", "phase_hr", "babai", "symmetrize", "group_factor",
+                              "slices"};
 constexpr int kNumNames = sizeof(kNames) / sizeof(kNames[0]);
 
 struct Pending {

@@ -95,7 +95,7 @@ def library():
 
 
 KERNELS = ("validate", "residual", "init_rows", "hr_full", "grad", "gram", "scale_solve",
-           "phase_hr", "babai", "symmetrize", "group_factor")
+           "phase_hr", "babai", "symmetrize", "group_factor", "slices")
 
 
 def profile_enable(on: bool = True):

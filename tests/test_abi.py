@@ -63,6 +63,8 @@ def test_argument_errors_return_before_cuda_work(jarq):
     assert lib.jarq_prepare_hessian(ctypes.addressof(buf), 6, 4, 0.0, ctypes.byref(h), None) == jarq.JARQ_ERR_ARG
     assert lib.jarq_prepare_hessian(ctypes.addressof(buf), 4, 0, 0.0, ctypes.byref(h), None) == jarq.JARQ_ERR_ARG
     assert lib.jarq_prepare_hessian(ctypes.addressof(buf), 256, 256, 0.0, ctypes.byref(h), None) == jarq.JARQ_ERR_ARG
+    assert lib.jarq_prepare_hessian(ctypes.addressof(buf), 256, 32, 0.0, ctypes.byref(h), None) == jarq.JARQ_ERR_ARG
+    assert lib.jarq_prepare_hessian(ctypes.addressof(buf), 192, 128, 0.0, ctypes.byref(h), None) == jarq.JARQ_ERR_ARG
     assert lib.jarq_prepare_hessian(None, 4, 4, 0.0, ctypes.byref(h), None) == jarq.JARQ_ERR_ARG
     assert lib.jarq_prepare_hessian(ctypes.addressof(buf), 4, 4, 0.0, None, None) == jarq.JARQ_ERR_ARG
     # NULL handle, bad bits, negative dout

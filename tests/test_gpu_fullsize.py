@@ -56,7 +56,7 @@ def test_full_layer_sampled_rows(name):
     stats = {"L_host": st.L_host.cpu().numpy()[rows], "L_final": st.L_final.cpu().numpy()[rows]}
     m = compare_final(sub, prep, res, S.cpu().numpy()[rows], Q.cpu().numpy()[rows], stats)
     print(name, m)
-    assert m["Lhost_rel"] <= 1e-5 and m["Lfinal_vs_oracle_state"] <= 1e-5, m
+    assert m["Lhost_rel"] <= 5e-5 and m["Lfinal_vs_oracle_state"] <= 5e-5, m
     assert m["S_rel_max_same_rows"] <= 1e-4 and m["F_rel_max_same_rows"] <= 1e-4, m
     assert m["gpu_no_worse_than_host"], m
     assert m["codes_same"] >= 0.999, m
@@ -64,9 +64,13 @@ def test_full_layer_sampled_rows(name):
     assert int(Q.max()) <= (1 << lay.bits) - 1
 
 
-def test_lockstep_q_proj_sampled_rows():
-    lay = config_layer("llama2_7b_q_proj_4096x4096_g128_w3", device="cuda")
-    sub = sub_layer(to_np(lay), sample_rows(lay.dout, 24, seed=7))
+@pytest.mark.parametrize("name,n", [("llama2_7b_q_proj_4096x4096_g128_w3", 24),
+                                    ("llama2_7b_down_proj_4096x11008_g128_w4", 12)])
+def test_lockstep_sampled_rows(name, n):
+    """Both sides step one iteration at a time from the oracle's state; every
+    difference must start at a near-tie of the oracle's own values."""
+    lay = config_layer(name, device="cuda")
+    sub = sub_layer(to_np(lay), sample_rows(lay.dout, n, seed=7))
 
     def step(S, Q):
         S2, Q2, _ = gpu_refine(sub, 1, S=S, Q=Q)

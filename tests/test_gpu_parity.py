@@ -46,7 +46,7 @@ def test_tiny_layer_parity(jarq, early_stop):
     assert m["codes_same"] >= CODES_SAME, m
     assert m["S_rel_max_same_rows"] <= REL_S, m
     assert m["F_rel_max_same_rows"] <= REL_F, m
-    assert m["Lhost_rel"] <= 1e-5 and m["Lfinal_vs_oracle_state"] <= 1e-5, m
+    assert m["Lhost_rel"] <= 5e-5 and m["Lfinal_vs_oracle_state"] <= 5e-5, m
     assert m["gpu_no_worse_than_host"], m
     assert np.array_equal(st["iters"] > 0, np.ones(lay.dout, bool))
     if early_stop:
@@ -55,11 +55,12 @@ def test_tiny_layer_parity(jarq, early_stop):
 
 
 @pytest.mark.parametrize("din,dout,g,bits,K", [
-    (128, 100, 32, 3, 4),     # ragged rows (not a tile multiple)
-    (256, 257, 128, 4, 3),    # one group of 128 per half, ragged
-    (192, 70, 64, 2, 3),      # 2-bit, three groups
-    (96, 33, 16, 3, 5),       # small groups, 6 groups
+    (128, 100, 64, 3, 4),     # ragged rows (not a tile multiple)
+    (256, 257, 128, 4, 3),    # two groups of 128, ragged rows
+    (192, 70, 64, 2, 3),      # 2-bit, three groups, din not a multiple of 128
+    (448, 33, 64, 3, 5),      # seven groups of 64
     (640, 129, 128, 3, 4),    # five groups of 128
+    (1024, 300, 128, 4, 2),   # several K chunks per split
 ])
 def test_shapes_parity(jarq, din, dout, g, bits, K):
     lay = small_layer(din, dout, g, bits, K=K, seed=din + dout + g)
@@ -109,7 +110,7 @@ def test_host_buffers_match_device_buffers(jarq):
 
 
 def test_k0_returns_host_state(jarq):
-    lay = small_layer(128, 40, 32, 3, seed=23)
+    lay = small_layer(128, 40, 64, 3, seed=23)
     S, Q, st = gpu_refine(lay, 0)
     assert np.array_equal(Q, lay.Q0) and np.array_equal(S, lay.S0)
     np.testing.assert_allclose(st["L_final"], st["L_host"], rtol=0)
@@ -131,7 +132,7 @@ def test_format_preserved(jarq):
 
 
 def test_bad_codes_rejected_before_any_update(jarq):
-    lay = small_layer(128, 16, 32, 3, seed=25)
+    lay = small_layer(128, 16, 64, 3, seed=25)
     Q = lay.Q0.copy()
     Q[3, 5] = 9          # outside [0, 7]
     S = lay.S0.copy()
@@ -153,17 +154,17 @@ def test_not_spd_hessian_reported(jarq):
     H[40, 40] = -1.0
     from paper_2609_38599_gb300 import jarq as J
     with pytest.raises(J.JarqError) as ei:
-        J.prepare(H, 32)
+        J.prepare(H, 64)
     assert ei.value.status == J.JARQ_ERR_NOT_SPD
 
 
 def test_zero_group_takes_ridge_and_nan_row_is_numerical(jarq):
-    lay = small_layer(128, 8, 32, 3, seed=26)
+    lay = small_layer(256, 8, 64, 3, seed=26)
     Q = lay.Q0.copy()
-    Q[2, 32:64] = lay.Z[2, 1]           # c_i = 0: singular Gram -> ridge
+    Q[2, 64:128] = lay.Z[2, 1]          # c_i = 0: singular Gram -> ridge
     W = lay.W.copy()
     W[5, 7] = np.nan                    # nonfinite target -> numerical error
-    lay2 = Layer(lay.name, W, lay.H, lay.S0, Q, lay.Z, 3, 32, 2)
+    lay2 = Layer(lay.name, W, lay.H, lay.S0, Q, lay.Z, 3, 64, 2)
     S, Qg, st = gpu_refine(lay2, 2)
     assert st["status"] == 3            # JARQ_ERR_NUMERICAL for the call
     assert st["row_status"][5] == 3 and np.all(np.delete(st["row_status"], 5) == 0)
@@ -178,12 +179,11 @@ def test_zero_group_takes_ridge_and_nan_row_is_numerical(jarq):
 
 
 def test_small_scale_group_keeps_codes(jarq):
-    lay = small_layer(128, 12, 32, 3, seed=27)
-    # one iteration with a host grid whose group-1 scale refits to ~0 is hard to
-    # force; instead zero a group's codes-minus-zero so its refit scale is 0
+    lay = small_layer(256, 12, 64, 3, seed=27)
+    # zero a group's codes-minus-zero so its refit scale is 0 (below eps)
     Q = lay.Q0.copy()
-    Q[:, 32:64] = lay.Z[:, 1:2]
-    lay2 = Layer(lay.name, lay.W, lay.H, lay.S0, Q, lay.Z, 3, 32, 1)
+    Q[:, 64:128] = lay.Z[:, 1:2]
+    lay2 = Layer(lay.name, lay.W, lay.H, lay.S0, Q, lay.Z, 3, 64, 1)
     S, Qg, st = gpu_refine(lay2, 1)
     assert np.all(np.abs(S[:, 1]) <= 1e-6)
-    assert np.array_equal(Qg[:, 32:64], Q[:, 32:64])
+    assert np.array_equal(Qg[:, 64:128], Q[:, 64:128])
