@@ -35,12 +35,36 @@ PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 SM_COUNT = 152
 FP32_LANES_PER_SM = 128
 SM_MAX_MHZ = 2070.0
+DTYPE = "f32 (bf16x3 split products on tensor cores, exact integer Gram)"
+
+# DRAM bytes (read + write) per launch from one ncu capture of this workload
+# (profiles/ncu_*_q_proj_4096x4096_g128_w3.md), valid while the kernel's
+# source file is unchanged (first 12 hex digits of its SHA-1).
+TRAFFIC = {
+    "babai": ("k_babai.cu", "126ba525ab8f", 10.3488e6),
+    "hr_full": ("k_tc_hr.cu", "18cbbd861ee9", 816.96896e6 + 62.980608e6),
+    "phase_hr": ("k_tc_hr.cu", "18cbbd861ee9", 103.852544e6 + 3.142656e6),
+    "gram": ("k_tc_gram.cu", "09948d7fccb2", 159.193856e6 + 26.183936e6),
+}
+
+
+def traffic_for(kernel):
+    import hashlib
+    ent = TRAFFIC.get(kernel)
+    if not ent:
+        return None
+    path = os.path.join(ROOT, "paper_2609_38599_gb300", "csrc", ent[0])
+    try:
+        sha = hashlib.sha1(open(path, "rb").read()).hexdigest()[:12]
+    except OSError:
+        return None
+    return ent[2] if sha == ent[1] else None
 
 
 def parse_args():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default=WORKLOAD)
@@ -195,11 +219,56 @@ def config_dict(lay, note=None):
 # our arm
 # --------------------------------------------------------------------------
 
-def algorithmic_flops(kernel, lay):
-    """One MMA-equivalent of useful work per launch (App. G.7 counts)."""
-    p, d, g = lay.dout, lay.din, lay.g
-    return {"phase_hr": 2.0 * p * g * d, "gram": 2.0 * p * d * d,
-            "hr_full": 2.0 * p * d * d}.get(kernel)
+def kernel_model(kernel, lay, nsplit_bytes=0):
+    """Algorithmic work of one launch and the roofline that bounds the kernel.
+
+    Contractions count one MMA of useful work (2 x M x N x K); the split
+    products they issue (6 for H r, 4 digit planes for the Gram) are reported
+    separately as ``issued``.  Babai counts its dense triangular work, 2 g^2
+    flops per (row, group): the R^{-T} product and the back substitution.
+    Memory-bound kernels count the bytes they must move once.
+    """
+    p, d, g, G = lay.dout, lay.din, lay.g, lay.din // lay.g
+    if kernel == "phase_hr":
+        return dict(bound="tensor", work=2.0 * p * g * d, issued=6 * 2.0 * p * g * d)
+    if kernel == "hr_full":
+        return dict(bound="tensor", work=2.0 * p * d * d, issued=6 * 2.0 * p * d * d)
+    if kernel == "gram":
+        blocks = G * (G + 1) / 2
+        return dict(bound="tensor", work=2.0 * p * g * g * blocks, issued=4 * 2.0 * p * g * g * blocks)
+    if kernel == "babai":
+        return dict(bound="alu", work=2.0 * g * g * p)
+    if kernel == "scale_solve":
+        # Gram (f64) + gradient + scales in; scales and the residual (f32 + 3 bf16 planes) out
+        return dict(bound="hbm", work=p * (8.0 * G * G + 8 * G + 8 * G) + p * d * (1 + 4 + 4 + 10))
+    if kernel == "grad":
+        return dict(bound="hbm", work=p * d * (4 + 4 + 1) + p * G * 8)
+    return None
+
+
+def roofline_entry(kernel, stats, lay, pk, peak_kind):
+    m = kernel_model(kernel, lay)
+    if not m or not stats.get("launches"):
+        return None
+    avg_s = stats["total_ms"] / stats["launches"] / 1e3
+    if m["bound"] == "tensor":
+        achieved = m["work"] / avg_s / 1e12
+        peak, unit = pk["bf16_tflops_sustained"], "TFLOP/s"
+        note = f"bf16 dense, sustained ({peak_kind})"
+    elif m["bound"] == "alu":
+        achieved = m["work"] / avg_s / 1e12
+        peak, unit = SM_COUNT * FP32_LANES_PER_SM * 2 * SM_MAX_MHZ * 1e6 / 1e12, "TFLOP/s"
+        note = "fp32 FMA: 152 SMs x 128 lanes x 2 flop x 2070 MHz"
+    else:
+        achieved = m["work"] / avg_s / 1e9
+        peak, unit = pk["hbm_gbs"], "GB/s"
+        note = f"HBM copy bandwidth ({peak_kind})"
+    e = {"kernel": kernel, "bound": m["bound"], "achieved": achieved, "peak": peak, "unit": unit,
+         "frac": achieved / peak, "traffic": traffic_for(kernel), "avg_us": avg_s * 1e6,
+         "peak_note": note}
+    if "issued" in m:
+        e["issued_frac"] = m["issued"] / avg_s / 1e12 / peak
+    return e
 
 
 def run_ours(args, rank, world):
@@ -231,8 +300,6 @@ def run_ours(args, rank, world):
     vis = os.environ.get("CUDA_VISIBLE_DEVICES", "")
     gpu_index = vis.split(",")[local] if vis and vis.split(",")[0].isdigit() else local
     sampler = ClockSampler(gpu_index)
-    jarq.profile_reset()
-    jarq.profile_enable(True)
     n0 = jarq.launch_count()
     sampler.start()
     if dist:
@@ -248,13 +315,20 @@ def run_ours(args, rank, world):
     if dist:
         dist.barrier()
     clocks = sampler.stop()
-    jarq.profile_enable(False)
     launches = jarq.launch_count() - n0
     ms = e0.elapsed_time(e1) / args.steps
     if dist:
         t = torch.tensor([ms], device=dev)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         ms = float(t.item())
+    # per-kernel device time: the same K steps again with a CUDA event pair
+    # around every library launch, on the stream the kernels run on
+    jarq.profile_reset()
+    jarq.profile_enable(True)
+    for _ in range(args.steps):
+        step()
+    torch.cuda.synchronize()
+    jarq.profile_enable(False)
     weights = lay.din * lay.dout
     value = world * weights / (ms / 1e3)
     kernels = {}
@@ -266,23 +340,21 @@ def run_ours(args, rank, world):
     tot_all = sum(v["total_ms"] for v in kernels.values()) or 1.0
     for v in kernels.values():
         v["share"] = v["total_ms"] / tot_all
-    # dominant contraction kernel and its roofline
-    cand = [k for k in kernels if algorithmic_flops(k, lay)]
-    dom = max(cand, key=lambda k: kernels[k]["total_ms"]) if cand else None
-    roof = None
-    if dom:
-        avg_s = kernels[dom]["total_ms"] / kernels[dom]["launches"] / 1e3
-        achieved = algorithmic_flops(dom, lay) / avg_s / 1e12
-        peak = SM_COUNT * FP32_LANES_PER_SM * 2 * SM_MAX_MHZ * 1e6 / 1e12
-        roof = {"kernel": dom, "bound": "alu", "achieved": achieved, "peak": peak,
-                "unit": "TFLOP/s", "frac": achieved / peak, "traffic": None,
-                "peak_note": "fp32 FMA: 152 SMs x 128 lanes x 2 flop x 2070 MHz (CUDA-core contraction)"}
+    # roofline of every modelled kernel; `roofline` is the one with the largest share
+    pk, peak_kind = peaks()
+    roofs = {k: roofline_entry(k, v, lay, pk, peak_kind) for k, v in kernels.items()}
+    roofs = {k: v for k, v in roofs.items() if v}
+    dom = max(kernels, key=lambda k: kernels[k]["total_ms"]) if kernels else None
+    roof = roofs.get(dom)
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "s_per_layer": ms / 1e3,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": DTYPE,
         "data": "synthetic (seeded Llama-2-7B-shaped layer, RTN host)",
-        "config": config_dict(lay), "roofline": roof, "gpu_launches": launches,
+        "config": config_dict(lay), "roofline": roof, "roofline_all": roofs,
+        "gpu_launches": launches,
+        "kernel_timing": "CUDA event pair around every library launch on its stream, in a second "
+                         "pass of the same K steps (the value pass runs without them)",
         "launches_per_step": launches / args.steps, "clocks": clocks, "kernels": kernels,
     }
     # end to end through the C ABI with pinned host buffers
