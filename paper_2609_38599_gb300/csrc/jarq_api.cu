@@ -417,7 +417,7 @@ jarq_status jarq_refine_layer(jarq_hessian *h, const float *W, float *S, uint8_t
             RUN("phase_hr", 1, launch_tc_hr_phase(w.mapR, h->mapH128, h->mapH64, w.hr, p, w.p_pad, h->d_pad,
                                                   g, i, nsplit, w.active, h->dstatus, st));
             RUN("babai", 1, launch_babai(w.hr, nsplit, h->Lf, h->Rinv, la.W, la.S, la.Q, la.Z, rv, w.active,
-                                         w.dF_sweep, w.accepted, p, g, i, qmax, o.eps, st));
+                                         w.dF_sweep, w.accepted, h->dstatus, p, g, i, qmax, o.eps, st));
         }
     }
     const bool want_final = stats && stats->L_final;

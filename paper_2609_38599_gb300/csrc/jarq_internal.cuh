@@ -144,7 +144,26 @@ cudaError_t launch_scale_solve(const double *gram, const double *gvec, const flo
 cudaError_t launch_babai(const float *hr, int nsplit, const float *Lf, const float *Rinv,
                          const float *W, const float *S, uint8_t *Q, const int32_t *Z,
                          ResidualView rv, const int *active, double *dF_sweep, int *accepted,
-                         int p, int g, int i, int qmax, float eps, cudaStream_t s);
+                         int *status, int p, int g, int i, int qmax, float eps, cudaStream_t s);
+
+// Launch with programmatic stream serialization: the kernel may start while
+// the previous kernel in the stream finishes; it must call griddepcontrol.wait
+// before touching that kernel's inputs or outputs.
+template <class... KArgs, class... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t s, Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
+}
 cudaError_t launch_init_rows(int *active, int *iters, int *accepted, int *ridge, int *rstat,
                              double *dF_sweep, int p, cudaStream_t s);
 

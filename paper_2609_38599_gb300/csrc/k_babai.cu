@@ -23,12 +23,12 @@
 // dF = s^2 (||R Delta - y||^2 - ||y||^2) = s^2 sum_l (a_l - y_l)(a_l + y_l)
 // with a_l = R_ll Delta_l - u_l, exactly zero for an unchanged proposal.  A
 // proposal is kept iff it changes a code, dF is finite and dF < 0.
-#include "jarq_internal.cuh"
+#include "tc_common.cuh"
 
 namespace jarq {
 namespace {
 
-constexpr int kWarps = 16;
+constexpr int kMaxWarps = 32;   // warps per block (one row each) at most
 
 struct BabaiArgs {
     const float *hr;      // [nsplit][p_pad][g]
@@ -41,6 +41,7 @@ struct BabaiArgs {
     const int *active;
     double *dF_sweep;
     int *accepted;
+    int *status;
     int p, g, i, qmax;
     float eps;
 };
@@ -60,30 +61,46 @@ __device__ __forceinline__ void load_vec(const float *p, float (&v)[NT]) {
 }
 
 template <int NT>
-__global__ void __launch_bounds__(32 * kWarps) babai_kernel(BabaiArgs a) {
+__global__ void __launch_bounds__(32 * kMaxWarps) babai_kernel(BabaiArgs a) {
     constexpr int g = 32 * NT;
     extern __shared__ __align__(16) float smem[];
     float *Lg = smem;                 // [g][g] lower factor of group i
     float *Rg = smem + g * g;         // [g][g] R_i^{-1}
     float *rdiag = Rg + g * g;        // [g] 1 / R_ll
-    float *hbuf = rdiag + g;          // [kWarps][g] this warp's (H r)_i row
+    float *hbuf = rdiag + g;          // [warps][g] this warp's (H r)_i row
+    __shared__ uint64_t bar;
+    __shared__ int load_ok;
     const int d = a.rv.d, G = d / g;
-    const float *Lsrc = a.Lf + (size_t)a.i * g * g;
-    const float *Rsrc = a.Rinv + (size_t)a.i * g * g;
-    for (int idx = threadIdx.x * 4; idx < g * g; idx += blockDim.x * 4) {
-        *reinterpret_cast<float4 *>(Lg + idx) = *reinterpret_cast<const float4 *>(Lsrc + idx);
-        *reinterpret_cast<float4 *>(Rg + idx) = *reinterpret_cast<const float4 *>(Rsrc + idx);
+    // group factors of group i: two bulk copies (they do not depend on the
+    // previous kernel, so they overlap its tail under programmatic launch)
+    if (threadIdx.x == 0) {
+        tc::mbar_init(tc::smem_u32(&bar), 1);
+        tc::fence_barrier_init();
+        tc::mbar_expect_tx(tc::smem_u32(&bar), 2u * g * g * sizeof(float));
+        tc::bulk_load(tc::smem_u32(Lg), a.Lf + (size_t)a.i * g * g, g * g * sizeof(float),
+                      tc::smem_u32(&bar));
+        tc::bulk_load(tc::smem_u32(Rg), a.Rinv + (size_t)a.i * g * g, g * g * sizeof(float),
+                      tc::smem_u32(&bar));
+        load_ok = tc::mbar_wait(tc::smem_u32(&bar), 0) ? 1 : 0;
     }
     __syncthreads();
+    if (!load_ok) {
+        if (threadIdx.x == 0) atomicOr(a.status, ST_TIMEOUT);
+        return;
+    }
     for (int l = threadIdx.x; l < g; l += blockDim.x) rdiag[l] = 1.0f / Lg[l * g + l];
     __syncthreads();
-    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    // the phase product (previous kernel) must be complete before its
+    // partials are read and before the residual it reads is rewritten
+    tc::pdl_wait();
+    tc::pdl_launch_dependents();
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
     float *hrow = hbuf + wid * g;
     const int l0 = NT * lane;
     const int col0 = a.i * g;
     float rd[NT];
     load_vec<NT>(rdiag + l0, rd);
-    for (int j = blockIdx.x * kWarps + wid; j < a.p; j += gridDim.x * kWarps) {
+    for (int j = blockIdx.x * nwarps + wid; j < a.p; j += gridDim.x * nwarps) {
         if (!a.active[j]) continue;
         const float s = a.S[(size_t)j * G + a.i];
         if (!(fabsf(s) > a.eps)) continue;  // small-scale skip (also NaN)
@@ -97,11 +114,19 @@ __global__ void __launch_bounds__(32 * kWarps) babai_kernel(BabaiArgs a) {
 #pragma unroll
             for (int t = 0; t < NT; ++t) hv[t] += t2[t];
         }
-        int qc[NT], qn[NT];
+        float qc[NT], qn[NT];   // current and proposed codes (small integers, exact)
+        {
+            uint32_t packed = 0;
+            if constexpr (NT == 4) {
+                packed = *reinterpret_cast<const uint32_t *>(a.Q + off + l0);
+            } else {
+                packed = *reinterpret_cast<const uint16_t *>(a.Q + off + l0);
+            }
 #pragma unroll
-        for (int t = 0; t < NT; ++t) {
-            qc[t] = a.Q[off + l0 + t];
-            qn[t] = qc[t];
+            for (int t = 0; t < NT; ++t) {
+                qc[t] = (float)((packed >> (8 * t)) & 0xFFu);
+                qn[t] = qc[t];
+            }
         }
         __syncwarp();
 #pragma unroll
@@ -129,36 +154,35 @@ __global__ void __launch_bounds__(32 * kWarps) babai_kernel(BabaiArgs a) {
             u[t] = y[t];
         }
         // back substitution by jumps (Eq. babai_update)
+        const float qmaxf = (float)a.qmax;
         int hi = g - 1;
         bool any = false;
-        while (hi >= 0) {
-            int dl[NT], best = -1;
+        while (true) {
+            // each lane: its highest still-undecided coordinate whose code changes
+            int tb = -1;
+            float db = 0.f;
 #pragma unroll
             for (int t = 0; t < NT; ++t) {
-                const int l = l0 + t;
-                dl[t] = 0;
-                if (l <= hi) {
-                    float q = rintf(fmaf(u[t], rd[t], (float)qc[t]));
-                    q = fminf(fmaxf(q, 0.f), (float)a.qmax);
-                    dl[t] = (int)q - qc[t];
-                    if (dl[t] != 0) best = l;
+                const float q = fminf(fmaxf(rintf(fmaf(u[t], rd[t], qc[t])), 0.f), qmaxf);
+                if (l0 + t <= hi && q != qc[t]) {
+                    tb = t;
+                    db = q - qc[t];
                 }
             }
-            const int lstar = __reduce_max_sync(0xffffffffu, best);
-            if (lstar < 0) break;
-            const int owner = lstar / NT, ts = lstar - owner * NT;
-            int mine = 0;
-#pragma unroll
-            for (int t = 0; t < NT; ++t)
-                if (t == ts) mine = dl[t];
-            const int dstar = __shfl_sync(0xffffffffu, mine, owner);
+            const uint32_t bal = __ballot_sync(0xffffffffu, tb >= 0);
+            if (!bal) break;
+            const int owner = 31 - __clz(bal);
+            // t (2 bits) and the code change (|delta| <= 255) in one word
+            const int word = __shfl_sync(0xffffffffu, (tb & 3) | (((int)db + 256) << 2), owner);
+            const int ts = word & 3;
+            const float fd = (float)((word >> 2) - 256);
+            const int lstar = owner * NT + ts;
             if (lane == owner) {
 #pragma unroll
                 for (int t = 0; t < NT; ++t)
-                    if (t == ts) qn[t] = qc[t] + dstar;
+                    if (t == ts) qn[t] = qc[t] + fd;
             }
             any = true;
-            const float fd = (float)dstar;
             float lr[NT];
             load_vec<NT>(Lg + lstar * g + l0, lr);   // R[l'][l*] for l' = l0..
 #pragma unroll
@@ -170,7 +194,7 @@ __global__ void __launch_bounds__(32 * kWarps) babai_kernel(BabaiArgs a) {
         float acc = 0.f;
 #pragma unroll
         for (int t = 0; t < NT; ++t) {
-            const float av = Lg[(l0 + t) * g + l0 + t] * (float)(qn[t] - qc[t]) - u[t];
+            const float av = Lg[(l0 + t) * g + l0 + t] * (qn[t] - qc[t]) - u[t];
             acc = fmaf(av - y[t], av + y[t], acc);
         }
         for (int o = 16; o; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
@@ -180,9 +204,10 @@ __global__ void __launch_bounds__(32 * kWarps) babai_kernel(BabaiArgs a) {
         for (int t = 0; t < NT; ++t) {
             if (qn[t] != qc[t]) {
                 const int l = l0 + t;
-                a.Q[off + l] = (uint8_t)qn[t];
-                store_residual(a.rv, j, col0 + l, fmaf(-s, (float)(qn[t] - z), a.W[off + l]));
-                store_code(a.rv, j, col0 + l, qn[t] - z);
+                const int qi = (int)qn[t];
+                a.Q[off + l] = (uint8_t)qi;
+                store_residual(a.rv, j, col0 + l, fmaf(-s, (float)(qi - z), a.W[off + l]));
+                store_code(a.rv, j, col0 + l, qi - z);
             }
         }
         if (lane == 0) {
@@ -197,26 +222,29 @@ __global__ void __launch_bounds__(32 * kWarps) babai_kernel(BabaiArgs a) {
 cudaError_t launch_babai(const float *hr, int nsplit, const float *Lf, const float *Rinv,
                          const float *W, const float *S, uint8_t *Q, const int32_t *Z,
                          ResidualView rv, const int *active, double *dF_sweep, int *accepted,
-                         int p, int g, int i, int qmax, float eps, cudaStream_t s) {
-    BabaiArgs a{hr, nsplit, Lf, Rinv, W, S, Q, Z, rv, active, dF_sweep, accepted, p, g, i, qmax, eps};
-    const size_t smem = ((size_t)2 * g * g + g + (size_t)kWarps * g) * sizeof(float);
-    int blocks = (p + kWarps - 1) / kWarps;
-    const int cap = num_sms() * (smem > 110 * 1024 ? 1 : 2);
-    if (blocks > cap) blocks = cap;
-    if (blocks < 1) blocks = 1;
+                         int *status, int p, int g, int i, int qmax, float eps, cudaStream_t s) {
+    BabaiArgs a{hr, nsplit, Lf, Rinv, W, S, Q, Z, rv, active, dF_sweep, accepted, status, p, g, i, qmax, eps};
+    // one block per SM, one warp per row: spread the rows evenly over the SMs
+    const int nsm = num_sms();
+    int warps = (p + nsm - 1) / nsm;
+    if (warps > kMaxWarps) warps = kMaxWarps;
+    if (warps < 1) warps = 1;
+    int blocks = (p + warps - 1) / warps;
+    if (blocks > nsm) blocks = nsm;
+    const size_t smem = ((size_t)2 * g * g + g + (size_t)warps * g) * sizeof(float);
     cudaError_t e = cudaSuccess;
     if (g == 128) {
         e = cudaFuncSetAttribute(babai_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
-        babai_kernel<4><<<blocks, 32 * kWarps, smem, s>>>(a);
+        e = launch_pdl(babai_kernel<4>, dim3(blocks), dim3(32 * warps), smem, s, a);
     } else if (g == 64) {
         e = cudaFuncSetAttribute(babai_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
-        babai_kernel<2><<<blocks, 32 * kWarps, smem, s>>>(a);
+        e = launch_pdl(babai_kernel<2>, dim3(blocks), dim3(32 * warps), smem, s, a);
     } else {
         return cudaErrorInvalidValue;
     }
-    return cudaGetLastError();
+    return e;
 }
 
 }  // namespace jarq

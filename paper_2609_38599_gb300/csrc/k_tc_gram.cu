@@ -180,14 +180,19 @@ __global__ void __launch_bounds__(192, 1)
             if (gi != cur_g) {
                 // stage this tile's codes of group gi (row rl written by its own thread)
                 __syncwarp();
-                for (int m = 0; m < g; ++m) {
-                    int c = 0;
-                    if (row < a.p) {
-                        const int cc = (int)a.Q[(size_t)row * a.d + gi * g + m] -
-                                       a.Z[(size_t)row * G + gi];
-                        c = cc;
+                if (row < a.p) {
+                    const int zz = a.Z[(size_t)row * G + gi];
+                    const uint4 *src = reinterpret_cast<const uint4 *>(a.Q + (size_t)row * a.d + gi * g);
+                    for (int m16 = 0; m16 < g / 16; ++m16) {
+                        const uint4 v = src[m16];
+                        const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                        for (int k = 0; k < 16; ++k)
+                            codes[rl * 128 + m16 * 16 + k] =
+                                (int16_t)((int)((w4[k >> 2] >> (8 * (k & 3))) & 0xFFu) - zz);
                     }
-                    codes[rl * 128 + m] = (int16_t)c;
+                } else {
+                    for (int m = 0; m < g; ++m) codes[rl * 128 + m] = 0;
                 }
                 __syncwarp();
                 cur_g = gi;
@@ -222,21 +227,25 @@ __global__ void __launch_bounds__(192, 1)
                     tc::tmem_ld16(base + t * 64 + hb + 16, v1);
                     tc::tmem_wait_ld();
                     if (WIDE) {
-                        long long part = 0;
+                        long long p0 = 0, p1 = 0, p2 = 0, p3 = 0;
 #pragma unroll
-                        for (int e = 0; e < 16; ++e) {
-                            part += (long long)cr[e] * exact_int(__uint_as_float(v0[e]));
-                            part += (long long)cr[16 + e] * exact_int(__uint_as_float(v1[e]));
+                        for (int e = 0; e < 16; e += 2) {
+                            p0 += (long long)cr[e] * exact_int(__uint_as_float(v0[e]));
+                            p1 += (long long)cr[e + 1] * exact_int(__uint_as_float(v0[e + 1]));
+                            p2 += (long long)cr[16 + e] * exact_int(__uint_as_float(v1[e]));
+                            p3 += (long long)cr[17 + e] * exact_int(__uint_as_float(v1[e + 1]));
                         }
-                        acc[t] += part;
+                        acc[t] += (p0 + p1) + (p2 + p3);
                     } else {
-                        int part = 0;
+                        int p0 = 0, p1 = 0, p2 = 0, p3 = 0;
 #pragma unroll
-                        for (int e = 0; e < 16; ++e) {
-                            part += cr[e] * exact_int(__uint_as_float(v0[e]));
-                            part += cr[16 + e] * exact_int(__uint_as_float(v1[e]));
+                        for (int e = 0; e < 16; e += 2) {
+                            p0 += cr[e] * exact_int(__uint_as_float(v0[e]));
+                            p1 += cr[e + 1] * exact_int(__uint_as_float(v0[e + 1]));
+                            p2 += cr[16 + e] * exact_int(__uint_as_float(v1[e]));
+                            p3 += cr[17 + e] * exact_int(__uint_as_float(v1[e + 1]));
                         }
-                        acc[t] += part;
+                        acc[t] += (long long)((p0 + p1) + (p2 + p3));
                     }
                 }
             }

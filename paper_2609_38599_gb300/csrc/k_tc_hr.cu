@@ -34,6 +34,7 @@ namespace {
 constexpr int kTileA = 128 * 64 * 2;  // bytes of one 128 x 64 bf16 A tile
 constexpr int kProducts = 6;
 constexpr int kPeriod = 2;            // 64-wide K chunks per drain period
+constexpr int kGroupRows = 8;         // row tiles per band in the full-product tile order
 // (A plane, B plane) of each product; product 5 = (0, 0) is the leading one.
 __host__ __device__ constexpr int prod_a(int k) { return k == 0 ? 2 : k == 1 ? 1 : k == 3 ? 1 : 0; }
 __host__ __device__ constexpr int prod_b(int k) { return k == 2 ? 2 : k == 1 ? 1 : k == 4 ? 1 : 0; }
@@ -75,16 +76,32 @@ __global__ void __launch_bounds__(320, 1)
     uint32_t *tmem_slot = (uint32_t *)(bars + 2 * S + 4);
     volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int j0 = blockIdx.x * 128;
-    const int ncol0 = blockIdx.y * BN;  // relative to n_base
+    // tile order: grouped so that consecutive CTAs share column tiles within
+    // a band of kGroupRows row tiles (L2 reuse of both operands)
+    int tile_m = blockIdx.x, tile_n = blockIdx.y;
+    if (gridDim.y > 1) {
+        const int lin = blockIdx.y * gridDim.x + blockIdx.x;
+        const int per_band = kGroupRows * gridDim.y;
+        const int band = lin / per_band, in_band = lin % per_band;
+        const int rows_in_band = min(kGroupRows, (int)gridDim.x - band * kGroupRows);
+        tile_m = band * kGroupRows + in_band % rows_in_band;
+        tile_n = in_band / rows_in_band;
+    }
+    const int j0 = tile_m * 128;
+    const int ncol0 = tile_n * BN;  // relative to n_base
     const int n0 = a.n_base + ncol0;
     const int kc0 = blockIdx.z * a.kc_per_split;
     const int nk = min(a.kc_total, kc0 + a.kc_per_split) - kc0;
 
     if (a.active) {
+        // row activity is written by the scale solve, never by the kernel this
+        // launch may overlap, so it can be read before griddepcontrol.wait
         int mine = 0;
         if (threadIdx.x < 128 && j0 + (int)threadIdx.x < a.rows) mine = a.active[j0 + threadIdx.x];
-        if (!__syncthreads_or(mine)) return;
+        if (!__syncthreads_or(mine)) {
+            tc::pdl_wait();
+            return;
+        }
     }
     auto full = [&](int s) { return tc::smem_u32(bars + s); };
     auto empty = [&](int s) { return tc::smem_u32(bars + S + s); };
@@ -120,6 +137,10 @@ __global__ void __launch_bounds__(320, 1)
     __syncthreads();
     tc::tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    // inputs (residual planes) and outputs (partials) are shared with the
+    // previous kernel when launched programmatically: wait for it here
+    tc::pdl_wait();
+    tc::pdl_launch_dependents();
 
     if (warp == 0 && lane == 0) {
         // ---------------- producer
@@ -237,7 +258,7 @@ __global__ void __launch_bounds__(320, 1)
 
 template <int BN>
 cudaError_t launch_tc_hr_bn(const CUtensorMap &mapA, const CUtensorMap &mapB, const HrArgs &a,
-                            dim3 grid, cudaStream_t s) {
+                            dim3 grid, cudaStream_t s, bool programmatic = false) {
     using C = HrCfg<BN>;
     static bool attr_set = false;
     if (!attr_set) {
@@ -246,6 +267,7 @@ cudaError_t launch_tc_hr_bn(const CUtensorMap &mapA, const CUtensorMap &mapB, co
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
+    if (programmatic) return launch_pdl(tc_hr_kernel<BN>, grid, dim3(320), C::kSmem, s, mapA, mapB, a);
     tc_hr_kernel<BN><<<grid, 320, C::kSmem, s>>>(mapA, mapB, a);
     return cudaGetLastError();
 }
@@ -270,8 +292,8 @@ cudaError_t launch_tc_hr_phase(const CUtensorMap &mapA, const CUtensorMap &mapB1
     const int kc_per = (kc_total + nsplit - 1) / nsplit;
     HrArgs a{out, (size_t)p_pad * g, g, p, p_pad, d_pad, i * g, g, kc_total, kc_per, active, status};
     dim3 grid(p_pad / 128, 1, nsplit);
-    if (g == 128) return launch_tc_hr_bn<128>(mapA, mapB128, a, grid, s);
-    if (g == 64) return launch_tc_hr_bn<64>(mapA, mapB64, a, grid, s);
+    if (g == 128) return launch_tc_hr_bn<128>(mapA, mapB128, a, grid, s, true);
+    if (g == 64) return launch_tc_hr_bn<64>(mapA, mapB64, a, grid, s, true);
     return cudaErrorInvalidValue;
 }
 
