@@ -136,6 +136,30 @@ jarq_status jarq_objective(jarq_hessian *h, const float *W, const float *S, cons
                            const int32_t *Z, int dout, int bits, double *F_per_row,
                            void *stream);
 
+/* Per-row objective without any device allocation.  The paper has no
+ * counterpart: this entry point exists for callers that cannot allocate
+ * device memory when they need the objective -- code running while a CUDA
+ * graph is being captured, serving processes that reserve all device memory
+ * at start-up and forbid later allocations, and callers that cannot afford
+ * the device-wide synchronisation an allocation may cause.  It computes the
+ * same values as jarq_objective.
+ *   All buffers must be device memory (host pointers return JARQ_ERR_ARG,
+ *   since staging them would allocate).  The prepared handle h comes from
+ *   jarq_prepare_hessian, which allocates once, up front.
+ *   Limit: ceil(dout/128)*128 * ceil(din/128)*128 <= 2^20 (for example a
+ *   1024 x 1024 layer); larger layers return JARQ_ERR_ARG.
+ *   Scratch: one statically sized device array (about 16 MiB) that every GPU
+ *   loading the library holds until the process exits.  All calls share it
+ *   and it keeps the last call's contents; the call clears what must start at
+ *   zero.  Calls that overlap on the GPU (from two streams or two host
+ *   threads) race on it: serialise them.
+ *   The first call on a device looks up the array's device address; make
+ *   that first call before any stream capture.
+ *   Returns after the results are in F_per_row. */
+jarq_status jarq_objective_noalloc(jarq_hessian *h, const float *W, const float *S,
+                                   const uint8_t *Q, const int32_t *Z, int dout, int bits,
+                                   double *F_per_row, void *stream);
+
 /* Input width and group size of a prepared handle (0 for NULL). */
 int jarq_hessian_din(const jarq_hessian *h);
 int jarq_hessian_group_size(const jarq_hessian *h);

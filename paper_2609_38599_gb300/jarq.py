@@ -29,7 +29,8 @@ JARQ_ERR_NOMEM = 6
 EXPORTS = ("jarq_default_options", "jarq_prepare_hessian", "jarq_refine_layer",
            "jarq_objective", "jarq_hessian_din", "jarq_hessian_group_size",
            "jarq_hessian_destroy", "jarq_status_string", "jarq_profile_enable",
-           "jarq_profile_reset", "jarq_profile_read", "jarq_launch_count")
+           "jarq_profile_reset", "jarq_profile_read", "jarq_launch_count",
+           "jarq_objective_noalloc")
 
 
 class JarqError(RuntimeError):
@@ -66,6 +67,8 @@ def _load():
                                       ctypes.POINTER(Stats), vp]
     lib.jarq_objective.restype = ci
     lib.jarq_objective.argtypes = [vp, vp, vp, vp, vp, ci, ci, vp, vp]
+    lib.jarq_objective_noalloc.restype = ci
+    lib.jarq_objective_noalloc.argtypes = [vp, vp, vp, vp, vp, ci, ci, vp, vp]
     lib.jarq_hessian_din.restype = ci
     lib.jarq_hessian_din.argtypes = [vp]
     lib.jarq_hessian_group_size.restype = ci
