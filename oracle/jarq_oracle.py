@@ -37,6 +37,13 @@ Readings of the paper that this oracle takes where the text is silent:
 5. The small-scale test is ``|s| > FLT_EPSILON`` (absolute).
 6. Early stop (Eq. strict_stopping) is tested for k >= 2 right after the
    scale update, using the full objective L^{(k)}; the new scales are kept.
+7. The scales are single-precision numbers: App. E states that the scale
+   system is solved in FP32, and the scale table the refinement updates is
+   an FP32 array.  The oracle solves in float64 and stores the correctly
+   rounded float32 value after every solve (``Options.fp32_scales``); the
+   objective, the Babai recursion and the acceptance test then run in
+   float64 on those float32 scales.  ``fp32_scales=False`` keeps float64
+   scales, for the paper's exact worked examples.
 
 Parity status: every function here is pinned by ``tests/test_oracle_*.py``
 against the paper's worked examples (App. G, Props. grid-staleness and
@@ -67,6 +74,7 @@ class Options:
     ridge: float = 1e-4         # lambda of the stabilised scale solve
     rcond: float = 1e-10        # spectrum test threshold
     eps: float = FP32_EPS       # eps_fp
+    fp32_scales: bool = True    # store each solved scale as float32 (reading 7)
 
 
 @dataclasses.dataclass
@@ -322,7 +330,7 @@ def refine_layer(prep: Prepared, W, S0, Q0, Z, bits: int, opt: Options = None,
                 status[j] = ROW_NUMERICAL
                 active[j] = False
                 continue
-            S[j] = s
+            S[j] = s.astype(np.float32) if opt.fp32_scales else s
         rows = np.nonzero(active)[0]
         iters[rows] = k
         L = np.full(p, np.nan)

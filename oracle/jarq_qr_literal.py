@@ -30,12 +30,15 @@ FP32_EPS = float(np.finfo(np.float32).eps)
 
 
 def refine_columns(X, W, S0, Q0, Z, bits, g, K, nu=0.0, Ystar=None, tau=1e-5,
-                   early_stop=True, ridge=1e-4, rcond=1e-10, eps=FP32_EPS):
+                   early_stop=True, ridge=1e-4, rcond=1e-10, eps=FP32_EPS,
+                   fp32_scales=True):
     """Refine every output column of a tiny layer with the paper's QR form.
 
     ``X``: n x din calibration inputs; ``W``: dout x din (row j = paper's
     column w_j); ``Ystar``: n x dout activation target (default ``X W^T``,
-    the main target of Sec. 3.2).  Returns ``(S, Q, F_final)``.
+    the main target of Sec. 3.2).  ``fp32_scales`` stores every solved scale
+    as float32, the single-precision scale solve of App. E.  Returns
+    ``(S, Q, F_final)``.
     """
     X = np.asarray(X, dtype=np.float64)
     W = np.asarray(W, dtype=np.float64)
@@ -80,7 +83,7 @@ def refine_columns(X, W, S0, Q0, Z, bits, g, K, nu=0.0, Ystar=None, tau=1e-5,
             except np.linalg.LinAlgError:
                 Lc = np.linalg.cholesky(Gm + ridge * np.eye(G))
                 s_new = np.linalg.solve(Lc.T, np.linalg.solve(Lc, rhs))
-            s = s_new
+            s = s_new.astype(np.float32).astype(np.float64) if fp32_scales else s_new
             L = full_obj(s, q)
             if early_stop and k >= 2:
                 dec = L_prev - L

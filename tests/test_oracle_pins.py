@@ -72,8 +72,9 @@ def test_multicode_babai_step_and_refit(golden_dir):
     Q0 = np.array([ex["q0"]], dtype=np.uint8)
     S0 = np.array([[F(ex["s0"])]])
     trace = []
+    # the worked example is exact arithmetic: keep float64 scales
     res = refine_layer(prep, W, S0, Q0, Z, ex["bits"],
-                       Options(max_iters=2, early_stop=False), trace=trace)
+                       Options(max_iters=2, early_stop=False, fp32_scales=False), trace=trace)
     scale1, babai1, sweep1, scale2 = trace[0], trace[1], trace[2], trace[3]
     assert scale1["S"][0, 0] == pytest.approx(F(ex["s0"]), rel=1e-14)
     assert scale1["L"][0] == pytest.approx(F(ex["phi_q0"]), rel=1e-12)
@@ -137,7 +138,8 @@ def test_staleness_refit_unlocks_descent(golden_dir):
     Z = np.zeros((1, 1), dtype=np.int32)
     trace = []
     res = refine_layer(prep, W, np.array([[F(ex["s0"])]]), np.array([ex["q0"]], dtype=np.uint8), Z,
-                       ex["bits"], Options(max_iters=2, early_stop=False), trace=trace)
+                       ex["bits"], Options(max_iters=2, early_stop=False, fp32_scales=False),
+                       trace=trace)
     sc1, b1, sw1, sc2, b2, sw2 = trace
     assert res.L_host[0] == pytest.approx(F(ex["F0"]), rel=1e-13)
     assert sc1["S"][0, 0] == pytest.approx(F(ex["s1"]), rel=1e-14)
@@ -153,6 +155,31 @@ def test_staleness_refit_unlocks_descent(golden_dir):
     assert not b2["accepted"][0] and b2["dF"][0] == 0.0
     assert list(res.Q[0]) == ex["q_plus"]
     assert res.L_final[0] == pytest.approx(F(ex["F_s2_qplus"]), rel=1e-13)
+
+
+def test_scales_are_stored_as_correctly_rounded_float32(golden_dir):
+    """App. E: the scale system is solved in single precision.  With the
+    default options every stored scale is the float32 value nearest to the
+    exact solve: on the staleness example s1 = 197/200 and s2 = 4631/5000
+    are stored as float32(197/200) and float32(4631/5000), and the objective
+    L^(k) is evaluated at those float32 scales."""
+    ex = load(golden_dir, "grid_staleness_example.json")
+    H, W = staleness_setup(ex)
+    prep = prepare_hessian(H, 2)
+    Z = np.zeros((1, 1), dtype=np.int32)
+    trace = []
+    refine_layer(prep, W, np.array([[F(ex["s0"])]]), np.array([ex["q0"]], dtype=np.uint8), Z,
+                 ex["bits"], Options(max_iters=2, early_stop=False), trace=trace)
+    sc1, _, _, sc2, _, _ = trace
+    s1 = float(np.float32(F(ex["s1"])))
+    s2 = float(np.float32(F(ex["s2"])))
+    assert s1 != F(ex["s1"]) and s2 != F(ex["s2"])   # neither is a float32
+    assert sc1["S"][0, 0] == s1
+    assert sc2["S"][0, 0] == s2
+    assert sc1["L"][0] == pytest.approx(objective(prep, W, np.array([[s1]]),
+                                                  np.array([ex["q0"]]), Z)[0], rel=1e-15)
+    # the float32 rounding moves the objective by a second-order amount only
+    assert sc1["L"][0] == pytest.approx(F(ex["F_s1_q0"]), rel=1e-12)
 
 
 # ---------------------------------------------------------------------------
@@ -482,10 +509,12 @@ def test_h_form_matches_paper_literal_qr_form():
     damp = 0.01 * float(np.mean(np.diag(Hx)))
     prep = prepare_hessian(Hx + damp * np.eye(lay.din), lay.g)
     rows = np.arange(0, lay.dout, 16)
+    # two formulations of the same float64 arithmetic: float64 scales on both
     res = refine_layer(prep, lay.W[rows], lay.S0[rows], lay.Q0[rows], lay.Z[rows], lay.bits,
-                       Options(max_iters=5))
+                       Options(max_iters=5, fp32_scales=False))
     S3, Q3, F3 = refine_columns(X / np.sqrt(n), lay.W[rows], lay.S0[rows], lay.Q0[rows],
-                                lay.Z[rows], lay.bits, lay.g, 5, nu=np.sqrt(damp))
+                                lay.Z[rows], lay.bits, lay.g, 5, nu=np.sqrt(damp),
+                                fp32_scales=False)
     assert np.array_equal(Q3, res.Q)
     np.testing.assert_allclose(S3, res.S, rtol=1e-10)
     np.testing.assert_allclose(F3, res.L_final, rtol=1e-9)
