@@ -35,7 +35,7 @@ PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 SM_COUNT = 152
 FP32_LANES_PER_SM = 128
 SM_MAX_MHZ = 2070.0
-DTYPE = "f32 (bf16x3 split products on tensor cores, exact integer Gram)"
+DTYPE = "f32 (bf16x3 split products on tensor cores; integer-digit Gram and projection)"
 
 # DRAM bytes (read + write) per launch from one ncu capture of this workload
 # (profiles/ncu_*_q_proj_4096x4096_g128_w3.md), valid while the kernel's
@@ -223,8 +223,8 @@ def kernel_model(kernel, lay, nsplit_bytes=0):
     """Algorithmic work of one launch and the roofline that bounds the kernel.
 
     Contractions count one MMA of useful work (2 x M x N x K); the split
-    products they issue (6 for H r, 4 digit planes for the Gram) are reported
-    separately as ``issued``.  Babai counts its dense triangular work, 2 g^2
+    products they issue (6 for H r, 4 digit planes for the Gram, 18 digit
+    pairs for the target projection) are reported separately as ``issued``.  Babai counts its dense triangular work, 2 g^2
     flops per (row, group): the R^{-T} product and the back substitution.
     Memory-bound kernels count the bytes they must move once.
     """
@@ -243,6 +243,15 @@ def kernel_model(kernel, lay, nsplit_bytes=0):
         return dict(bound="hbm", work=p * (8.0 * G * G + 8 * G + 8 * G) + p * d * (1 + 4 + 4 + 10))
     if kernel == "grad":
         return dict(bound="hbm", work=p * d * (4 + 4 + 1) + p * G * 8)
+    if kernel == "proj":
+        return dict(bound="tensor", work=2.0 * p * d * d, issued=18 * 2.0 * p * d * d)
+    if kernel == "rhs":
+        # codes + double-float projection in, rhs (f64) out
+        return dict(bound="hbm", work=p * d * (1 + 4 + 4) + p * G * (4 + 8))
+    if kernel == "whw":
+        return dict(bound="hbm", work=p * d * (4 + 4 + 4) + p * 8)
+    if kernel == "slice_rows":
+        return dict(bound="hbm", work=p * d * (4 + 4 * 2) + p * G * 4)
     return None
 
 

@@ -26,7 +26,9 @@
  *   [dout][G]; H is float32 [din][din]; G = din / group_size.
  * - Pointers may be device memory or host memory (pageable or pinned).
  *   Host buffers are staged through library-owned device buffers; device
- *   buffers are used in place.  The caller owns every buffer it passes.
+ *   buffers are used in place, except a device Q that is not 16-byte
+ *   aligned, which is staged like host memory.  The caller owns every
+ *   buffer it passes.
  * - `stream` is a cudaStream_t passed as void* (NULL = the legacy default
  *   stream).  Work is enqueued on it in order.  Calls return after the work
  *   they enqueued has finished and its status has been read back.
@@ -112,6 +114,8 @@ jarq_status jarq_prepare_hessian(const float *H, int din, int group_size, float 
 
 /* Refine one layer in place: K iterations of joint scale fit + Babai sweep
  * (Sec. 3.3; App. E "Order of updates", "Early stopping", "Small scales").
+ * Each solved scale is stored as float32, the precision of the paper's scale
+ * solve (App. E "Solving for scales"), before the codes are updated.
  *   h      : prepared Hessian for this layer's input (din, group size).
  *   W      : float32 [dout][din], original weights (read only).
  *   S      : float32 [dout][G], host scales in, refined signed scales out.
@@ -135,6 +139,16 @@ jarq_status jarq_refine_layer(jarq_hessian *h, const float *W, float *S, uint8_t
 jarq_status jarq_objective(jarq_hessian *h, const float *W, const float *S, const uint8_t *Q,
                            const int32_t *Z, int dout, int bits, double *F_per_row,
                            void *stream);
+
+/* The residual product H r_j of every row, r_j = w_j - D_{s_j}(q_j - z_j),
+ * written as float32 to HR[dout][din] (host or device), computed by the
+ * split-precision tensor-core kernel that gives the Gauss-Seidel sweep its
+ * group slices (H r_j)_i (Sec. 3.3.2, Eq. conditional_residual).  It exists
+ * so that tests can compare that contraction element by element with a
+ * reference.  Same layouts and checks as jarq_refine_layer. */
+jarq_status jarq_residual_product(jarq_hessian *h, const float *W, const float *S,
+                                  const uint8_t *Q, const int32_t *Z, int dout, int bits,
+                                  float *HR, void *stream);
 
 /* Per-row objective without any device allocation.  The paper has no
  * counterpart: this entry point exists for callers that cannot allocate

@@ -1,11 +1,13 @@
 // C ABI entry points: handle lifecycle, argument checks, staging of host
 // buffers and the refinement loop (Sec. 3.3; App. E "Order of updates").
 //
-// Per iteration k = 1..K: the product H r of the current residual (giving
-// the objective and the scale gradient g_i = c_i^T (H r)_i), the Gram
-// matrices of the current codes, the joint scale solve with the early-stop
-// bookkeeping, and one Gauss-Seidel sweep over the groups, each group being
-// a residual-product phase followed by a Babai phase.
+// Once per call: the target projection P = W H, w^T H w and the folded
+// projection Pt_i = R_i^{-T} P_i (App. G "Computational Complexity",
+// target-projection shortcut).  Per iteration k = 1..K: the Gram matrices of
+// the current codes and rhs_i = c_i^T P_i, the joint scale solve (gradient
+// rhs - Gram s, objective, early stop), and one Gauss-Seidel sweep over the
+// groups, each group being a target-product phase (T_i) followed by a Babai
+// phase on y = (Pt_i - T_i) / s_i.
 #include <float.h>
 #include <stdlib.h>
 #include <string.h>
@@ -52,10 +54,11 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t
                                   const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
-// 2D bf16 tensor map over [rows][cols] (pitch = cols), box_rows x 64 boxes,
-// 128-byte swizzle, out-of-range elements read as zero.
-cudaError_t make_tmap_bf16(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols,
-                           uint32_t box_rows) {
+// 2D tensor map of 2-byte elements (bf16 or fp16) over [rows][cols]
+// (pitch = cols), box_rows x 64 boxes, 128-byte swizzle, out-of-range
+// elements read as zero.
+cudaError_t make_tmap_2b(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols,
+                         uint32_t box_rows, CUtensorMapDataType dtype) {
     static EncodeTiledFn fn = nullptr;
     if (!fn) {
         void *ptr = nullptr;
@@ -70,10 +73,20 @@ cudaError_t make_tmap_bf16(CUtensorMap *m, const void *base, uint64_t rows, uint
     cuuint64_t strides[1] = {cols * 2};
     cuuint32_t box[2] = {64, box_rows};
     cuuint32_t es[2] = {1, 1};
-    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides,
+    CUresult r = fn(m, dtype, 2, const_cast<void *>(base), dims, strides,
                     box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+cudaError_t make_tmap_bf16(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols,
+                           uint32_t box_rows) {
+    return make_tmap_2b(m, base, rows, cols, box_rows, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16);
+}
+
+cudaError_t make_tmap_f16(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols,
+                          uint32_t box_rows) {
+    return make_tmap_2b(m, base, rows, cols, box_rows, CU_TENSOR_MAP_DATA_TYPE_FLOAT16);
 }
 
 // Split-K factor of the phase product: enough CTAs to cover the SMs.
@@ -99,11 +112,17 @@ void free_ws(Workspace &w) {
     cudaFree(w.Hr);
     cudaFree(w.r);
     cudaFree(w.gram);
-    cudaFree(w.gvec);
-    cudaFree(w.hr);
-    cudaFree(w.F_start);
+    cudaFree(w.rhs);
+    cudaFree(w.t_hi);
+    cudaFree(w.t_lo);
+    cudaFree(w.Pt_hi);
+    cudaFree(w.Pt_lo);
+    cudaFree(w.wdig);
+    cudaFree(w.wexp);
+    cudaFree(w.Phi);
+    cudaFree(w.Plo);
+    cudaFree(w.wHw);
     cudaFree(w.L_prev);
-    cudaFree(w.dF_sweep);
     cudaFree(w.L_host);
     cudaFree(w.L_final);
     cudaFree(w.active);
@@ -133,17 +152,26 @@ cudaError_t ensure_ws(jarq_hessian *h, int p) {
         return e;
     if ((e = dalloc(&w.cplane, (size_t)p_pad * h->d_pad)) != cudaSuccess) return e;
     if ((e = cudaMemset(w.cplane, 0, (size_t)p_pad * h->d_pad * 2)) != cudaSuccess) return e;
-    if ((e = make_tmap_bf16(&w.mapC, w.cplane, (uint64_t)p_pad, h->d_pad, 128)) != cudaSuccess)
+    if ((e = make_tmap_f16(&w.mapC, w.cplane, (uint64_t)p_pad, h->d_pad, 128)) != cudaSuccess)
+        return e;
+    if ((e = dalloc(&w.wdig, (size_t)4 * p_pad * h->d_pad)) != cudaSuccess) return e;
+    if ((e = cudaMemset(w.wdig, 0, (size_t)4 * p_pad * h->d_pad * 2)) != cudaSuccess) return e;
+    if ((e = make_tmap_bf16(&w.mapWd, w.wdig, (uint64_t)4 * p_pad, h->d_pad, 128)) != cudaSuccess)
         return e;
     w.p_pad = p_pad;
     if ((e = dalloc(&w.Hr, (size_t)p * d)) != cudaSuccess) return e;
     if ((e = dalloc(&w.r, (size_t)p * d)) != cudaSuccess) return e;
     if ((e = dalloc(&w.gram, (size_t)p * G * G)) != cudaSuccess) return e;
-    if ((e = dalloc(&w.gvec, (size_t)p * G)) != cudaSuccess) return e;
-    if ((e = dalloc(&w.hr, (size_t)kMaxSplit * p_pad * g)) != cudaSuccess) return e;
-    if ((e = dalloc(&w.F_start, (size_t)p)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.rhs, (size_t)p * G)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.t_hi, (size_t)kMaxSplit * p_pad * g)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.t_lo, (size_t)kMaxSplit * p_pad * g)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.Pt_hi, (size_t)p * d)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.Pt_lo, (size_t)p * d)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.wexp, (size_t)p * G)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.Phi, (size_t)p * d)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.Plo, (size_t)p * d)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.wHw, (size_t)p)) != cudaSuccess) return e;
     if ((e = dalloc(&w.L_prev, (size_t)p)) != cudaSuccess) return e;
-    if ((e = dalloc(&w.dF_sweep, (size_t)p)) != cudaSuccess) return e;
     if ((e = dalloc(&w.L_host, (size_t)p)) != cudaSuccess) return e;
     if ((e = dalloc(&w.L_final, (size_t)p)) != cudaSuccess) return e;
     if ((e = dalloc(&w.active, (size_t)p)) != cudaSuccess) return e;
@@ -168,8 +196,10 @@ cudaError_t stage_layer(jarq_hessian *h, const float *W, const float *S, const u
                         const int32_t *Z, int p, LayerArgs &out, cudaStream_t st) {
     Workspace &w = h->ws;
     const size_t d = h->din, G = h->G;
-    const bool dW = is_device_ptr(W), dS = is_device_ptr(S), dQ = is_device_ptr(Q),
-               dZ = is_device_ptr(Z);
+    // the kernels read the codes in 16-byte vectors: a device Q that is not
+    // 16-byte aligned is staged like host memory
+    const bool dW = is_device_ptr(W), dS = is_device_ptr(S),
+               dQ = is_device_ptr(Q) && ((uintptr_t)Q & 15) == 0, dZ = is_device_ptr(Z);
     if ((!dW || !dS || !dQ || !dZ) && w.stage_rows < p) {
         cudaFree(w.sW);
         cudaFree(w.sS);
@@ -202,7 +232,7 @@ cudaError_t stage_layer(jarq_hessian *h, const float *W, const float *S, const u
         out.hS = true;
     }
     if (e == cudaSuccess && !dQ) {
-        e = cudaMemcpyAsync(w.sQ, Q, (size_t)p * d, cudaMemcpyHostToDevice, st);
+        e = cudaMemcpyAsync(w.sQ, Q, (size_t)p * d, cudaMemcpyDefault, st);
         out.Q = w.sQ;
         out.hQ = true;
     }
@@ -236,7 +266,8 @@ ResidualView rview(jarq_hessian *h) {
 
 // Common front half of refine/objective: stage, validate, residual.
 jarq_status layer_front(jarq_hessian *h, const float *W, const float *S, const uint8_t *Q,
-                        const int32_t *Z, int dout, int bits, LayerArgs &la, cudaStream_t st) {
+                        const int32_t *Z, int dout, int bits, LayerArgs &la, cudaStream_t st,
+                        bool codes_only = false) {
     CK(cudaSetDevice(h->device));
     CK(ensure_ws(h, dout));
     CK(stage_layer(h, W, S, Q, Z, dout, la, st));
@@ -245,7 +276,9 @@ jarq_status layer_front(jarq_hessian *h, const float *W, const float *S, const u
     int sb = 0;
     CK(read_status(h, st, &sb));
     if (sb) return status_from_bits(sb);
-    RUN("residual", 1, launch_residual(la.W, la.S, la.Q, la.Z, rview(h), dout, h->g, st));
+    ResidualView rv = rview(h);
+    if (codes_only) rv.r = nullptr;
+    RUN("residual", 1, launch_residual(la.W, la.S, la.Q, la.Z, rv, dout, h->g, st));
     return JARQ_OK;
 }
 
@@ -295,10 +328,13 @@ void jarq_hessian_destroy(jarq_hessian *h) {
     free_ws(h->ws);
     cudaFree(h->Hs);
     cudaFree(h->Hplanes);
-    cudaFree(h->Hdigits);
+    cudaFree(h->Hdig8);
+    cudaFree(h->Hdig10);
     cudaFree(h->expo);
     cudaFree(h->Lf);
     cudaFree(h->Rinv);
+    cudaFree(h->Htdig);
+    cudaFree(h->expoT);
     cudaFree(h->dstatus);
     cudaFreeHost(h->hstatus);
     (void)cudaGetLastError();
@@ -318,7 +354,7 @@ jarq_status jarq_prepare_hessian(const float *H, int din, int group_size, float 
     h->G = din / group_size;
     h->d_pad = round_up(din, 128);
     jarq_status rc = JARQ_OK;
-    float *Hdev = nullptr;
+    float *Hdev = nullptr, *Ht_hi = nullptr, *Ht_lo = nullptr;
     do {
         if (cudaGetDevice(&h->device) != cudaSuccess) { rc = JARQ_ERR_CUDA; break; }
         const size_t dd = (size_t)din * din;
@@ -329,12 +365,19 @@ jarq_status jarq_prepare_hessian(const float *H, int din, int group_size, float 
         if ((e = cudaMemsetAsync(h->Hplanes, 0, 3 * pd * 2, st)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = make_tmap_bf16(&h->mapH128, h->Hplanes, (uint64_t)3 * h->d_pad, h->d_pad, 128)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = make_tmap_bf16(&h->mapH64, h->Hplanes, (uint64_t)3 * h->d_pad, h->d_pad, 64)) != cudaSuccess) { rc = cuda_fail(e); break; }
-        if ((e = dalloc(&h->Hdigits, 4 * pd)) != cudaSuccess) { rc = cuda_fail(e); break; }
-        if ((e = cudaMemsetAsync(h->Hdigits, 0, 4 * pd * 2, st)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = dalloc(&h->Hdig8, 6 * pd)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = cudaMemsetAsync(h->Hdig8, 0, 6 * pd * 2, st)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = dalloc(&h->Hdig10, 4 * pd)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = cudaMemsetAsync(h->Hdig10, 0, 4 * pd * 2, st)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->expo, (size_t)h->G * h->G)) != cudaSuccess) { rc = cuda_fail(e); break; }
-        if ((e = make_tmap_bf16(&h->mapD, h->Hdigits, (uint64_t)4 * h->d_pad, h->d_pad, 64)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = make_tmap_bf16(&h->mapD8, h->Hdig8, (uint64_t)6 * h->d_pad, h->d_pad, 64)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = make_tmap_f16(&h->mapD10, h->Hdig10, (uint64_t)4 * h->d_pad, h->d_pad, 64)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->Lf, (size_t)h->G * group_size * group_size)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->Rinv, (size_t)h->G * group_size * group_size)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = dalloc(&h->Htdig, 4 * pd)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = cudaMemsetAsync(h->Htdig, 0, 4 * pd * 2, st)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = dalloc(&h->expoT, (size_t)h->G * h->G)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = make_tmap_f16(&h->mapHt, h->Htdig, (uint64_t)4 * h->d_pad, h->d_pad, 64)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->dstatus, 1)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = cudaMallocHost((void **)&h->hstatus, sizeof(int))) != cudaSuccess) { rc = cuda_fail(e); break; }
         const float *Hsrc = H;
@@ -348,15 +391,24 @@ jarq_status jarq_prepare_hessian(const float *H, int din, int group_size, float 
         if (e != cudaSuccess) { rc = cuda_fail(e); break; }
         { ProfScope ps("group_factor", st); e = launch_group_factor(h->Hs, h->Lf, h->Rinv, din, group_size, h->dstatus, st); ps.done(); count_launches(1); }
         if (e != cudaSuccess) { rc = cuda_fail(e); break; }
-        { ProfScope ps("slices", st); e = launch_slices(h->Hs, h->expo, h->Hdigits, din, h->d_pad, group_size, st); ps.done(); count_launches(2); }
+        // folded rows R_i^{-T} H[grp i, :] (double-float, temporary) -> digits
+        if ((e = dalloc(&Ht_hi, dd)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = dalloc(&Ht_lo, dd)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        { ProfScope ps("htilde", st); e = launch_htilde(h->Hs, h->Rinv, Ht_hi, Ht_lo, din, group_size, st); ps.done(); count_launches(1); }
+        if (e != cudaSuccess) { rc = cuda_fail(e); break; }
+        { ProfScope ps("slices", st); e = launch_slice10(Ht_hi, Ht_lo, h->expoT, h->Htdig, din, h->d_pad, group_size, st); ps.done(); count_launches(2); }
+        if (e != cudaSuccess) { rc = cuda_fail(e); break; }
+        { ProfScope ps("slices", st); e = launch_slices(h->Hs, h->expo, h->Hdig8, h->Hdig10, din, h->d_pad, group_size, st); ps.done(); count_launches(2); }
         if (e != cudaSuccess) { rc = cuda_fail(e); break; }
         int sb = 0;
         if ((e = read_status(h, st, &sb)) != cudaSuccess) { rc = cuda_fail(e); break; }
         rc = status_from_bits(sb);
     } while (0);
-    if (Hdev) {
+    if (Hdev || Ht_hi || Ht_lo) {
         cudaStreamSynchronize(st);
         cudaFree(Hdev);
+        cudaFree(Ht_hi);
+        cudaFree(Ht_lo);
     }
     if (rc != JARQ_OK) {
         jarq_hessian_destroy(h);
@@ -386,6 +438,24 @@ jarq_status jarq_objective(jarq_hessian *h, const float *W, const float *S, cons
     return status_from_bits(sb);
 }
 
+jarq_status jarq_residual_product(jarq_hessian *h, const float *W, const float *S,
+                                  const uint8_t *Q, const int32_t *Z, int dout, int bits,
+                                  float *HR, void *stream) {
+    if (!layer_args_ok(h, W, S, Q, Z, dout, bits) || (dout > 0 && !HR)) return JARQ_ERR_ARG;
+    if (dout == 0) return JARQ_OK;
+    cudaStream_t st = (cudaStream_t)stream;
+    LayerArgs la;
+    jarq_status rc = layer_front(h, W, S, Q, Z, dout, bits, la, st);
+    if (rc != JARQ_OK) return rc;
+    Workspace &w = h->ws;
+    CK(cudaMemsetAsync(h->dstatus, 0, sizeof(int), st));
+    RUN("hr_full", 1, launch_tc_hr_full(w.mapR, h->mapH128, w.Hr, h->din, dout, w.p_pad, h->din, h->d_pad, h->dstatus, st));
+    CK(cudaMemcpyAsync(HR, w.Hr, (size_t)dout * h->din * sizeof(float), cudaMemcpyDefault, st));
+    int sb = 0;
+    CK(read_status(h, st, &sb));
+    return status_from_bits(sb);
+}
+
 jarq_status jarq_refine_layer(jarq_hessian *h, const float *W, float *S, uint8_t *Q,
                               const int32_t *Z, int dout, int bits, const jarq_options *opt,
                               jarq_stats *stats, void *stream) {
@@ -396,40 +466,51 @@ jarq_status jarq_refine_layer(jarq_hessian *h, const float *W, float *S, uint8_t
     if (dout == 0) return JARQ_OK;
     cudaStream_t st = (cudaStream_t)stream;
     LayerArgs la;
-    jarq_status rc = layer_front(h, W, S, Q, Z, dout, bits, la, st);
+    jarq_status rc = layer_front(h, W, S, Q, Z, dout, bits, la, st, true);
     if (rc != JARQ_OK) return rc;
     Workspace &w = h->ws;
     const int p = dout, d = h->din, g = h->g, G = h->G, qmax = (1 << bits) - 1;
-    RUN("init_rows", 1, launch_init_rows(w.active, w.iters, w.accepted, w.ridge, w.rstat, w.dF_sweep, p, st));
+    RUN("init_rows", 1, launch_init_rows(w.active, w.iters, w.accepted, w.ridge, w.rstat, p, st));
     const ResidualView rv = rview(h);
-    const int nsplit = phase_splits(w.p_pad, h->d_pad);
+    const int nsplit = target_splits(w.p_pad, g, G);
+    // target projection P = W H, w^T H w and the folded Pt, once per call
+    RUN("slice_rows", 1, launch_slice_rows(la.W, w.wdig, w.wexp, p, d, h->d_pad, w.p_pad, g, st));
+    RUN("proj", 1, launch_tc_proj(w.mapWd, h->mapD8, w.Phi, w.Plo, w.wexp, h->expo, p, w.p_pad, d,
+                                  h->d_pad, g, h->dstatus, st));
+    RUN("whw", 1, launch_whw(la.W, w.Phi, w.Plo, w.wHw, p, d, st));
+    RUN("ptilde", 1, launch_ptilde(w.Phi, w.Plo, h->Rinv, w.Pt_hi, w.Pt_lo, p, d, g, st));
     for (int k = 1; k <= o.max_iters; ++k) {
-        RUN("hr_full", 1, launch_tc_hr_full(w.mapR, h->mapH128, w.Hr, d, p, w.p_pad, d, h->d_pad, h->dstatus, st));
-        RUN("grad", 1, launch_grad(la.Q, la.Z, w.r, w.Hr, w.gvec, w.F_start, p, d, g, st));
-        if (k == 1 && stats && stats->L_host)
-            CK(cudaMemcpyAsync(w.L_host, w.F_start, p * sizeof(double), cudaMemcpyDeviceToDevice, st));
-        RUN("gram", 1, launch_tc_gram(w.mapC, h->mapD, la.Q, la.Z, h->expo, w.active, w.gram, p,
+        RUN("gram", 1, launch_tc_gram(w.mapC, h->mapD10, la.Q, la.Z, h->expo, w.active, w.gram, p,
                                       w.p_pad, d, h->d_pad, g, bits, h->dstatus, st));
-        RUN("scale_solve", 1, launch_scale_solve(w.gram, w.gvec, la.W, la.Q, la.Z, w.F_start, la.S, rv,
-                                                 w.L_prev, w.dF_sweep, w.active, w.iters, w.ridge, w.rstat,
-                                                 h->dstatus, p, d, g, k, o, st));
+        RUN("rhs", 1, launch_rhs(la.Q, la.Z, w.Phi, w.Plo, w.active, w.rhs, p, d, g, st));
+        double *L_out = (k == 1 && stats && stats->L_host) ? w.L_host : nullptr;
+        RUN("scale_solve", 1, launch_scale_solve(w.gram, w.rhs, w.wHw, la.S, w.L_prev, L_out,
+                                                 w.active, w.iters, w.ridge, w.rstat, h->dstatus,
+                                                 p, d, g, k, false, o, st));
         for (int i = 0; i < G; ++i) {
-            RUN("phase_hr", 1, launch_tc_hr_phase(w.mapR, h->mapH128, h->mapH64, w.hr, p, w.p_pad, h->d_pad,
-                                                  g, i, nsplit, w.active, h->dstatus, st));
-            RUN("babai", 1, launch_babai(w.hr, nsplit, h->Lf, h->Rinv, la.W, la.S, la.Q, la.Z, rv, w.active,
-                                         w.dF_sweep, w.accepted, h->dstatus, p, g, i, qmax, o.eps, st));
+            RUN("target", 1, launch_tc_target(w.mapC, h->mapHt, w.t_hi, w.t_lo, la.S, h->expoT,
+                                              w.active, p, w.p_pad, h->d_pad, g, G, i, nsplit,
+                                              h->dstatus, st));
+            RUN("babai", 1, launch_babai(w.t_hi, w.t_lo, w.Pt_hi, w.Pt_lo, nsplit, h->Lf, la.S, la.Q,
+                                         la.Z, rv, w.active, w.accepted, h->dstatus, p, g, i, qmax,
+                                         o.eps, st));
         }
     }
+    // objective of the returned state (and of the input state when K = 0)
     const bool want_final = stats && stats->L_final;
     const bool want_host0 = stats && stats->L_host && o.max_iters == 0;
     if (want_final || want_host0) {
-        RUN("hr_full", 1, launch_tc_hr_full(w.mapR, h->mapH128, w.Hr, d, p, w.p_pad, d, h->d_pad, h->dstatus, st));
-        RUN("grad", 1, launch_grad(la.Q, la.Z, w.r, w.Hr, nullptr, w.L_final, p, d, g, st));
+        RUN("gram", 1, launch_tc_gram(w.mapC, h->mapD10, la.Q, la.Z, h->expo, nullptr, w.gram, p,
+                                      w.p_pad, d, h->d_pad, g, bits, h->dstatus, st));
+        RUN("rhs", 1, launch_rhs(la.Q, la.Z, w.Phi, w.Plo, nullptr, w.rhs, p, d, g, st));
+        RUN("scale_solve", 1, launch_scale_solve(w.gram, w.rhs, w.wHw, la.S, w.L_prev, w.L_final,
+                                                 w.active, w.iters, w.ridge, w.rstat, h->dstatus,
+                                                 p, d, g, 0, true, o, st));
         if (want_host0)
             CK(cudaMemcpyAsync(w.L_host, w.L_final, p * sizeof(double), cudaMemcpyDeviceToDevice, st));
     }
     if (la.hS) CK(cudaMemcpyAsync(S, la.S, (size_t)p * G * sizeof(float), cudaMemcpyDeviceToHost, st));
-    if (la.hQ) CK(cudaMemcpyAsync(Q, la.Q, (size_t)p * d, cudaMemcpyDeviceToHost, st));
+    if (la.hQ) CK(cudaMemcpyAsync(Q, la.Q, (size_t)p * d, cudaMemcpyDefault, st));
     if (stats) {
         if (stats->L_host) CK(cudaMemcpyAsync(stats->L_host, w.L_host, p * sizeof(double), cudaMemcpyDefault, st));
         if (stats->L_final) CK(cudaMemcpyAsync(stats->L_final, w.L_final, p * sizeof(double), cudaMemcpyDefault, st));

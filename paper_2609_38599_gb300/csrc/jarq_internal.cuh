@@ -4,6 +4,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <stdint.h>
 
 #include "../../include/jarq.h"
@@ -26,11 +27,11 @@ __host__ __device__ inline int round_up(int x, int m) { return (x + m - 1) / m *
 
 // View of the residual r = w - D_s (q - z): float32 [p][d] plus its exact
 // three-plane bf16 split [3][p_pad][d_pad] read by the tensor cores, and the
-// integer codes c = q - z as bf16 [p_pad][d_pad] (exact for |c| <= 256).
+// integer codes c = q - z as fp16 [p_pad][d_pad] (exact for |c| <= 2048).
 struct ResidualView {
     float *r;
     __nv_bfloat16 *planes;
-    __nv_bfloat16 *cplane;
+    __half *cplane;
     int d, d_pad, p_pad;
 };
 
@@ -46,7 +47,7 @@ __device__ __forceinline__ void split3(float x, __nv_bfloat16 &a, __nv_bfloat16 
 }
 
 __device__ __forceinline__ void store_code(const ResidualView &v, size_t j, int col, int c) {
-    v.cplane[j * v.d_pad + col] = __int2bfloat16_rn(c);
+    v.cplane[j * v.d_pad + col] = __int2half_rn(c);
 }
 
 __device__ __forceinline__ void store_residual(const ResidualView &v, size_t j, int col, float x) {
@@ -63,18 +64,26 @@ __device__ __forceinline__ void store_residual(const ResidualView &v, size_t j, 
 struct Workspace {
     int cap_rows = 0;
     int p_pad = 0;               // rows of the bf16 residual planes (multiple of 128)
-    float *Hr = nullptr;         // [p][d]  H r for every row (start of an iteration)
+    float *Hr = nullptr;         // [p][d]  H r for every row (objective entry point)
     float *r = nullptr;          // [p][d]  residual r = w - D_s (q - z)
-    double *gram = nullptr;      // [p][G][G]  exact Gram matrices
-    double *gvec = nullptr;      // [p][G]  scale gradient g_i = c_i^T (H r)_i
-    float *hr = nullptr;         // [nsplit][p_pad][g]  split-K partials of (H r)_i
+    double *gram = nullptr;      // [p][G][G]  Gram matrices of the current codes
+    double *rhs = nullptr;       // [p][G]  rhs_i = c_i^T P_i (also the scratch of grad)
+    float *t_hi = nullptr;       // [nsplit][p_pad][g]  split-K partials of the phase
+    float *t_lo = nullptr;       //   product T_i (double-float)
     __nv_bfloat16 *rplanes = nullptr;  // [3][p_pad][d_pad] bf16 split of r
-    __nv_bfloat16 *cplane = nullptr;   // [p_pad][d_pad] codes c = q - z
+    __half *cplane = nullptr;          // [p_pad][d_pad] codes c = q - z
     CUtensorMap mapR;            // tensor map of rplanes, 128 x 64 boxes
     CUtensorMap mapC;            // tensor map of cplane, 128 x 64 boxes
-    double *F_start = nullptr;   // [p]  objective at the start of the iteration
-    double *L_prev = nullptr;    // [p]  L^{(k-1)} (stop denominator)
-    double *dF_sweep = nullptr;  // [p]  sum of accepted Babai dF in the current sweep
+    // target projection P = W H (once per call)
+    __nv_bfloat16 *wdig = nullptr;     // [4][p_pad][d_pad] integer digits of W
+    int *wexp = nullptr;               // [p][G] exponents of the digits of W
+    CUtensorMap mapWd;                 // tensor map of wdig, 128 x 64 boxes
+    float *Phi = nullptr;        // [p][d]  P = Phi + Plo (double-float)
+    float *Plo = nullptr;        // [p][d]
+    float *Pt_hi = nullptr;      // [p][d]  folded projection Pt_i = R_i^{-T} P_i
+    float *Pt_lo = nullptr;      // [p][d]
+    double *wHw = nullptr;       // [p]  w_j^T H w_j
+    double *L_prev = nullptr;    // [p]  L^{(k-1)} of the early stop
     double *L_host = nullptr;    // [p]
     double *L_final = nullptr;   // [p]
     int *active = nullptr;       // [p]
@@ -98,12 +107,18 @@ struct jarq_hessian {
     int d_pad = 0;
     float *Hs = nullptr;          // [d][d] symmetrised H (+ nu2 I), fp32
     __nv_bfloat16 *Hplanes = nullptr;  // [3][d_pad][d_pad] exact bf16 split of Hs
-    __nv_bfloat16 *Hdigits = nullptr;  // [4][d_pad][d_pad] per-block integer digits of Hs
+    // per-block integer digits of Hs (block exponents in expo):
+    __nv_bfloat16 *Hdig8 = nullptr;    // [6][d_pad][d_pad] base 2^8, |digit| <= 128
+    __half *Hdig10 = nullptr;          // [4][d_pad][d_pad] base 2^10, |digit| <= 512
     int *expo = nullptr;          // [G][G] block exponents of the digits
     CUtensorMap mapH128, mapH64;  // tensor maps of Hplanes, 128 x 64 and 64 x 64 boxes
-    CUtensorMap mapD;             // tensor map of Hdigits, 64 x 64 boxes
+    CUtensorMap mapD8, mapD10;    // tensor maps of Hdig8 / Hdig10, 64 x 64 boxes
     float *Lf = nullptr;          // [G][g][g] lower factor L_i = R_i^T, row-major
-    float *Rinv = nullptr;        // [G][g][g] R_i^{-1} (upper), row-major
+    double *Rinv = nullptr;       // [G][g][g] R_i^{-1} (upper), row-major, float64
+    // folded rows Ht[grp i, :] = R_i^{-T} H[grp i, :] in the base-2^10 digit scheme
+    __half *Htdig = nullptr;      // [4][d_pad][d_pad] fp16 digits, |digit| <= 512
+    int *expoT = nullptr;         // [G][G] block exponents of Ht
+    CUtensorMap mapHt;            // tensor map of Htdig, 64 x 64 boxes
     int *dstatus = nullptr;       // device status word
     int *hstatus = nullptr;       // pinned host mirror
     jarq::Workspace ws;
@@ -114,8 +129,12 @@ namespace jarq {
 // ---- launchers (each returns the cudaError_t of its launch) ----
 cudaError_t launch_symmetrize(const float *H, float *Hs, __nv_bfloat16 *Hplanes, int d, int d_pad,
                               float nu2, cudaStream_t s);
-cudaError_t launch_group_factor(const float *Hs, float *Lf, float *Rinv, int d, int g,
+cudaError_t launch_group_factor(const float *Hs, float *Lf, double *Rinv, int d, int g,
                                 int *status, cudaStream_t s);
+cudaError_t launch_htilde(const float *Hs, const double *Rinv, float *out_hi, float *out_lo,
+                          int d, int g, cudaStream_t s);
+cudaError_t launch_slice10(const float *hi, const float *lo, int *expo, __half *dig, int d,
+                           int d_pad, int g, cudaStream_t s);
 
 cudaError_t launch_validate(const uint8_t *Q, const int32_t *Z, int p, int d, int G, int qmax,
                             int *status, cudaStream_t s);
@@ -130,21 +149,38 @@ cudaError_t launch_tc_hr_phase(const CUtensorMap &mapA, const CUtensorMap &mapB1
                                cudaStream_t s);
 cudaError_t launch_grad(const uint8_t *Q, const int32_t *Z, const float *r, const float *Hr,
                         double *gvec, double *F, int p, int d, int g, cudaStream_t s);
-cudaError_t launch_slices(const float *Hs, int *expo, __nv_bfloat16 *planes, int d, int d_pad,
-                          int g, cudaStream_t s);
+cudaError_t launch_slices(const float *Hs, int *expo, __nv_bfloat16 *dig8, __half *dig10, int d,
+                          int d_pad, int g, cudaStream_t s);
 cudaError_t launch_tc_gram(const CUtensorMap &mapC, const CUtensorMap &mapS, const uint8_t *Q,
                            const int32_t *Z, const int *expo, const int *active, double *gram,
                            int p, int p_pad, int d, int d_pad, int g, int bits, int *status,
                            cudaStream_t s);
-cudaError_t launch_scale_solve(const double *gram, const double *gvec, const float *W,
-                               const uint8_t *Q, const int32_t *Z, const double *F_start, float *S,
-                               ResidualView rv, double *L_prev, double *dF_sweep, int *active,
+cudaError_t launch_slice_rows(const float *W, __nv_bfloat16 *planes, int *wexp, int p, int d,
+                              int d_pad, int p_pad, int g, cudaStream_t s);
+cudaError_t launch_tc_proj(const CUtensorMap &mapW, const CUtensorMap &mapH, float *Phi,
+                           float *Plo, const int *wexp, const int *hexp, int p, int p_pad, int d,
+                           int d_pad, int g, int *status, cudaStream_t s);
+cudaError_t launch_whw(const float *W, const float *Phi, const float *Plo, double *out, int p,
+                       int d, cudaStream_t s);
+cudaError_t launch_rhs(const uint8_t *Q, const int32_t *Z, const float *Phi, const float *Plo,
+                       const int *active, double *rhs, int p, int d, int g, cudaStream_t s);
+cudaError_t launch_scale_solve(const double *gram, const double *rhs, const double *wHw, float *S,
+                               double *L_prev, double *L_out, int *active,
                                int *iters, int *ridge, int *rstat, int *status, int p, int d,
-                               int g, int k, const jarq_options &o, cudaStream_t s);
-cudaError_t launch_babai(const float *hr, int nsplit, const float *Lf, const float *Rinv,
-                         const float *W, const float *S, uint8_t *Q, const int32_t *Z,
-                         ResidualView rv, const int *active, double *dF_sweep, int *accepted,
-                         int *status, int p, int g, int i, int qmax, float eps, cudaStream_t s);
+                               int g, int k, bool eval_only, const jarq_options &o,
+                               cudaStream_t s);
+cudaError_t launch_babai(const float *t_hi, const float *t_lo, const float *pt_hi,
+                         const float *pt_lo, int nsplit, const float *Lf, const float *S,
+                         uint8_t *Q, const int32_t *Z, ResidualView rv, const int *active,
+                         int *accepted, int *status, int p, int g, int i, int qmax, float eps,
+                         cudaStream_t s);
+cudaError_t launch_ptilde(const float *Phi, const float *Plo, const double *Rinv, float *out_hi,
+                          float *out_lo, int p, int d, int g, cudaStream_t s);
+int target_splits(int p_pad, int g, int G);
+cudaError_t launch_tc_target(const CUtensorMap &mapC, const CUtensorMap &mapT, float *out_hi,
+                             float *out_lo, const float *S, const int *expoT, const int *active,
+                             int p, int p_pad, int d_pad, int g, int G, int i, int nsplit,
+                             int *status, cudaStream_t s);
 
 // Launch with programmatic stream serialization: the kernel may start while
 // the previous kernel in the stream finishes; it must call griddepcontrol.wait
@@ -165,7 +201,7 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
     return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
 }
 cudaError_t launch_init_rows(int *active, int *iters, int *accepted, int *ridge, int *rstat,
-                             double *dF_sweep, int p, cudaStream_t s);
+                             int p, cudaStream_t s);
 
 int num_sms();
 

@@ -3,11 +3,15 @@
 // babai_update; App. E "Small scales").
 //
 // One warp per output row; lane owns the NT = g/32 consecutive coordinates
-// l = NT*lane .. NT*lane + NT - 1.  The group factors L_i = R_i^T and
-// R_i^{-1} are staged in shared memory.
+// l = NT*lane .. NT*lane + NT - 1.  The group factor L_i = R_i^T is staged in
+// shared memory.
 //
-// The recursion is evaluated relative to the row's current codes q:
-// with (H r)_i from the phase product and y = R_i^{-T} (H r)_i / s,
+// The recursion is evaluated relative to the row's current codes q.  The
+// target y = R_i^{-T} (H r)_i / s is formed in double-float as
+// (Pt_i - T_i) / s: Pt_i = R_i^{-T} (H w)_i from the folded target projection
+// and T_i = sum_h s_h R_i^{-T} H_ih c_h from the phase product (split-K
+// partials), so that the cancellation of H's low-rank part costs no
+// precision.  Then
 //     v = R_i^{-T} [(H r)_i + s H_ii c] / s = y + R_i c,   c = q - z,
 // so the pre-round value of Eq. babai_update is
 //     z + x_l = q_l + (y_l - sum_{h>l} R_lh Delta_h) / R_ll,
@@ -31,15 +35,15 @@ namespace {
 constexpr int kMaxWarps = 32;   // warps per block (one row each) at most
 
 struct BabaiArgs {
-    const float *hr;      // [nsplit][p_pad][g]
+    const float *t_hi, *t_lo;    // [nsplit][p_pad][g] split-K partials of T_i
+    const float *pt_hi, *pt_lo;  // [p][d] folded target projection Pt
     int nsplit;
-    const float *Lf, *Rinv;
-    const float *W, *S;
+    const float *Lf;
+    const float *S;
     uint8_t *Q;
     const int32_t *Z;
     ResidualView rv;
     const int *active;
-    double *dF_sweep;
     int *accepted;
     int *status;
     int p, g, i, qmax;
@@ -65,21 +69,18 @@ __global__ void __launch_bounds__(32 * kMaxWarps) babai_kernel(BabaiArgs a) {
     constexpr int g = 32 * NT;
     extern __shared__ __align__(16) float smem[];
     float *Lg = smem;                 // [g][g] lower factor of group i
-    float *Rg = smem + g * g;         // [g][g] R_i^{-1}
-    float *rdiag = Rg + g * g;        // [g] 1 / R_ll
-    float *hbuf = rdiag + g;          // [warps][g] this warp's (H r)_i row
+    float *rdiag = Lg + g * g;        // [g] 1 / R_ll
     __shared__ uint64_t bar;
     __shared__ int load_ok;
     const int d = a.rv.d, G = d / g;
-    // group factors of group i: two bulk copies (they do not depend on the
-    // previous kernel, so they overlap its tail under programmatic launch)
+    // group factor of group i: one bulk copy (it does not depend on the
+    // previous kernel, so it overlaps that kernel's tail under programmatic
+    // launch)
     if (threadIdx.x == 0) {
         tc::mbar_init(tc::smem_u32(&bar), 1);
         tc::fence_barrier_init();
-        tc::mbar_expect_tx(tc::smem_u32(&bar), 2u * g * g * sizeof(float));
+        tc::mbar_expect_tx(tc::smem_u32(&bar), (uint32_t)(g * g * sizeof(float)));
         tc::bulk_load(tc::smem_u32(Lg), a.Lf + (size_t)a.i * g * g, g * g * sizeof(float),
-                      tc::smem_u32(&bar));
-        tc::bulk_load(tc::smem_u32(Rg), a.Rinv + (size_t)a.i * g * g, g * g * sizeof(float),
                       tc::smem_u32(&bar));
         load_ok = tc::mbar_wait(tc::smem_u32(&bar), 0) ? 1 : 0;
     }
@@ -95,7 +96,6 @@ __global__ void __launch_bounds__(32 * kMaxWarps) babai_kernel(BabaiArgs a) {
     tc::pdl_wait();
     tc::pdl_launch_dependents();
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
-    float *hrow = hbuf + wid * g;
     const int l0 = NT * lane;
     const int col0 = a.i * g;
     float rd[NT];
@@ -106,14 +106,26 @@ __global__ void __launch_bounds__(32 * kMaxWarps) babai_kernel(BabaiArgs a) {
         if (!(fabsf(s) > a.eps)) continue;  // small-scale skip (also NaN)
         const int z = a.Z[(size_t)j * G + a.i];
         const size_t off = (size_t)j * d + col0;
-        float hv[NT];
-        load_vec<NT>(a.hr + (size_t)j * g + l0, hv);
-        for (int sp = 1; sp < a.nsplit; ++sp) {
-            float t2[NT];
-            load_vec<NT>(a.hr + ((size_t)sp * a.rv.p_pad + j) * g + l0, t2);
+        // s y = Pt_i - sum_sp T_sp, in double-float
+        float y[NT], yl[NT];
+        load_vec<NT>(a.pt_hi + off + l0, y);
+        load_vec<NT>(a.pt_lo + off + l0, yl);
+        for (int sp = 0; sp < a.nsplit; ++sp) {
+            float th[NT], tl[NT];
+            const size_t o = ((size_t)sp * a.rv.p_pad + j) * g + l0;
+            load_vec<NT>(a.t_hi + o, th);
+            load_vec<NT>(a.t_lo + o, tl);
 #pragma unroll
-            for (int t = 0; t < NT; ++t) hv[t] += t2[t];
+            for (int t = 0; t < NT; ++t) {
+                const float sm = y[t] - th[t];
+                const float bb = sm - y[t];
+                const float e = (y[t] - (sm - bb)) + (-th[t] - bb);
+                y[t] = sm;
+                yl[t] += e - tl[t];
+            }
         }
+#pragma unroll
+        for (int t = 0; t < NT; ++t) y[t] += yl[t];
         float qc[NT], qn[NT];   // current and proposed codes (small integers, exact)
         {
             uint32_t packed = 0;
@@ -128,25 +140,7 @@ __global__ void __launch_bounds__(32 * kMaxWarps) babai_kernel(BabaiArgs a) {
                 qn[t] = qc[t];
             }
         }
-        __syncwarp();
-#pragma unroll
-        for (int t = 0; t < NT; ++t) hrow[l0 + t] = hv[t];
-        __syncwarp();
-        // y = R^{-T} (H r)_i / s :  y_l = sum_{m <= l} Rinv[m][l] hr_m
-        float y[NT];
-#pragma unroll
-        for (int t = 0; t < NT; ++t) y[t] = 0.f;
-        for (int m = 0; m < g; m += 4) {
-            const float4 h4 = *reinterpret_cast<const float4 *>(hrow + m);
-            const float hm[4] = {h4.x, h4.y, h4.z, h4.w};
-#pragma unroll
-            for (int mm = 0; mm < 4; ++mm) {
-                float rr[NT];
-                load_vec<NT>(Rg + (m + mm) * g + l0, rr);
-#pragma unroll
-                for (int t = 0; t < NT; ++t) y[t] = fmaf(rr[t], hm[mm], y[t]);
-            }
-        }
+        // y = R^{-T} (H r)_i / s
         float u[NT];
 #pragma unroll
         for (int t = 0; t < NT; ++t) {
@@ -206,24 +200,22 @@ __global__ void __launch_bounds__(32 * kMaxWarps) babai_kernel(BabaiArgs a) {
                 const int l = l0 + t;
                 const int qi = (int)qn[t];
                 a.Q[off + l] = (uint8_t)qi;
-                store_residual(a.rv, j, col0 + l, fmaf(-s, (float)(qi - z), a.W[off + l]));
                 store_code(a.rv, j, col0 + l, qi - z);
             }
         }
-        if (lane == 0) {
-            a.dF_sweep[j] += (double)dF;
-            a.accepted[j] += 1;
-        }
+        if (lane == 0) a.accepted[j] += 1;
     }
 }
 
 }  // namespace
 
-cudaError_t launch_babai(const float *hr, int nsplit, const float *Lf, const float *Rinv,
-                         const float *W, const float *S, uint8_t *Q, const int32_t *Z,
-                         ResidualView rv, const int *active, double *dF_sweep, int *accepted,
-                         int *status, int p, int g, int i, int qmax, float eps, cudaStream_t s) {
-    BabaiArgs a{hr, nsplit, Lf, Rinv, W, S, Q, Z, rv, active, dF_sweep, accepted, status, p, g, i, qmax, eps};
+cudaError_t launch_babai(const float *t_hi, const float *t_lo, const float *pt_hi,
+                         const float *pt_lo, int nsplit, const float *Lf, const float *S,
+                         uint8_t *Q, const int32_t *Z, ResidualView rv, const int *active,
+                         int *accepted, int *status, int p, int g, int i, int qmax, float eps,
+                         cudaStream_t s) {
+    BabaiArgs a{t_hi, t_lo, pt_hi, pt_lo, nsplit, Lf, S, Q, Z, rv, active, accepted, status,
+                p, g, i, qmax, eps};
     // one block per SM, one warp per row: spread the rows evenly over the SMs
     const int nsm = num_sms();
     int warps = (p + nsm - 1) / nsm;
@@ -231,7 +223,7 @@ cudaError_t launch_babai(const float *hr, int nsplit, const float *Lf, const flo
     if (warps < 1) warps = 1;
     int blocks = (p + warps - 1) / warps;
     if (blocks > nsm) blocks = nsm;
-    const size_t smem = ((size_t)2 * g * g + g + (size_t)warps * g) * sizeof(float);
+    const size_t smem = ((size_t)g * g + g) * sizeof(float);
     cudaError_t e = cudaSuccess;
     if (g == 128) {
         e = cudaFuncSetAttribute(babai_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

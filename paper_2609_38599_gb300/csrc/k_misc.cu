@@ -22,7 +22,8 @@ __global__ void validate_kernel(const uint8_t *__restrict__ Q, const int32_t *__
     if (threadIdx.x == 0 && flag) atomicOr(status, flag);
 }
 
-// r = w - s (q - z), one rounding (fma) per element (Eq. quantized_group).
+// r = w - s (q - z), one rounding (fma) per element (Eq. quantized_group),
+// and the code plane c = q - z; with rv.r == nullptr only the code plane.
 __global__ void residual_kernel(const float *__restrict__ W, const float *__restrict__ S,
                                 const uint8_t *__restrict__ Q, const int32_t *__restrict__ Z,
                                 ResidualView rv, int p, int g) {
@@ -33,13 +34,13 @@ __global__ void residual_kernel(const float *__restrict__ W, const float *__rest
         const size_t j = idx / d;
         const int grp = (int)(idx - j * d) / g;
         const int ci = (int)Q[idx] - Z[j * G + grp];
-        store_residual(rv, j, (int)(idx - j * d), fmaf(-S[j * G + grp], (float)ci, W[idx]));
+        if (rv.r) store_residual(rv, j, (int)(idx - j * d), fmaf(-S[j * G + grp], (float)ci, W[idx]));
         store_code(rv, j, (int)(idx - j * d), ci);
     }
 }
 
 __global__ void init_rows_kernel(int *active, int *iters, int *accepted, int *ridge, int *rstat,
-                                 double *dF_sweep, int p) {
+                                 int p) {
     int j = blockIdx.x * blockDim.x + threadIdx.x;
     if (j < p) {
         active[j] = 1;
@@ -47,7 +48,6 @@ __global__ void init_rows_kernel(int *active, int *iters, int *accepted, int *ri
         accepted[j] = 0;
         ridge[j] = 0;
         rstat[j] = 0;
-        dF_sweep[j] = 0.0;
     }
 }
 
@@ -85,9 +85,8 @@ cudaError_t launch_residual(const float *W, const float *S, const uint8_t *Q, co
 }
 
 cudaError_t launch_init_rows(int *active, int *iters, int *accepted, int *ridge, int *rstat,
-                             double *dF_sweep, int p, cudaStream_t s) {
-    init_rows_kernel<<<(p + 255) / 256, 256, 0, s>>>(active, iters, accepted, ridge, rstat,
-                                                      dF_sweep, p);
+                             int p, cudaStream_t s) {
+    init_rows_kernel<<<(p + 255) / 256, 256, 0, s>>>(active, iters, accepted, ridge, rstat, p);
     return cudaGetLastError();
 }
 

@@ -1,13 +1,21 @@
-// Hessian preparation: symmetrisation and per-group Cholesky factors.
+// Hessian preparation: symmetrisation, per-group Cholesky factors and the
+// folded operand of the sweep's residual products.
 //
 // Sec. 3.3.2, Eq. group_qr: each group's factor R_i (A_i = U_i R_i) is
 // computed once per layer and reused for every output row and iteration.
 // With H = A^T A, R_i^T R_i = H_ii, so R_i is taken as the upper Cholesky
 // factor of H_ii (equal to the QR factor up to row signs, to which the
 // Babai recursion is invariant).  The factor and its inverse are computed in
-// float64 in shared memory and stored as float32:
-//   Lf[i]   = L_i = R_i^T          (lower, row-major: Lf[l][m] = R_i[m][l])
-//   Rinv[i] = R_i^{-1}             (upper, row-major)
+// float64 in shared memory:
+//   Lf[i]   = L_i = R_i^T          (lower, row-major: Lf[l][m] = R_i[m][l]), float32
+//   Rinv[i] = R_i^{-1}             (upper, row-major), float64
+// The Babai target of Eq. babai_update needs y = R_i^{-T} (H r)_i / s.  The
+// rows H_i of group i are dominated by the low-rank part of H, which R_i^{-T}
+// cancels: forming (H r)_i first and applying R_i^{-T} afterwards amplifies
+// the product's rounding by up to sqrt(cond(H_ii)).  The sweep therefore
+// works with the folded rows
+//   Ht[grp i, :] = R_i^{-T} H[grp i, :]
+// computed here once, in double-float (hi + lo) from the float64 inverse.
 #include "jarq_internal.cuh"
 
 namespace jarq {
@@ -45,7 +53,7 @@ __global__ void symmetrize_kernel(const float *__restrict__ H, float *__restrict
 // One block per group: float64 Cholesky of H_ii in shared memory, then an
 // in-place inverse of the lower factor.
 __global__ void group_factor_kernel(const float *__restrict__ Hs, float *__restrict__ Lf,
-                                    float *__restrict__ Rinv, int d, int g, int *status) {
+                                    double *__restrict__ Rinv, int d, int g, int *status) {
     extern __shared__ double smem[];
     const int ld = g + 1;
     double *A = smem;               // [g][g+1]
@@ -108,10 +116,69 @@ __global__ void group_factor_kernel(const float *__restrict__ Hs, float *__restr
         __syncthreads();
     }
     // Rinv = (L^{-1})^T : Rinv[m][l] = Linv[l][m]
-    float *Ri = Rinv + (size_t)grp * g * g;
+    double *Ri = Rinv + (size_t)grp * g * g;
     for (int idx = tid; idx < g * g; idx += nt) {
         int m = idx / g, l = idx % g;
-        Ri[idx] = (l >= m) ? (float)A[l * ld + m] : 0.f;
+        Ri[idx] = (l >= m) ? A[l * ld + m] : 0.0;
+    }
+}
+
+// (s, e) with s + e = a + b exactly
+__device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
+    s = a + b;
+    const float bb = s - a;
+    e = (a - (s - bb)) + (b - bb);
+}
+
+// Ht[i g + a, k] = sum_{b <= a} Rinv_i[b][a] Hs[i g + b, k] for one group i
+// (blockIdx.y) and 64 columns k (blockIdx.x): Rinv_i as float pairs (hi, lo)
+// and the H tile in shared memory, double-float accumulation, written as the
+// float pair (hi, lo) [d][d].
+constexpr int kHtCols = 64;
+
+__global__ void __launch_bounds__(256) htilde_kernel(const float *__restrict__ Hs,
+                                                     const double *__restrict__ Rinv,
+                                                     float *__restrict__ out_hi,
+                                                     float *__restrict__ out_lo, int d, int g) {
+    extern __shared__ float hsm[];
+    float *rh = hsm;                   // [g][g] hi parts, Rinv[b][a] at b * g + a
+    float *rl = rh + g * g;            // [g][g] lo parts
+    float *ht = rl + g * g;            // [g][kHtCols] rows of H for this group
+    const int i = blockIdx.y, k0 = blockIdx.x * kHtCols;
+    const int tid = threadIdx.x;
+    const double *Ri = Rinv + (size_t)i * g * g;
+    for (int idx = tid; idx < g * g; idx += blockDim.x) {
+        const double v = Ri[idx];
+        const float hi = (float)v;
+        rh[idx] = hi;
+        rl[idx] = (float)(v - (double)hi);
+    }
+    for (int idx = tid; idx < g * kHtCols; idx += blockDim.x) {
+        const int b = idx / kHtCols, kk = idx % kHtCols;
+        ht[idx] = (k0 + kk < d) ? Hs[(size_t)(i * g + b) * d + k0 + kk] : 0.f;
+    }
+    __syncthreads();
+    const int kk = tid % kHtCols, a0 = tid / kHtCols, astep = blockDim.x / kHtCols;
+    for (int a = a0; a < g; a += astep) {
+        float sh = 0.f, sl = 0.f;
+        for (int b = 0; b <= a; ++b) {
+            const float hv = ht[b * kHtCols + kk];
+            const float r_hi = rh[b * g + a], r_lo = rl[b * g + a];
+            const float m = r_hi * hv;
+            float e = fmaf(r_hi, hv, -m);
+            e = fmaf(r_lo, hv, e);
+            float s2, e2;
+            two_sum(sh, m, s2, e2);
+            sh = s2;
+            sl += e2 + e;
+        }
+        if (k0 + kk < d) {
+            float s2, e2;
+            two_sum(sh, sl, s2, e2);
+            const size_t off = (size_t)(i * g + a) * d + k0 + kk;
+            out_hi[off] = s2;
+            out_lo[off] = e2;
+        }
     }
 }
 
@@ -124,13 +191,24 @@ cudaError_t launch_symmetrize(const float *H, float *Hs, __nv_bfloat16 *Hplanes,
     return cudaGetLastError();
 }
 
-cudaError_t launch_group_factor(const float *Hs, float *Lf, float *Rinv, int d, int g,
+cudaError_t launch_group_factor(const float *Hs, float *Lf, double *Rinv, int d, int g,
                                 int *status, cudaStream_t s) {
     size_t smem = (size_t)(g * (g + 1) + g) * sizeof(double);
     cudaError_t e = cudaFuncSetAttribute(group_factor_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     group_factor_kernel<<<d / g, 256, smem, s>>>(Hs, Lf, Rinv, d, g, status);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_htilde(const float *Hs, const double *Rinv, float *out_hi, float *out_lo,
+                          int d, int g, cudaStream_t s) {
+    const size_t smem = ((size_t)2 * g * g + (size_t)g * kHtCols) * sizeof(float);
+    cudaError_t e = cudaFuncSetAttribute(htilde_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    dim3 grid((d + kHtCols - 1) / kHtCols, d / g);
+    htilde_kernel<<<grid, 256, smem, s>>>(Hs, Rinv, out_hi, out_lo, d, g);
     return cudaGetLastError();
 }
 

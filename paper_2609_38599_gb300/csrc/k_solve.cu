@@ -1,26 +1,24 @@
 // Joint scale solve, one warp per output row (Sec. 3.3.1; App. E).
 //
 // For each active row j the warp
-//  1. symmetrises its G x G Gram matrix (App. E "Solving for scales");
-//  2. factors it by Cholesky in float32 (the paper solves this system in
-//     FP32).  A pivot at or below rcond * max(max diag, eps), a nonfinite
-//     entry or a failed factorisation adds ridge * I and retries once; a
-//     second failure marks the row numerical and keeps its state;
+//  1. symmetrises its G x G Gram matrix (App. E "Solving for scales") and
+//     forms, in float64, the gradient g = rhs - Gram s_old of the current
+//     scales (rhs_i = c_i^T P_i from the target projection) and the
+//     objective F(s_old) = wHw - s_old^T (rhs + g);
+//  2. factors the Gram matrix by Cholesky in float32 (the paper solves this
+//     system in FP32).  A pivot at or below rcond * max(max diag, eps), a
+//     nonfinite entry or a failed factorisation adds ridge * I and retries
+//     once; a second failure marks the row numerical and keeps its state;
 //  3. solves the normal equations of Eq. scale_normal_equations for the
-//     increment of the scales (float32 Cholesky, then two refinement steps
-//     whose residuals are formed in float64 from the exact Gram matrix): with
-//     rhs = B^T y and the gradient
-//     g = rhs - Gram s_old, whose entries are g_i = c_i^T (H r)_i at the
-//     current state, Gram s_new = rhs  <=>  Gram (s_new - s_old) = g.  With the
-//     ridge, (Gram + lambda I) s_new = rhs  <=>  (Gram + lambda I) delta =
-//     g - lambda s_old.  g comes from a direct product with the residual, so
-//     the solve's rounding only touches the (small) increment;
-//  4. updates the bookkeeping for the early stop of Eq. strict_stopping:
-//     the objective change at fixed codes is
-//     dF_scale = -2 delta^T g + delta^T Gram delta, L^{(k)} = F(s_old) + dF_scale,
-//     and L^{(k-1)} - L^{(k)} = -(accepted Babai dF of sweep k-1) - dF_scale
-//     is formed from small terms only;
-//  5. rewrites the row's residual r = w - D_s (q - z) for the new scales.
+//     increment of the scales: Gram s_new = rhs <=> Gram (s_new - s_old) = g,
+//     and with the ridge (Gram + lambda I) delta = g - lambda s_old (float32
+//     Cholesky, then two refinement steps whose residuals are formed in
+//     float64), and stores s_new rounded to float32;
+//  4. evaluates L^{(k)} = F(s_new) = wHw - 2 s_new^T rhs + s_new^T Gram s_new
+//     at the stored float32 scales and applies the early stop of Eq.
+//     strict_stopping against L^{(k-1)}.
+// In evaluation mode it only writes F(s) of the current state, for every
+// row.
 #include <float.h>
 
 #include "jarq_internal.cuh"
@@ -62,20 +60,17 @@ __device__ __forceinline__ float warp_max(float v) {
 }
 
 struct SolveArgs {
-    const double *gram, *gvec;
-    const float *W;
-    const uint8_t *Q;
-    const int32_t *Z;
-    const double *F_start;
+    const double *gram, *rhs, *wHw;
     float *S;
-    ResidualView rv;
-    double *L_prev, *dF_sweep;
+    double *L_prev;
+    double *L_out;       // optional: F(s_old) of every processed row
     int *active, *iters, *ridge, *rstat, *status;
     int p, d, g, k;
+    bool eval_only;
     jarq_options o;
 };
 
-// Per-warp shared memory: float A[G][G+1], s_old[G], work[G]; double rhs[G], inc[G].
+// Per-warp shared memory: float A[G][G+1], s_old[G], work[G]; double g[G], inc[G].
 __host__ __device__ inline size_t solve_warp_bytes(int G) {
     size_t f = (size_t)G * (G + 1) + 2 * (size_t)G;
     f = (f + 1) & ~(size_t)1;   // 8-byte alignment of the double part
@@ -107,7 +102,7 @@ __global__ void scale_solve_kernel(SolveArgs a) {
     const int G = a.d / a.g, ld = G + 1;
     const int wpb = blockDim.x >> 5, w = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int j = blockIdx.x * wpb + w;
-    if (j >= a.p || !a.active[j]) return;  // warp-uniform
+    if (j >= a.p || (!a.eval_only && !a.active[j])) return;  // warp-uniform
     unsigned char *base = smem_raw + (size_t)w * solve_warp_bytes(G);
     float *A = (float *)base;
     float *so = A + G * ld;         // s_old
@@ -117,7 +112,24 @@ __global__ void scale_solve_kernel(SolveArgs a) {
     double *b = (double *)(base + fcount * sizeof(float));   // gradient g
     double *inc = b + G;                                      // increment of the scales
     const double *gj = a.gram + (size_t)j * G * G;
+    const double *rj = a.rhs + (size_t)j * G;
     auto gsym = [&](int r0, int c0) { return 0.5 * (gj[r0 * G + c0] + gj[c0 * G + r0]); };
+    for (int t = lane; t < G; t += 32) so[t] = a.S[(size_t)j * G + t];
+    __syncwarp();
+    // gradient g = rhs - Gram s_old and F(s_old) = wHw - s_old^T (rhs + g)
+    bool bfin = true;
+    double fs = 0.0;
+    for (int r0 = lane; r0 < G; r0 += 32) {
+        double gs = 0.0;
+        for (int c0 = 0; c0 < G; ++c0) gs = fma(gsym(r0, c0), (double)so[c0], gs);
+        const double gr = rj[r0] - gs;
+        b[r0] = gr;
+        fs += (double)so[r0] * (rj[r0] + gr);
+        bfin &= (bool)isfinite(gr);
+    }
+    const double F_old = a.wHw[j] - warp_sum(fs);
+    if (a.L_out && lane == 0) a.L_out[j] = F_old;
+    if (a.eval_only) return;
     auto load_sym = [&](float shift) -> bool {
         bool finite = true;
         for (int idx = lane; idx < G * G; idx += 32) {
@@ -130,12 +142,6 @@ __global__ void scale_solve_kernel(SolveArgs a) {
         __syncwarp();
         return __all_sync(0xffffffffu, finite);
     };
-    bool bfin = true;
-    for (int t = lane; t < G; t += 32) {
-        b[t] = a.gvec[(size_t)j * G + t];
-        so[t] = a.S[(size_t)j * G + t];
-        bfin &= (bool)isfinite(b[t]);
-    }
     bool finite = load_sym(0.f);
     float md = 0.f;
     for (int t = lane; t < G; t += 32) md = fmaxf(md, A[t * ld + t]);
@@ -184,51 +190,39 @@ __global__ void scale_solve_kernel(SolveArgs a) {
         fail();
         return;
     }
-    // objective bookkeeping with the unridged symmetrised Gram matrix
+    for (int t = lane; t < G; t += 32) y[t] = (float)((double)so[t] + inc[t]);   // s_new
+    __syncwarp();
+    // L^{(k)} at the stored float32 scales, from the unridged symmetrised Gram
     double t1 = 0.0, t2 = 0.0;
     for (int r0 = lane; r0 < G; r0 += 32) {
-        double gdl = 0.0;
-        for (int c0 = 0; c0 < G; ++c0) gdl = fma(gsym(r0, c0), inc[c0], gdl);
-        t1 += inc[r0] * b[r0];
-        t2 += inc[r0] * gdl;
+        double gs = 0.0;
+        for (int c0 = 0; c0 < G; ++c0) gs = fma(gsym(r0, c0), (double)y[c0], gs);
+        t1 += (double)y[r0] * rj[r0];
+        t2 += (double)y[r0] * gs;
     }
-    t1 = warp_sum(t1);
-    t2 = warp_sum(t2);
-    const double dF_scale = -2.0 * t1 + t2;
-    const double L_new = a.F_start[j] + dF_scale;
+    const double L_new = a.wHw[j] - 2.0 * warp_sum(t1) + warp_sum(t2);
     bool stop = false;
     if (a.o.early_stop && a.k >= 2) {
-        const double dec = -(a.dF_sweep[j] + dF_scale);
+        const double dec = a.L_prev[j] - L_new;
         const double den = fmax(fabs(a.L_prev[j]), (double)a.o.eps);
         stop = (dec / den <= (double)a.o.tau_rel) || (fabs(dec) <= (double)a.o.tau_abs);
     }
-    for (int t = lane; t < G; t += 32) y[t] = (float)((double)so[t] + inc[t]);   // s_new
-    __syncwarp();
     for (int t = lane; t < G; t += 32) a.S[(size_t)j * G + t] = y[t];
     if (lane == 0) {
         a.L_prev[j] = L_new;
-        a.dF_sweep[j] = 0.0;
         a.iters[j] = a.k;
         a.ridge[j] += used_ridge;
         if (stop) a.active[j] = 0;
-    }
-    // residual for the new scales
-    const size_t rowoff = (size_t)j * a.d;
-    const int32_t *zj = a.Z + (size_t)j * G;
-    for (int c0 = lane; c0 < a.d; c0 += 32) {
-        const int grp = c0 / a.g;
-        const float c = (float)((int)a.Q[rowoff + c0] - zj[grp]);
-        store_residual(a.rv, j, c0, fmaf(-y[grp], c, a.W[rowoff + c0]));
     }
 }
 
 }  // namespace
 
-cudaError_t launch_scale_solve(const double *gram, const double *gvec, const float *W,
-                               const uint8_t *Q, const int32_t *Z, const double *F_start, float *S,
-                               ResidualView rv, double *L_prev, double *dF_sweep, int *active,
+cudaError_t launch_scale_solve(const double *gram, const double *rhs, const double *wHw, float *S,
+                               double *L_prev, double *L_out, int *active,
                                int *iters, int *ridge, int *rstat, int *status, int p, int d,
-                               int g, int k, const jarq_options &o, cudaStream_t s) {
+                               int g, int k, bool eval_only, const jarq_options &o,
+                               cudaStream_t s) {
     const int G = d / g;
     const size_t per_warp = solve_warp_bytes(G);
     int wpb = (int)((96 * 1024) / per_warp);
@@ -238,8 +232,8 @@ cudaError_t launch_scale_solve(const double *gram, const double *gvec, const flo
     cudaError_t e = cudaFuncSetAttribute(scale_solve_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    SolveArgs a{gram, gvec, W, Q, Z, F_start, S, rv, L_prev, dF_sweep, active, iters, ridge, rstat,
-                status, p, d, g, k, o};
+    SolveArgs a{gram, rhs, wHw, S, L_prev, L_out, active, iters, ridge, rstat,
+                status, p, d, g, k, eval_only, o};
     scale_solve_kernel<<<(p + wpb - 1) / wpb, 32 * wpb, smem, s>>>(a);
     return cudaGetLastError();
 }

@@ -1,18 +1,20 @@
-// Exact Gram matrices of the joint scale fit on the tensor cores.
+// Gram matrices of the joint scale fit on the tensor cores, exact for the
+// digit representation of H.
 //
 // Sec. 3.3.1, Eq. scale_design: Gram_j[i,h] = (A_i c_i)^T (A_h c_h)
 // = c_i^T H_ih c_h with integer codes c = q - z.  Each g x g block H_ih is
-// written as 2^(E_ih - 7) * sum_t a_t 2^(-8 t), t = 0..3, with integer
-// digits |a_t| <= 128 (exact in bf16) and E_ih the block's exponent, so
+// written as 2^(E_ih - 9) * sum_t a_t 2^(-10 t), t = 0..3, with integer
+// digits |a_t| <= 512 (exact in fp16) and E_ih the block's exponent
+// (max |H_ih| <= 2^E_ih), which represents every entry to within
+// 2^(E_ih - 40).  The codes are fp16 as well (|c| <= 255), so
 //     D_t[j, m] = sum_{k in grp h} c_j[k] a_t[k, m]
-// is an integer of at most 23 bits: every tensor-core partial sum is exact
-// whatever the accumulator's rounding.  The epilogue forms the integer dots
-// G_t = sum_{m in grp i} c_j[m] D_t[j, m] and
-//     Gram_j[i,h] = 2^(E_ih - 7) (G_0 + G_1 2^-8 + G_2 2^-16 + G_3 2^-24)
-// in float64, exactly for the digit-represented block (whose error is at
-// most 2^(E_ih - 32) per entry).  Only h <= i is computed; the block is
-// mirrored.  A CTA owns one 128-row tile and the group pair {i, G-1-i}, so
-// every CTA processes G + 1 blocks.
+// is an integer below 128 * 255 * 512 < 2^24: every tensor-core partial sum
+// is exact whatever the accumulator's rounding.  The epilogue forms the
+// integer dots G_t = sum_{m in grp i} c_j[m] D_t[j, m] and
+//     Gram_j[i,h] = 2^(E_ih - 9) (G_0 + G_1 2^-10 + G_2 2^-20 + G_3 2^-30)
+// in float64.  Only h <= i is computed; the block is mirrored.  A CTA owns
+// one 128-row tile and the group pair {i, G-1-i}, so every CTA processes
+// G + 1 blocks.
 //
 // Roles: warp 0 TMA producer; warp 1 TMEM allocation and MMA issuer;
 // warps 2..5 epilogue (TMEM lanes 32 (w % 4) ..).  One unit of work is
@@ -23,19 +25,19 @@
 namespace jarq {
 namespace {
 
-constexpr int kTileA = 128 * 64 * 2;   // 128 code rows x 64 K
-constexpr int kTileB = 64 * 64 * 2;    // 64 H rows x 64 K, one digit plane
+constexpr int kTileA = 128 * 64 * 2;   // 128 code rows x 64 K (fp16)
+constexpr int kTileB = 64 * 64 * 2;    // 64 H rows x 64 K, one digit plane (fp16)
 constexpr int kStage = kTileA + 4 * kTileB;
 constexpr int kStages = 3;
 constexpr int kCodesBytes = 128 * 128 * 2;  // int16 codes of group i for the tile
 constexpr int kSmem = 1024 + kStages * kStage + kCodesBytes + 256;
-constexpr uint32_t kIdesc = tc::idesc_bf16_f32(128, 64);
+constexpr uint32_t kIdesc = tc::idesc_f16_f32(128, 64);
 
 struct GramArgs {
     const uint8_t *Q;
     const int32_t *Z;
     const int *expo;     // [G][G] block exponents E_ih
-    const int *active;
+    const int *active;   // optional: rows whose Gram matrix is needed
     double *gram;        // [p][G][G]
     int *status;
     int p, d, g, G, d_pad;
@@ -46,8 +48,9 @@ __device__ __forceinline__ int exact_int(float x) {
     return __float_as_int(x + 12582912.0f) - 0x4B400000;
 }
 
-// WIDE: 64-bit integer dots (codes wider than 4 bits); otherwise every
-// per-slice dot of 64 terms fits in 32 bits (|c| <= 15, |D_t| < 2^18).
+// WIDE: codes wider than 4 bits, |D_t| < 2^24 converted by cvt and 64-bit
+// integer dots; otherwise |c| <= 15, |D_t| < 2^20 and every partial dot of
+// 8 terms fits in 32 bits.
 template <bool WIDE>
 __global__ void __launch_bounds__(192, 1)
     tc_gram_kernel(const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapS,
@@ -65,7 +68,8 @@ __global__ void __launch_bounds__(192, 1)
 
     {
         int mine = 0;
-        if (threadIdx.x < 128 && j0 + (int)threadIdx.x < a.p) mine = a.active[j0 + threadIdx.x];
+        if (threadIdx.x < 128 && j0 + (int)threadIdx.x < a.p)
+            mine = a.active ? a.active[j0 + threadIdx.x] : 1;
         if (!__syncthreads_or(mine)) return;
     }
     // groups handled by this CTA and the unit list: for each group i (h = 0..i,
@@ -230,10 +234,10 @@ __global__ void __launch_bounds__(192, 1)
                         long long p0 = 0, p1 = 0, p2 = 0, p3 = 0;
 #pragma unroll
                         for (int e = 0; e < 16; e += 2) {
-                            p0 += (long long)cr[e] * exact_int(__uint_as_float(v0[e]));
-                            p1 += (long long)cr[e + 1] * exact_int(__uint_as_float(v0[e + 1]));
-                            p2 += (long long)cr[16 + e] * exact_int(__uint_as_float(v1[e]));
-                            p3 += (long long)cr[17 + e] * exact_int(__uint_as_float(v1[e + 1]));
+                            p0 += (long long)cr[e] * __float2int_rn(__uint_as_float(v0[e]));
+                            p1 += (long long)cr[e + 1] * __float2int_rn(__uint_as_float(v0[e + 1]));
+                            p2 += (long long)cr[16 + e] * __float2int_rn(__uint_as_float(v1[e]));
+                            p3 += (long long)cr[17 + e] * __float2int_rn(__uint_as_float(v1[e + 1]));
                         }
                         acc[t] += (p0 + p1) + (p2 + p3);
                     } else {
@@ -255,9 +259,9 @@ __global__ void __launch_bounds__(192, 1)
             if (half == nhalf - 1) {
                 if (row < a.p) {
                     const int E = a.expo[gi * G + h];
-                    const double v = ldexp((double)acc[0] + ldexp((double)acc[1], -8) +
-                                               ldexp((double)acc[2], -16) + ldexp((double)acc[3], -24),
-                                           E - 7);
+                    const double v = ldexp((double)acc[0] + ldexp((double)acc[1], -10) +
+                                               ldexp((double)acc[2], -20) + ldexp((double)acc[3], -30),
+                                           E - 9);
                     double *gr = a.gram + (size_t)row * G * G;
                     gr[(size_t)gi * G + h] = v;
                     gr[(size_t)h * G + gi] = v;
@@ -300,10 +304,15 @@ __global__ void block_exponent_kernel(const float *__restrict__ Hs, int *__restr
     }
 }
 
-// Digits a_t of every entry: x = H 2^(7 - E) in [-128, 128], a_0 = rint(x),
-// a_t = rint(256 (remainder)), four planes [4][d_pad][d_pad].
+// Digits of every entry of H for the two integer-digit schemes, from the
+// block exponent E (max |H_blk| <= 2^E):
+//  * dig8 (bf16, six planes, target projection): x = H 2^(7 - E) in
+//    [-128, 128], a_0 = rint(x), a_t = rint(256 * remainder);
+//  * dig10 (fp16, four planes, Gram): x = H 2^(9 - E) in [-512, 512],
+//    a_0 = rint(x), a_t = rint(1024 * remainder).
 __global__ void slice_kernel(const float *__restrict__ Hs, const int *__restrict__ expo,
-                             __nv_bfloat16 *__restrict__ planes, int d, int d_pad, int g) {
+                             __nv_bfloat16 *__restrict__ dig8, __half *__restrict__ dig10, int d,
+                             int d_pad, int g) {
     const int G = d / g;
     const size_t n = (size_t)d * d;
     const size_t plane = (size_t)d_pad * d_pad;
@@ -311,21 +320,69 @@ __global__ void slice_kernel(const float *__restrict__ Hs, const int *__restrict
          idx += (size_t)gridDim.x * blockDim.x) {
         const int r = (int)(idx / d), c = (int)(idx % d);
         const int E = expo[(r / g) * G + c / g];
-        float x = ldexpf(Hs[idx], 7 - E);
         const size_t off = (size_t)r * d_pad + c;
+        float x = ldexpf(Hs[idx], 7 - E);
+#pragma unroll
+        for (int t = 0; t < 6; ++t) {
+            const float dgt = rintf(x);
+            dig8[t * plane + off] = __float2bfloat16_rn(dgt);
+            x = (x - dgt) * 256.f;
+        }
+        x = ldexpf(Hs[idx], 9 - E);
 #pragma unroll
         for (int t = 0; t < 4; ++t) {
             const float dgt = rintf(x);
-            planes[t * plane + off] = __float2bfloat16_rn(dgt);
-            x = (x - dgt) * 256.f;
+            dig10[t * plane + off] = __float2half_rn(dgt);
+            x = (x - dgt) * 1024.f;
+        }
+    }
+}
+
+// Digits of a double-float matrix M = hi + lo (not necessarily symmetric) in
+// the Gram scheme: x = M 2^(9 - E) in [-512, 512] with E the block exponent,
+// four fp16 planes base 2^10.  The low part enters before the remainder is
+// scaled, so the digits represent hi + lo to 2^(E - 40).
+__global__ void slice10_kernel(const float *__restrict__ hi, const float *__restrict__ lo,
+                               const int *__restrict__ expo, __half *__restrict__ dig, int d,
+                               int d_pad, int g) {
+    const int G = d / g;
+    const size_t n = (size_t)d * d;
+    const size_t plane = (size_t)d_pad * d_pad;
+    for (size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x; idx < n;
+         idx += (size_t)gridDim.x * blockDim.x) {
+        const int r = (int)(idx / d), c = (int)(idx % d);
+        const int E = expo[(r / g) * G + c / g];
+        const size_t off = (size_t)r * d_pad + c;
+        float x = ldexpf(hi[idx], 9 - E);
+        const float xl = ldexpf(lo[idx], 9 - E);
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+            const float dgt = rintf(x);
+            dig[t * plane + off] = __float2half_rn(dgt);
+            x = x - dgt;
+            if (t == 0) x += xl;
+            x *= 1024.f;
         }
     }
 }
 
 }  // namespace
 
-cudaError_t launch_slices(const float *Hs, int *expo, __nv_bfloat16 *planes, int d, int d_pad,
-                          int g, cudaStream_t s) {
+cudaError_t launch_slice10(const float *hi, const float *lo, int *expo, __half *dig, int d,
+                           int d_pad, int g, cudaStream_t s) {
+    const int G = d / g;
+    block_exponent_kernel<<<dim3(G, G), 256, 0, s>>>(hi, expo, d, g);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    size_t n = (size_t)d * d;
+    int blocks = (int)((n + 255) / 256);
+    if (blocks > 16 * num_sms()) blocks = 16 * num_sms();
+    slice10_kernel<<<blocks, 256, 0, s>>>(hi, lo, expo, dig, d, d_pad, g);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_slices(const float *Hs, int *expo, __nv_bfloat16 *dig8, __half *dig10, int d,
+                          int d_pad, int g, cudaStream_t s) {
     const int G = d / g;
     block_exponent_kernel<<<dim3(G, G), 256, 0, s>>>(Hs, expo, d, g);
     cudaError_t e = cudaGetLastError();
@@ -333,7 +390,7 @@ cudaError_t launch_slices(const float *Hs, int *expo, __nv_bfloat16 *planes, int
     size_t n = (size_t)d * d;
     int blocks = (int)((n + 255) / 256);
     if (blocks > 16 * num_sms()) blocks = 16 * num_sms();
-    slice_kernel<<<blocks, 256, 0, s>>>(Hs, expo, planes, d, d_pad, g);
+    slice_kernel<<<blocks, 256, 0, s>>>(Hs, expo, dig8, dig10, d, d_pad, g);
     return cudaGetLastError();
 }
 

@@ -32,12 +32,19 @@ namespace jarq {
 namespace {
 
 constexpr int kTileA = 128 * 64 * 2;  // bytes of one 128 x 64 bf16 A tile
-constexpr int kProducts = 6;
-constexpr int kPeriod = 2;            // 64-wide K chunks per drain period
+constexpr int kProducts = 8;
+constexpr int kPeriod = 1;            // 64-wide K chunks per drain period
 constexpr int kGroupRows = 8;         // row tiles per band in the full-product tile order
-// (A plane, B plane) of each product; product 5 = (0, 0) is the leading one.
-__host__ __device__ constexpr int prod_a(int k) { return k == 0 ? 2 : k == 1 ? 1 : k == 3 ? 1 : 0; }
-__host__ __device__ constexpr int prod_b(int k) { return k == 2 ? 2 : k == 1 ? 1 : k == 4 ? 1 : 0; }
+// (A plane, B plane) of each product, smallest first; the last, (0, 0), is
+// the leading one.
+__host__ __device__ constexpr int prod_a(int k) {
+    constexpr int t[8] = {2, 1, 2, 1, 0, 1, 0, 0};
+    return t[k];
+}
+__host__ __device__ constexpr int prod_b(int k) {
+    constexpr int t[8] = {1, 2, 0, 1, 2, 0, 1, 0};
+    return t[k];
+}
 
 struct HrArgs {
     float *out;            // output tile base (split 0)

@@ -1,0 +1,479 @@
+// Target projection P = W H on the tensor cores, exact to double-float
+// accuracy, and the quantities derived from it.  For the main target the
+// reduced target is R W, so the right-hand side of Eq.
+// scale_normal_equations is rhs_j[i] = c_i^T P_j[grp i] with P_j = H w_j
+// (App. G "Computational Complexity", the target-projection shortcut), and
+// the objective is F_j = w_j^T H w_j - 2 s^T rhs_j + s^T Gram_j s.
+//
+// Both operands are written in integer digits so that every tensor-core
+// partial sum is exact:
+//   W[j, k] = 2^(ew(j,h) - 7) sum_{t<4} a_t 2^(-8t),  k in group h, one exponent
+//             per (row, group) with max |W[j, grp h]| <= 2^ew;
+//   H[k, m] = 2^(E(h,n) - 7) sum_{u<6} b_u 2^(-8u),   the block exponent of
+//             block (h, n), n = the group of m,
+// with |a_t|, |b_u| <= 128 (exact in bf16).  Four digits hold every float32 W
+// entry within 2^7 of its group maximum exactly, six every H entry within
+// 2^24 of its block maximum.  For each group h of K the eighteen digit
+// products with t + u <= 5 accumulate in six TMEM "levels" l = t + u; a
+// level sums at most 4 x 128 products of 14-bit integers per output, an
+// exact integer below 2^23.  The epilogue combines the levels in
+// double-float (pairs of float32), applies 2^(ew + E - 14) and adds the
+// group's contribution to a double-float accumulator.  The dropped products
+// (t + u >= 6) are below 2^-48 of the block scales.
+//
+// Roles: warp 0 TMA producer (4 W planes + 6 H planes per 64-wide K chunk),
+// warp 1 TMEM allocation and MMA issue, warps 2..9 drain (warp w reads TMEM
+// lanes 32 (w % 4) and 32 of the tile's 64 columns).  Tile 128 x 64; the six
+// levels take 384 TMEM columns, single-buffered: the drain warps release
+// them as soon as their loads have landed and combine from registers while
+// the next group's products run.
+#include "tc_common.cuh"
+
+namespace jarq {
+namespace {
+
+constexpr int kWDig = 4, kHDig = 6, kLevels = 6;
+constexpr int kTileA = 128 * 64 * 2;   // one W digit plane, 128 rows x 64 K
+constexpr int kTileB = 64 * 64 * 2;    // one H digit plane, 64 rows x 64 K
+constexpr int kStage = kWDig * kTileA + kHDig * kTileB;
+constexpr int kStages = 2;
+constexpr int kSmem = 1024 + kStages * kStage + 256;
+constexpr uint32_t kIdesc = tc::idesc_bf16_f32(128, 64);
+constexpr int kGroupRows = 8;
+
+struct ProjArgs {
+    float *Phi, *Plo;    // [p][d] double-float result
+    const int *wexp;     // [p][G] row-group exponents of W
+    const int *hexp;     // [G][G] block exponents of H
+    int *status;
+    int p, d, g, G, w_plane, h_plane;   // rows between digit planes in the two maps
+};
+
+// (s, e) with s + e = a + b exactly
+__device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
+    s = a + b;
+    const float bb = s - a;
+    e = (a - (s - bb)) + (b - bb);
+}
+
+__global__ void __launch_bounds__(320, 1)
+    tc_proj_kernel(const __grid_constant__ CUtensorMap mapW, const __grid_constant__ CUtensorMap mapH,
+                   ProjArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint64_t *bars = (uint64_t *)(smem + kStages * kStage);
+    uint32_t *tmem_slot = (uint32_t *)(bars + 2 * kStages + 2);
+    volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // grouped tile order: bands of kGroupRows row tiles sweep all column tiles
+    const int lin = blockIdx.y * gridDim.x + blockIdx.x;
+    const int per_band = kGroupRows * gridDim.y;
+    const int band = lin / per_band, in_band = lin % per_band;
+    const int rows_in_band = min(kGroupRows, (int)gridDim.x - band * kGroupRows);
+    const int j0 = (band * kGroupRows + in_band % rows_in_band) * 128;
+    const int n0 = (in_band / rows_in_band) * 64;
+    const int nkc = a.g / 64;               // K chunks per group
+    const int nseg = a.G;                   // K segments = groups
+    const int nchunks = nseg * nkc;
+    const int hblk = n0 / a.g;              // column group of the tile (a 64-wide tile lies in one)
+
+    auto full = [&](int s) { return tc::smem_u32(bars + s); };
+    auto empty = [&](int s) { return tc::smem_u32(bars + kStages + s); };
+    const uint32_t afull = tc::smem_u32(bars + 2 * kStages);
+    const uint32_t aempty = tc::smem_u32(bars + 2 * kStages + 1);
+    auto tileA = [&](int s, int t) { return tc::smem_u32(smem + s * kStage + t * kTileA); };
+    auto tileB = [&](int s, int u) {
+        return tc::smem_u32(smem + s * kStage + kWDig * kTileA + u * kTileB);
+    };
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            tc::mbar_init(full(s), 1);
+            tc::mbar_init(empty(s), 1);
+        }
+        tc::mbar_init(afull, 1);
+        tc::mbar_init(aempty, 8);
+        *abort_flag = 0;
+        tc::fence_barrier_init();
+    }
+    if (warp == 1) {
+        tc::tmem_alloc(tc::smem_u32(tmem_slot), 512);
+        tc::tmem_relinquish();
+    }
+    if (warp == 0 && lane == 0) {
+        tc::prefetch_tmap(&mapW);
+        tc::prefetch_tmap(&mapH);
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0 && lane == 0) {
+        // ---------------- producer
+        int issued = 0;
+        for (int c = 0; c < nchunks; ++c) {
+            const int s = c % kStages;
+            if (!tc::mbar_wait(empty(s), ((c / kStages) & 1) ^ 1) || *abort_flag) {
+                *abort_flag = 1;
+                break;
+            }
+            const int k = c * 64;
+            tc::mbar_expect_tx(full(s), kStage);
+#pragma unroll
+            for (int t = 0; t < kWDig; ++t)
+                tc::tma_load_2d(tileA(s, t), &mapW, full(s), k, t * a.w_plane + j0);
+#pragma unroll
+            for (int u = 0; u < kHDig; ++u)
+                tc::tma_load_2d(tileB(s, u), &mapH, full(s), k, u * a.h_plane + n0);
+            issued = c + 1;
+        }
+        // do not leave with copies in flight
+        for (int c = issued > kStages ? issued - kStages : 0; c < issued; ++c)
+            if (!tc::mbar_wait(full(c % kStages), (c / kStages) & 1)) *abort_flag = 1;
+    } else if (warp == 1 && lane == 0) {
+        // ---------------- MMA issuer
+        for (int sg = 0; sg < nseg && !*abort_flag; ++sg) {
+            if (!tc::mbar_wait(aempty, (sg & 1) ^ 1)) {
+                *abort_flag = 1;
+                break;
+            }
+            tc::tc_fence_after();
+            for (int kc = 0; kc < nkc; ++kc) {
+                const int c = sg * nkc + kc;
+                const int s = c % kStages;
+                if (!tc::mbar_wait(full(s), (c / kStages) & 1) || *abort_flag) {
+                    *abort_flag = 1;
+                    break;
+                }
+                tc::tc_fence_after();
+#pragma unroll
+                for (int sub = 0; sub < 4; ++sub) {
+#pragma unroll
+                    for (int t = 0; t < kWDig; ++t) {
+                        const uint64_t ad = tc::sdesc_sw128(tileA(s, t)) + 2 * sub;
+#pragma unroll
+                        for (int u = 0; u < kHDig; ++u) {
+                            if (t + u >= kLevels) continue;
+                            const uint64_t bd = tc::sdesc_sw128(tileB(s, u)) + 2 * sub;
+                            // the product (0, l) opens level l of the group
+                            const uint32_t acc = (kc | sub | t) != 0;
+                            tc::mma_bf16(tmem + (t + u) * 64, ad, bd, kIdesc, acc);
+                        }
+                    }
+                }
+                tc::mma_commit(empty(s));
+            }
+            tc::mma_commit(afull);
+        }
+    } else if (warp >= 2) {
+        // ---------------- drain: levels -> double-float per group -> accumulator
+        const int q = warp & 3, half = (warp - 2) >> 2;
+        const int row = j0 + 32 * q + lane;
+        float hi[32], lo[32];
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+            hi[e] = 0.f;
+            lo[e] = 0.f;
+        }
+        bool ok = true;
+        const uint32_t base = tmem + ((uint32_t)(32 * q) << 16) + half * 32;
+        for (int sg = 0; sg < nseg; ++sg) {
+            bool w = tc::mbar_wait(afull, sg & 1);
+            w = __shfl_sync(0xffffffffu, w && !*abort_flag, 0);
+            tc::tc_fence_after();
+            if (!w) {
+                ok = false;
+                *abort_flag = 1;
+                break;
+            }
+            const int ew = row < a.p ? a.wexp[(size_t)row * a.G + sg] : 0;
+            const int eh = hblk < a.G ? a.hexp[sg * a.G + hblk] : 0;
+            const float scale = ldexpf(1.0f, ew + eh - 14);
+            // value of the group = sum_l L_l 2^(-8 l), as (vh, vl), 32 columns
+            float vh[32], vl[32];
+#pragma unroll
+            for (int l = 0; l < kLevels; ++l) {
+                uint32_t x[32];
+                tc::tmem_ld32(base + l * 64, x);
+                tc::tmem_wait_ld();
+                if (l == kLevels - 1) {
+                    // every level is in registers: hand the columns back
+                    tc::tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) tc::mbar_arrive(aempty);
+                }
+                const float f = ldexpf(1.0f, -8 * l);
+#pragma unroll
+                for (int e = 0; e < 32; ++e) {
+                    const float v = __uint_as_float(x[e]) * f;   // exact (power of two)
+                    if (l == 0) {
+                        vh[e] = v;
+                        vl[e] = 0.f;
+                    } else {
+                        float s2, e2;
+                        two_sum(vh[e], v, s2, e2);
+                        vh[e] = s2;
+                        vl[e] += e2;
+                    }
+                }
+            }
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+                float s2, e2;
+                two_sum(hi[e], vh[e] * scale, s2, e2);
+                hi[e] = s2;
+                lo[e] += e2 + vl[e] * scale;
+            }
+        }
+        if (ok && row < a.p) {
+            const int ncol = n0 + half * 32;
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+                const int col = ncol + e;
+                if (col < a.d) {
+                    float s2, e2;
+                    two_sum(hi[e], lo[e], s2, e2);
+                    a.Phi[(size_t)row * a.d + col] = s2;
+                    a.Plo[(size_t)row * a.d + col] = e2;
+                }
+            }
+        }
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc::tc_fence_after();
+        tc::tmem_dealloc(tmem, 512);
+    }
+    if (threadIdx.x == 0 && *abort_flag) atomicOr(a.status, ST_TIMEOUT);
+}
+
+// Digits of W per (row, group): x = W 2^(7 - ew) in [-128, 128] with
+// max |W[j, grp h]| <= 2^ew; a_0 = rint(x), a_t = rint(256 * remainder).
+// One warp per (row, group).
+__global__ void slice_rows_kernel(const float *__restrict__ W, __nv_bfloat16 *__restrict__ planes,
+                                  int *__restrict__ wexp, int p, int d, int d_pad, int p_pad, int g) {
+    const int G = d / g;
+    const long long warp = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (warp >= (long long)p * G) return;
+    const int j = (int)(warp / G), h = (int)(warp % G);
+    const float *src = W + (size_t)j * d + (size_t)h * g;
+    float mx = 0.f;
+    for (int m = lane; m < g; m += 32) mx = fmaxf(mx, fabsf(src[m]));
+    for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    int e = 0;
+    if (mx > 0.f) frexpf(mx, &e);
+    if (lane == 0) wexp[(size_t)j * G + h] = e;
+    const size_t plane = (size_t)p_pad * d_pad;
+    for (int m = lane; m < g; m += 32) {
+        float x = ldexpf(src[m], 7 - e);
+        const size_t off = (size_t)j * d_pad + (size_t)h * g + m;
+#pragma unroll
+        for (int t = 0; t < kWDig; ++t) {
+            const float dg = rintf(x);
+            planes[t * plane + off] = __float2bfloat16_rn(dg);
+            x = (x - dg) * 256.f;
+        }
+    }
+}
+
+// Exact product c * (ph + pl) added to the double-float (sh, sl): c is a small
+// integer, so c * ph splits exactly by one fma.
+__device__ __forceinline__ void df_axpy(float c, float ph, float pl, float &sh, float &sl) {
+    const float m = c * ph;
+    const float me = fmaf(c, ph, -m);
+    float s2, e2;
+    two_sum(sh, m, s2, e2);
+    sh = s2;
+    sl += e2 + fmaf(c, pl, me);
+}
+
+__device__ __forceinline__ void df_warp_sum(float &sh, float &sl) {
+    for (int o = 16; o; o >>= 1) {
+        const float oh = __shfl_xor_sync(0xffffffffu, sh, o);
+        const float ol = __shfl_xor_sync(0xffffffffu, sl, o);
+        float s2, e2;
+        two_sum(sh, oh, s2, e2);
+        sh = s2;
+        sl += e2 + ol;
+    }
+}
+
+// rhs_j[i] = sum_{l in grp i} (q_l - z_i) P_j[l], one warp per row, lane owns
+// NT = g/32 consecutive entries of every group.
+template <int NT>
+__global__ void rhs_kernel(const uint8_t *__restrict__ Q, const int32_t *__restrict__ Z,
+                           const float *__restrict__ Phi, const float *__restrict__ Plo,
+                           const int *__restrict__ active, double *__restrict__ rhs, int p, int d) {
+    constexpr int g = 32 * NT;
+    const int G = d / g;
+    const int j = (int)(((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+    const int lane = threadIdx.x & 31;
+    if (j >= p || (active && !active[j])) return;   // warp-uniform
+    const size_t off = (size_t)j * d + NT * lane;
+    for (int i = 0; i < G; ++i) {
+        const float z = (float)Z[(size_t)j * G + i];
+        const size_t o = off + (size_t)i * g;
+        float ph[NT], pl[NT], qc[NT];
+        if constexpr (NT == 4) {
+            const float4 a4 = *reinterpret_cast<const float4 *>(Phi + o);
+            const float4 b4 = *reinterpret_cast<const float4 *>(Plo + o);
+            const uint32_t q4 = *reinterpret_cast<const uint32_t *>(Q + o);
+            ph[0] = a4.x; ph[1] = a4.y; ph[2] = a4.z; ph[3] = a4.w;
+            pl[0] = b4.x; pl[1] = b4.y; pl[2] = b4.z; pl[3] = b4.w;
+#pragma unroll
+            for (int t = 0; t < 4; ++t) qc[t] = (float)((q4 >> (8 * t)) & 0xFFu);
+        } else {
+            const float2 a2 = *reinterpret_cast<const float2 *>(Phi + o);
+            const float2 b2 = *reinterpret_cast<const float2 *>(Plo + o);
+            const uint32_t q2 = *reinterpret_cast<const uint16_t *>(Q + o);
+            ph[0] = a2.x; ph[1] = a2.y;
+            pl[0] = b2.x; pl[1] = b2.y;
+            qc[0] = (float)(q2 & 0xFFu);
+            qc[1] = (float)(q2 >> 8);
+        }
+        float sh = 0.f, sl = 0.f;
+#pragma unroll
+        for (int t = 0; t < NT; ++t) df_axpy(qc[t] - z, ph[t], pl[t], sh, sl);
+        df_warp_sum(sh, sl);
+        if (lane == 0) rhs[(size_t)j * G + i] = (double)sh + (double)sl;
+    }
+}
+
+// wHw_j = sum_k W[j,k] P[j,k] with P = Phi + Plo, double-float per lane, one
+// warp per row.
+__global__ void whw_kernel(const float *__restrict__ W, const float *__restrict__ Phi,
+                           const float *__restrict__ Plo, double *__restrict__ out, int p, int d) {
+    const int j = (int)(((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+    const int lane = threadIdx.x & 31;
+    if (j >= p) return;
+    const size_t off = (size_t)j * d;
+    float sh = 0.f, sl = 0.f;
+    for (int k = lane; k < d; k += 32) {
+        const float w = W[off + k], ph = Phi[off + k], pl = Plo[off + k];
+        const float m = w * ph;
+        const float me = fmaf(w, ph, -m);
+        float s2, e2;
+        two_sum(sh, m, s2, e2);
+        sh = s2;
+        sl += e2 + fmaf(w, pl, me);
+    }
+    df_warp_sum(sh, sl);
+    if (lane == 0) out[j] = (double)sh + (double)sl;
+}
+
+// Folded target projection Pt_j[grp i] = R_i^{-T} P_j[grp i], i.e.
+// Pt[j, i g + a] = sum_{b <= a} Rinv_i[b][a] P[j, i g + b], in double-float
+// from the float64 inverse and the double-float P.  One CTA per (64 rows,
+// group i); Rinv_i and the rows' P slice in shared memory.
+constexpr int kPtRows = 64;
+
+__global__ void __launch_bounds__(256) ptilde_kernel(const float *__restrict__ Phi,
+                                                     const float *__restrict__ Plo,
+                                                     const double *__restrict__ Rinv,
+                                                     float *__restrict__ out_hi,
+                                                     float *__restrict__ out_lo, int p, int d,
+                                                     int g) {
+    extern __shared__ float psm[];
+    float *rh = psm;                   // [g][g] Rinv[b][a] at b * g + a
+    float *rl = rh + g * g;
+    float *ph = rl + g * g;            // [kPtRows][g]
+    float *pl = ph + kPtRows * g;
+    const int i = blockIdx.y, r0 = blockIdx.x * kPtRows;
+    const int tid = threadIdx.x;
+    const double *Ri = Rinv + (size_t)i * g * g;
+    for (int idx = tid; idx < g * g; idx += blockDim.x) {
+        const double v = Ri[idx];
+        const float hv = (float)v;
+        rh[idx] = hv;
+        rl[idx] = (float)(v - (double)hv);
+    }
+    for (int idx = tid; idx < kPtRows * g; idx += blockDim.x) {
+        const int jj = idx / g, b = idx % g;
+        const bool in = r0 + jj < p;
+        const size_t o = (size_t)(r0 + jj) * d + (size_t)i * g + b;
+        ph[idx] = in ? Phi[o] : 0.f;
+        pl[idx] = in ? Plo[o] : 0.f;
+    }
+    __syncthreads();
+    const int a = tid % g, jstep = blockDim.x / g;
+    for (int jj = tid / g; jj < kPtRows; jj += jstep) {
+        if (r0 + jj >= p) break;
+        float sh = 0.f, sl = 0.f;
+        for (int b = 0; b <= a; ++b) {
+            const float xh = rh[b * g + a], xl = rl[b * g + a];
+            const float yh = ph[jj * g + b], yl = pl[jj * g + b];
+            const float m = xh * yh;
+            float e = fmaf(xh, yh, -m);
+            e = fmaf(xh, yl, fmaf(xl, yh, e));
+            float s2, e2;
+            two_sum(sh, m, s2, e2);
+            sh = s2;
+            sl += e2 + e;
+        }
+        float s2, e2;
+        two_sum(sh, sl, s2, e2);
+        const size_t o = (size_t)(r0 + jj) * d + (size_t)i * g + a;
+        out_hi[o] = s2;
+        out_lo[o] = e2;
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_ptilde(const float *Phi, const float *Plo, const double *Rinv, float *out_hi,
+                          float *out_lo, int p, int d, int g, cudaStream_t s) {
+    const size_t smem = ((size_t)2 * g * g + (size_t)2 * kPtRows * g) * sizeof(float);
+    cudaError_t e = cudaFuncSetAttribute(ptilde_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    dim3 grid((p + kPtRows - 1) / kPtRows, d / g);
+    ptilde_kernel<<<grid, 256, smem, s>>>(Phi, Plo, Rinv, out_hi, out_lo, p, d, g);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_slice_rows(const float *W, __nv_bfloat16 *planes, int *wexp, int p, int d,
+                              int d_pad, int p_pad, int g, cudaStream_t s) {
+    const long long warps = (long long)p * (d / g);
+    slice_rows_kernel<<<(unsigned)((warps * 32 + 255) / 256), 256, 0, s>>>(W, planes, wexp, p, d,
+                                                                          d_pad, p_pad, g);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_tc_proj(const CUtensorMap &mapW, const CUtensorMap &mapH, float *Phi,
+                           float *Plo, const int *wexp, const int *hexp, int p, int p_pad, int d,
+                           int d_pad, int g, int *status, cudaStream_t s) {
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(tc_proj_kernel,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    ProjArgs a{Phi, Plo, wexp, hexp, status, p, d, g, d / g, p_pad, d_pad};
+    dim3 grid(p_pad / 128, d_pad / 64, 1);
+    tc_proj_kernel<<<grid, 320, kSmem, s>>>(mapW, mapH, a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_whw(const float *W, const float *Phi, const float *Plo, double *out, int p,
+                       int d, cudaStream_t s) {
+    whw_kernel<<<(unsigned)(((long long)p * 32 + 255) / 256), 256, 0, s>>>(W, Phi, Plo, out, p, d);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_rhs(const uint8_t *Q, const int32_t *Z, const float *Phi, const float *Plo,
+                       const int *active, double *rhs, int p, int d, int g, cudaStream_t s) {
+    const unsigned blocks = (unsigned)(((long long)p * 32 + 255) / 256);
+    if (g == 128)
+        rhs_kernel<4><<<blocks, 256, 0, s>>>(Q, Z, Phi, Plo, active, rhs, p, d);
+    else if (g == 64)
+        rhs_kernel<2><<<blocks, 256, 0, s>>>(Q, Z, Phi, Plo, active, rhs, p, d);
+    else
+        return cudaErrorInvalidValue;
+    return cudaGetLastError();
+}
+
+}  // namespace jarq

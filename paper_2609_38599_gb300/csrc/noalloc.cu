@@ -23,7 +23,7 @@ namespace {
 // Largest padded layer (rows rounded up to 128 times input width rounded up
 // to 128) this entry point accepts.
 constexpr size_t kNoAllocMaxElems = (size_t)1 << 20;
-// r (f32) + residual planes (3 x bf16) + code plane (bf16) + H r (f32), each
+// r (f32) + residual planes (3 x bf16) + code plane (fp16) + H r (f32), each
 // region padded to 256 bytes.
 constexpr size_t kRegionR = kNoAllocMaxElems * 4;
 constexpr size_t kRegionPlanes = kNoAllocMaxElems * 2 * 3;
@@ -104,7 +104,7 @@ extern "C" jarq_status jarq_objective_noalloc(jarq_hessian *h, const float *W, c
     unsigned char *base = (unsigned char *)g_scratch_ptr[h->device];
     float *r = (float *)base;
     __nv_bfloat16 *planes = (__nv_bfloat16 *)(base + kRegionR);
-    __nv_bfloat16 *cplane = (__nv_bfloat16 *)(base + kRegionR + kRegionPlanes);
+    __half *cplane = (__half *)(base + kRegionR + kRegionPlanes);
     float *Hr = (float *)(base + kRegionR + kRegionPlanes + kRegionCodes);
     CUtensorMap mapR;
     if (!encode_planes_map(&mapR, planes, (uint64_t)3 * p_pad, d_pad)) return JARQ_ERR_CUDA;

@@ -10,7 +10,8 @@ namespace {
 
 const char *const kNames[] = {"validate", "residual", "init_rows", "hr_full", "grad", "gram",
                               "scale_solve", "phase_hr", "babai", "symmetrize", "group_factor",
-                              "slices"};
+                              "slices", "slice_rows", "proj", "whw", "rhs", "htilde", "ptilde",
+                              "target"};
 constexpr int kNumNames = sizeof(kNames) / sizeof(kNames[0]);
 
 struct Pending {

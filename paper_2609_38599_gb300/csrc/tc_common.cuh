@@ -142,6 +142,13 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
            | ((uint32_t)(M >> 4) << 24);    // M >> 4
 }
 
+// The same with fp16 x fp16 operands (A and B formats 0 = F16).
+__host__ __device__ constexpr uint32_t idesc_f16_f32(int M, int N) {
+    return (1u << 4)                        // D format: F32
+           | ((uint32_t)(N >> 3) << 17)     // N >> 3
+           | ((uint32_t)(M >> 4) << 24);    // M >> 4
+}
+
 // Shared-memory matrix descriptor of a K-major tile written by TMA with
 // 128-byte swizzle: rows of 128 bytes (64 bf16), 8-row atoms 1024 bytes apart.
 __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {

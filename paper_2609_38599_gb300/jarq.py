@@ -30,7 +30,7 @@ EXPORTS = ("jarq_default_options", "jarq_prepare_hessian", "jarq_refine_layer",
            "jarq_objective", "jarq_hessian_din", "jarq_hessian_group_size",
            "jarq_hessian_destroy", "jarq_status_string", "jarq_profile_enable",
            "jarq_profile_reset", "jarq_profile_read", "jarq_launch_count",
-           "jarq_objective_noalloc")
+           "jarq_objective_noalloc", "jarq_residual_product")
 
 
 class JarqError(RuntimeError):
@@ -69,6 +69,8 @@ def _load():
     lib.jarq_objective.argtypes = [vp, vp, vp, vp, vp, ci, ci, vp, vp]
     lib.jarq_objective_noalloc.restype = ci
     lib.jarq_objective_noalloc.argtypes = [vp, vp, vp, vp, vp, ci, ci, vp, vp]
+    lib.jarq_residual_product.restype = ci
+    lib.jarq_residual_product.argtypes = [vp, vp, vp, vp, vp, ci, ci, vp, vp]
     lib.jarq_hessian_din.restype = ci
     lib.jarq_hessian_din.argtypes = [vp]
     lib.jarq_hessian_group_size.restype = ci
@@ -98,7 +100,8 @@ def library():
 
 
 KERNELS = ("validate", "residual", "init_rows", "hr_full", "grad", "gram", "scale_solve",
-           "phase_hr", "babai", "symmetrize", "group_factor", "slices")
+           "phase_hr", "babai", "symmetrize", "group_factor", "slices", "slice_rows", "proj",
+           "whw", "rhs", "htilde", "ptilde", "target")
 
 
 def profile_enable(on: bool = True):
@@ -243,6 +246,24 @@ def refine(hess: Hessian, W, S, Q, Z, bits: int, options: Options = None,
     if raise_on_error and status not in (JARQ_OK,):
         raise JarqError(status, "jarq_refine_layer")
     return st if st is not None else status
+
+
+def residual_product(hess: Hessian, W, S, Q, Z, bits: int, out=None):
+    """``jarq_residual_product``: H r of every row (float32, dout x din), from
+    the tensor-core kernel of the sweep's residual products."""
+    dout, din = int(W.shape[0]), int(W.shape[1])
+    if out is None:
+        if _is_torch(W):
+            import torch
+            out = torch.empty(dout, din, dtype=torch.float32, device=W.device)
+        else:
+            out = np.empty((dout, din), dtype=np.float32)
+    status = _lib.jarq_residual_product(hess.handle, _ptr(W, np.float32), _ptr(S, np.float32),
+                                        _ptr(Q, np.uint8), _ptr(Z, np.int32), dout, int(bits),
+                                        _ptr(out, np.float32), _stream(W, S, Q, Z))
+    if status != JARQ_OK:
+        raise JarqError(status, "jarq_residual_product")
+    return out
 
 
 def objective(hess: Hessian, W, S, Q, Z, bits: int, out=None):
