@@ -19,9 +19,10 @@
 // where Delta != 0, so the back substitution proceeds by jumps: every still
 // undecided coordinate rounds its current value in parallel, the highest one
 // whose code changes is fixed, its column updates u below it, and the scan
-// continues beneath it.  Every u_l receives exactly the updates, in the
-// order, of the one-coordinate-at-a-time recursion; the number of serial
-// steps is the number of changed codes plus one.
+// continues beneath it (one warp-wide max reduction per step picks the
+// coordinate and carries its code change).  Every u_l receives exactly the
+// updates, in the order, of the one-coordinate-at-a-time recursion; the
+// number of serial steps is the number of changed codes plus one.
 //
 // The change of the group objective (Eq. group_bils) is
 // dF = s^2 (||R Delta - y||^2 - ||y||^2) = s^2 sum_l (a_l - y_l)(a_l + y_l)
@@ -152,30 +153,23 @@ __global__ void __launch_bounds__(32 * kMaxWarps) babai_kernel(BabaiArgs a) {
         int hi = g - 1;
         bool any = false;
         while (true) {
-            // each lane: its highest still-undecided coordinate whose code changes
-            int tb = -1;
-            float db = 0.f;
+            // each lane: its highest still-undecided coordinate whose code
+            // changes, as the key (l + 1) << 9 | (delta + 256); the warp-wide
+            // maximum is the highest such coordinate of the row
+            uint32_t key = 0;
 #pragma unroll
             for (int t = 0; t < NT; ++t) {
                 const float q = fminf(fmaxf(rintf(fmaf(u[t], rd[t], qc[t])), 0.f), qmaxf);
-                if (l0 + t <= hi && q != qc[t]) {
-                    tb = t;
-                    db = q - qc[t];
-                }
+                if (l0 + t <= hi && q != qc[t])
+                    key = ((uint32_t)(l0 + t + 1) << 9) | (uint32_t)((int)(q - qc[t]) + 256);
             }
-            const uint32_t bal = __ballot_sync(0xffffffffu, tb >= 0);
-            if (!bal) break;
-            const int owner = 31 - __clz(bal);
-            // t (2 bits) and the code change (|delta| <= 255) in one word
-            const int word = __shfl_sync(0xffffffffu, (tb & 3) | (((int)db + 256) << 2), owner);
-            const int ts = word & 3;
-            const float fd = (float)((word >> 2) - 256);
-            const int lstar = owner * NT + ts;
-            if (lane == owner) {
+            const uint32_t best = __reduce_max_sync(0xffffffffu, key);
+            if (!best) break;
+            const int lstar = (int)(best >> 9) - 1;
+            const float fd = (float)((int)(best & 511u) - 256);
 #pragma unroll
-                for (int t = 0; t < NT; ++t)
-                    if (t == ts) qn[t] = qc[t] + fd;
-            }
+            for (int t = 0; t < NT; ++t)
+                if (l0 + t == lstar) qn[t] = qc[t] + fd;
             any = true;
             float lr[NT];
             load_vec<NT>(Lg + lstar * g + l0, lr);   // R[l'][l*] for l' = l0..

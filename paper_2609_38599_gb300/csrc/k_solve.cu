@@ -1,10 +1,12 @@
 // Joint scale solve, one warp per output row (Sec. 3.3.1; App. E).
 //
 // For each active row j the warp
-//  1. symmetrises its G x G Gram matrix (App. E "Solving for scales") and
-//     forms, in float64, the gradient g = rhs - Gram s_old of the current
-//     scales (rhs_i = c_i^T P_i from the target projection) and the
-//     objective F(s_old) = wHw - s_old^T (rhs + g);
+//  1. reads its G x G Gram matrix -- symmetric by construction, since the
+//     Gram kernel computes each block once and writes it to both triangles,
+//     so the symmetrisation of App. E "Solving for scales" is the identity
+//     on it -- and forms, in float64, the gradient g = rhs - Gram s_old of
+//     the current scales (rhs_i = c_i^T P_i from the target projection) and
+//     the objective F(s_old) = wHw - s_old^T (rhs + g);
 //  2. factors the Gram matrix by Cholesky in float32 (the paper solves this
 //     system in FP32).  A pivot at or below rcond * max(max diag, eps), a
 //     nonfinite entry or a failed factorisation adds ridge * I and retries
@@ -113,7 +115,7 @@ __global__ void scale_solve_kernel(SolveArgs a) {
     double *inc = b + G;                                      // increment of the scales
     const double *gj = a.gram + (size_t)j * G * G;
     const double *rj = a.rhs + (size_t)j * G;
-    auto gsym = [&](int r0, int c0) { return 0.5 * (gj[r0 * G + c0] + gj[c0 * G + r0]); };
+    auto gsym = [&](int r0, int c0) { return gj[r0 * G + c0]; };
     for (int t = lane; t < G; t += 32) so[t] = a.S[(size_t)j * G + t];
     __syncwarp();
     // gradient g = rhs - Gram s_old and F(s_old) = wHw - s_old^T (rhs + g)

@@ -178,7 +178,17 @@ __global__ void __launch_bounds__(320, 1)
         }
         bool ok = true;
         const uint32_t base = tmem + ((uint32_t)(32 * q) << 16) + half * 32;
+        // exponents of the next group, loaded one group ahead
+        const int *wrow = a.wexp + (size_t)min(row, a.p - 1) * a.G;
+        const int hb = min(hblk, a.G - 1);
+        int ew_next = wrow[0], eh_next = a.hexp[hb];
         for (int sg = 0; sg < nseg; ++sg) {
+            const int ew = row < a.p ? ew_next : 0;
+            const int eh = hblk < a.G ? eh_next : 0;
+            if (sg + 1 < nseg) {
+                ew_next = wrow[sg + 1];
+                eh_next = a.hexp[(sg + 1) * a.G + hb];
+            }
             bool w = tc::mbar_wait(afull, sg & 1);
             w = __shfl_sync(0xffffffffu, w && !*abort_flag, 0);
             tc::tc_fence_after();
@@ -187,8 +197,6 @@ __global__ void __launch_bounds__(320, 1)
                 *abort_flag = 1;
                 break;
             }
-            const int ew = row < a.p ? a.wexp[(size_t)row * a.G + sg] : 0;
-            const int eh = hblk < a.G ? a.hexp[sg * a.G + hblk] : 0;
             const float scale = ldexpf(1.0f, ew + eh - 14);
             // value of the group = sum_l L_l 2^(-8 l), as (vh, vl), 32 columns
             float vh[32], vl[32];
@@ -370,7 +378,7 @@ __global__ void whw_kernel(const float *__restrict__ W, const float *__restrict_
 // group i); Rinv_i and the rows' P slice in shared memory.
 constexpr int kPtRows = 64;
 
-__global__ void __launch_bounds__(256) ptilde_kernel(const float *__restrict__ Phi,
+__global__ void __launch_bounds__(512) ptilde_kernel(const float *__restrict__ Phi,
                                                      const float *__restrict__ Plo,
                                                      const double *__restrict__ Rinv,
                                                      float *__restrict__ out_hi,
@@ -398,26 +406,40 @@ __global__ void __launch_bounds__(256) ptilde_kernel(const float *__restrict__ P
         pl[idx] = in ? Plo[o] : 0.f;
     }
     __syncthreads();
+    // each thread: one output column a and kRowsPer rows, independent chains
+    constexpr int kRowsPer = 8;
     const int a = tid % g, jstep = blockDim.x / g;
-    for (int jj = tid / g; jj < kPtRows; jj += jstep) {
-        if (r0 + jj >= p) break;
-        float sh = 0.f, sl = 0.f;
+    for (int jb = (tid / g) * kRowsPer; jb < kPtRows; jb += jstep * kRowsPer) {
+        float sh[kRowsPer], sl[kRowsPer];
+#pragma unroll
+        for (int r = 0; r < kRowsPer; ++r) {
+            sh[r] = 0.f;
+            sl[r] = 0.f;
+        }
         for (int b = 0; b <= a; ++b) {
             const float xh = rh[b * g + a], xl = rl[b * g + a];
-            const float yh = ph[jj * g + b], yl = pl[jj * g + b];
-            const float m = xh * yh;
-            float e = fmaf(xh, yh, -m);
-            e = fmaf(xh, yl, fmaf(xl, yh, e));
-            float s2, e2;
-            two_sum(sh, m, s2, e2);
-            sh = s2;
-            sl += e2 + e;
+#pragma unroll
+            for (int r = 0; r < kRowsPer; ++r) {
+                const float yh = ph[(jb + r) * g + b], yl = pl[(jb + r) * g + b];
+                const float m = xh * yh;
+                float e = fmaf(xh, yh, -m);
+                e = fmaf(xh, yl, fmaf(xl, yh, e));
+                float s2, e2;
+                two_sum(sh[r], m, s2, e2);
+                sh[r] = s2;
+                sl[r] += e2 + e;
+            }
         }
-        float s2, e2;
-        two_sum(sh, sl, s2, e2);
-        const size_t o = (size_t)(r0 + jj) * d + (size_t)i * g + a;
-        out_hi[o] = s2;
-        out_lo[o] = e2;
+#pragma unroll
+        for (int r = 0; r < kRowsPer; ++r) {
+            if (r0 + jb + r < p) {
+                float s2, e2;
+                two_sum(sh[r], sl[r], s2, e2);
+                const size_t o = (size_t)(r0 + jb + r) * d + (size_t)i * g + a;
+                out_hi[o] = s2;
+                out_lo[o] = e2;
+            }
+        }
     }
 }
 
@@ -430,7 +452,7 @@ cudaError_t launch_ptilde(const float *Phi, const float *Plo, const double *Rinv
                                          (int)smem);
     if (e != cudaSuccess) return e;
     dim3 grid((p + kPtRows - 1) / kPtRows, d / g);
-    ptilde_kernel<<<grid, 256, smem, s>>>(Phi, Plo, Rinv, out_hi, out_lo, p, d, g);
+    ptilde_kernel<<<grid, 512, smem, s>>>(Phi, Plo, Rinv, out_hi, out_lo, p, d, g);
     return cudaGetLastError();
 }
 

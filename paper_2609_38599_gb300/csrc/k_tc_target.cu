@@ -20,10 +20,13 @@
 // precision float32 would.
 //
 // One CTA: 128 rows x 64 columns of group i over the groups of one K split.
-//   warp 0      TMA producer: codes tile + 4 digit tiles per 64-wide K chunk
-//   warp 1      TMEM allocation and the single-thread MMA issuer
-//   warps 2..9  drain: warp w reads TMEM lanes 32 (w % 4) and 32 columns
+//   warp 0       TMA producer: codes tile + 4 digit tiles per 64-wide K chunk
+//   warp 1       TMEM allocation and the single-thread MMA issuer
+//   warps 2..17  drain: warp w reads TMEM lanes 32 (w % 4) and 16 columns
 // Four 64-column accumulators per group h, double-buffered (512 columns).
+// The drain does about 19 float32 operations per output and group, hence
+// sixteen drain warps; the scale and block exponent of the next group are
+// loaded one group ahead.
 #include "tc_common.cuh"
 
 namespace jarq {
@@ -35,6 +38,8 @@ constexpr int kStage = kTileA + 4 * kTileB;
 constexpr int kStages = 4;
 constexpr int kSmem = 1024 + kStages * kStage + 256;
 constexpr uint32_t kIdesc = tc::idesc_f16_f32(128, 64);
+constexpr int kDrainWarps = 16;
+constexpr int kThreads = 32 * (2 + kDrainWarps);
 
 struct TargetArgs {
     float *out_hi, *out_lo;   // [nsplit][p_pad][g]
@@ -51,7 +56,7 @@ __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
     e = (a - (s - bb)) + (b - bb);
 }
 
-__global__ void __launch_bounds__(320, 1)
+__global__ void __launch_bounds__(kThreads, 1)
     tc_target_kernel(const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapT,
                      TargetArgs a) {
     extern __shared__ uint8_t smem_raw[];
@@ -93,7 +98,7 @@ __global__ void __launch_bounds__(320, 1)
         }
         for (int b = 0; b < 2; ++b) {
             tc::mbar_init(afull(b), 1);
-            tc::mbar_init(aempty(b), 8);
+            tc::mbar_init(aempty(b), kDrainWarps);
         }
         *abort_flag = 0;
         tc::fence_barrier_init();
@@ -164,17 +169,27 @@ __global__ void __launch_bounds__(320, 1)
         }
     } else if (warp >= 2) {
         // ---------------- drain: digits -> double-float x s_h 2^(E - 9) -> accumulator
-        const int q = warp & 3, half = (warp - 2) >> 2;
+        const int q = warp & 3, cq = (warp - 2) >> 2;    // lane quarter, 16-column quarter
         const int row = j0 + 32 * q + lane;
-        float hi[32], lo[32];
+        float hi[16], lo[16];
 #pragma unroll
-        for (int e = 0; e < 32; ++e) {
+        for (int e = 0; e < 16; ++e) {
             hi[e] = 0.f;
             lo[e] = 0.f;
         }
         bool ok = true;
+        const float *srow = a.S + (size_t)min(row, a.p - 1) * a.G;
+        const int *erow = a.expoT + (size_t)a.i * a.G;
+        float s_next = nseg > 0 ? srow[h0] : 0.f;
+        int e_next = nseg > 0 ? erow[h0] : 0;
         for (int u = 0; u < nseg; ++u) {
             const int b = u & 1, h = h0 + u;
+            const float s_cur = row < a.p ? s_next : 0.f;
+            const int e_cur = e_next;
+            if (u + 1 < nseg) {
+                s_next = srow[h + 1];
+                e_next = erow[h + 1];
+            }
             bool w = tc::mbar_wait(afull(b), (u >> 1) & 1);
             w = __shfl_sync(0xffffffffu, w && !*abort_flag, 0);
             tc::tc_fence_after();
@@ -183,25 +198,30 @@ __global__ void __launch_bounds__(320, 1)
                 *abort_flag = 1;
                 break;
             }
-            const float sh = row < a.p ? a.S[(size_t)row * a.G + h] : 0.f;
-            const float scale = ldexpf(sh, a.expoT[a.i * a.G + h] - 9);
-            const uint32_t base = tmem + ((uint32_t)(32 * q) << 16) + b * 256 + half * 32;
+            const float scale = ldexpf(s_cur, e_cur - 9);
+            const uint32_t base = tmem + ((uint32_t)(32 * q) << 16) + b * 256 + cq * 16;
 #pragma unroll
-            for (int cc = 0; cc < 32; cc += 16) {
-                uint32_t v0[16], v1[16], v2[16], v3[16];
-                tc::tmem_ld16(base + 0 * 64 + cc, v0);
-                tc::tmem_ld16(base + 1 * 64 + cc, v1);
-                tc::tmem_ld16(base + 2 * 64 + cc, v2);
-                tc::tmem_ld16(base + 3 * 64 + cc, v3);
+            for (int cc = 0; cc < 16; cc += 8) {
+                uint32_t v0[8], v1[8], v2[8], v3[8];
+                tc::tmem_ld8(base + 0 * 64 + cc, v0);
+                tc::tmem_ld8(base + 1 * 64 + cc, v1);
+                tc::tmem_ld8(base + 2 * 64 + cc, v2);
+                tc::tmem_ld8(base + 3 * 64 + cc, v3);
                 tc::tmem_wait_ld();
+                if (cc == 8) {
+                    // every digit sum of this group is in registers
+                    tc::tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) tc::mbar_arrive(aempty(b));
+                }
 #pragma unroll
-                for (int e = 0; e < 16; ++e) {
-                    // exact digit sums -> (vh, vl); every scaling below is by a power of two
+                for (int e = 0; e < 8; ++e) {
+                    // D_0 + D_1 2^-10 exactly as (vh, vl); the D_2, D_3 terms are
+                    // below 2^-20 of it and enter the low part
                     float vh, vl, s2, e2;
                     two_sum(__uint_as_float(v0[e]), __uint_as_float(v1[e]) * 0x1p-10f, vh, vl);
-                    two_sum(vh, __uint_as_float(v2[e]) * 0x1p-20f, s2, e2);
-                    vh = s2;
-                    vl += e2 + __uint_as_float(v3[e]) * 0x1p-30f;
+                    vl = fmaf(__uint_as_float(v2[e]), 0x1p-20f, vl);
+                    vl = fmaf(__uint_as_float(v3[e]), 0x1p-30f, vl);
                     // (vh + vl) * scale, added to the accumulator
                     const float ph = vh * scale;
                     const float pe = fmaf(vh, scale, -ph);
@@ -210,14 +230,11 @@ __global__ void __launch_bounds__(320, 1)
                     lo[cc + e] += e2 + fmaf(vl, scale, pe);
                 }
             }
-            tc::tc_fence_before();
-            __syncwarp();
-            if (lane == 0) tc::mbar_arrive(aempty(b));
         }
         if (ok && row < a.p) {
-            const size_t o = (size_t)blockIdx.z * a.p_pad * a.g + (size_t)row * a.g + blockIdx.y * 64 + half * 32;
+            const size_t o = (size_t)blockIdx.z * a.p_pad * a.g + (size_t)row * a.g + blockIdx.y * 64 + cq * 16;
 #pragma unroll
-            for (int e = 0; e < 32; e += 4) {
+            for (int e = 0; e < 16; e += 4) {
                 float x[4], y[4];
 #pragma unroll
                 for (int k = 0; k < 4; ++k) two_sum(hi[e + k], lo[e + k], x[k], y[k]);
@@ -261,7 +278,7 @@ cudaError_t launch_tc_target(const CUtensorMap &mapC, const CUtensorMap &mapT, f
     const int per = (G + nsplit - 1) / nsplit;
     TargetArgs a{out_hi, out_lo, S, expoT, active, status, p, p_pad, d_pad, g, G, i, per};
     dim3 grid(p_pad / 128, g / 64, nsplit);
-    return launch_pdl(tc_target_kernel, grid, dim3(320), (size_t)kSmem, s, mapC, mapT, a);
+    return launch_pdl(tc_target_kernel, grid, dim3(kThreads), (size_t)kSmem, s, mapC, mapT, a);
 }
 
 }  // namespace jarq
