@@ -31,7 +31,9 @@ constexpr int kStage = kTileA + 4 * kTileB;
 constexpr int kStages = 3;
 constexpr int kCodesBytes = 128 * 128 * 2;  // int16 codes of group i for the tile
 constexpr int kSmem = 1024 + kStages * kStage + kCodesBytes + 256;
-constexpr uint32_t kIdesc = tc::idesc_f16_f32(128, 64);
+// one MMA covers the four digit planes: they are consecutive 64-row tiles
+// in shared memory, and their accumulators consecutive 64-column blocks
+constexpr uint32_t kIdesc = tc::idesc_f16_f32(128, 256);
 
 struct GramArgs {
     const uint8_t *Q;
@@ -161,11 +163,8 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
                 for (int sub = 0; sub < 4; ++sub) {
                     const uint64_t ad = tc::sdesc_sw128(tileA(s)) + 2 * sub;
-#pragma unroll
-                    for (int t = 0; t < 4; ++t) {
-                        const uint64_t bd = tc::sdesc_sw128(tileB(s, t)) + 2 * sub;
-                        tc::mma_bf16(tmem + b * 256 + t * 64, ad, bd, kIdesc, (kc | sub) != 0);
-                    }
+                    const uint64_t bd = tc::sdesc_sw128(tileB(s, 0)) + 2 * sub;
+                    tc::mma_bf16(tmem + b * 256, ad, bd, kIdesc, (kc | sub) != 0);
                 }
                 tc::mma_commit(empty(s));
             }

@@ -14,9 +14,9 @@
 // with |a_t|, |b_u| <= 128 (exact in bf16).  Four digits hold every float32 W
 // entry within 2^7 of its group maximum exactly, six every H entry within
 // 2^24 of its block maximum.  For each group h of K the eighteen digit
-// products with t + u <= 5 accumulate in six TMEM "levels" l = t + u; a
-// level sums at most 4 x 128 products of 14-bit integers per output, an
-// exact integer below 2^23.  The epilogue combines the levels in
+// products with t + u <= 5 (six MMAs per K step) accumulate in six TMEM
+// "levels" l = t + u; a level sums at most 4 x 128 products of 14-bit
+// integers per output, an exact integer below 2^23.  The epilogue combines the levels in
 // double-float (pairs of float32), applies 2^(ew + E - 14) and adds the
 // group's contribution to a double-float accumulator.  The dropped products
 // (t + u >= 6) are below 2^-48 of the block scales.
@@ -38,7 +38,10 @@ constexpr int kTileB = 64 * 64 * 2;    // one H digit plane, 64 rows x 64 K
 constexpr int kStage = kWDig * kTileA + kHDig * kTileB;
 constexpr int kStages = 2;
 constexpr int kSmem = 1024 + kStages * kStage + 256;
-constexpr uint32_t kIdesc = tc::idesc_bf16_f32(128, 64);
+// For a W digit t the H digit planes u are consecutive 64-row tiles and the
+// levels t + u consecutive 64-column blocks, so one MMA covers up to four
+// planes (N = 64 per plane).
+__host__ __device__ constexpr uint32_t idesc_n(int n) { return tc::idesc_bf16_f32(128, n); }
 constexpr int kGroupRows = 8;
 
 struct ProjArgs {
@@ -152,13 +155,14 @@ __global__ void __launch_bounds__(320, 1)
 #pragma unroll
                     for (int t = 0; t < kWDig; ++t) {
                         const uint64_t ad = tc::sdesc_sw128(tileA(s, t)) + 2 * sub;
+                        // the products of W digit t with H digits u < kLevels - t,
+                        // in runs of at most four planes; t = 0 opens every level
+                        const uint32_t acc = (kc | sub | t) != 0;
 #pragma unroll
-                        for (int u = 0; u < kHDig; ++u) {
-                            if (t + u >= kLevels) continue;
-                            const uint64_t bd = tc::sdesc_sw128(tileB(s, u)) + 2 * sub;
-                            // the product (0, l) opens level l of the group
-                            const uint32_t acc = (kc | sub | t) != 0;
-                            tc::mma_bf16(tmem + (t + u) * 64, ad, bd, kIdesc, acc);
+                        for (int u0 = 0; u0 < kLevels - t; u0 += 4) {
+                            const int nu = min(4, kLevels - t - u0);
+                            const uint64_t bd = tc::sdesc_sw128(tileB(s, u0)) + 2 * sub;
+                            tc::mma_bf16(tmem + (t + u0) * 64, ad, bd, idesc_n(64 * nu), acc);
                         }
                     }
                 }

@@ -20,13 +20,19 @@
 // precision float32 would.
 //
 // One CTA: 128 rows x 64 columns of group i over the groups of one K split.
-//   warp 0       TMA producer: codes tile + 4 digit tiles per 64-wide K chunk
+//   warp 0       TMA producer: codes tile + its share of the digit tiles
 //   warp 1       TMEM allocation and the single-thread MMA issuer
 //   warps 2..17  drain: warp w reads TMEM lanes 32 (w % 4) and 16 columns
 // Four 64-column accumulators per group h, double-buffered (512 columns).
 // The drain does about 19 float32 operations per output and group, hence
 // sixteen drain warps; the scale and block exponent of the next group are
 // loaded one group ahead.
+// The kernel is bound by moving tiles into shared memory, and the digit
+// tiles are the same for every row tile.  CTAs of consecutive row tiles
+// therefore form a cluster of C: each loads 4/C of the digit planes and
+// multicasts them to all C, cutting that traffic by C.  A stage is refilled
+// only after every CTA of the cluster has consumed it (its "empty" barrier
+// counts one MMA commit per CTA), and no CTA leaves before the others.
 #include "tc_common.cuh"
 
 namespace jarq {
@@ -37,7 +43,9 @@ constexpr int kTileB = 64 * 64 * 2;    // one digit plane: 64 rows of Ht x 64 K
 constexpr int kStage = kTileA + 4 * kTileB;
 constexpr int kStages = 4;
 constexpr int kSmem = 1024 + kStages * kStage + 256;
-constexpr uint32_t kIdesc = tc::idesc_f16_f32(128, 64);
+// one MMA covers the four digit planes: they are consecutive 64-row tiles
+// in shared memory, and their accumulators consecutive 64-column blocks
+constexpr uint32_t kIdesc = tc::idesc_f16_f32(128, 256);
 constexpr int kDrainWarps = 16;
 constexpr int kThreads = 32 * (2 + kDrainWarps);
 
@@ -48,6 +56,7 @@ struct TargetArgs {
     const int *active;
     int *status;
     int p, p_pad, d_pad, g, G, i, seg_per_split;
+    int csize;                // CTAs per cluster (1, 2 or 4)
 };
 
 __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
@@ -73,16 +82,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int nkc = a.g / 64;
     const int nchunks = nseg * nkc;
 
-    // the codes are rewritten by the previous Babai phase
-    tc::pdl_wait();
-    {
-        int mine = 0;
-        if (threadIdx.x < 128 && j0 + (int)threadIdx.x < a.p) mine = a.active[j0 + threadIdx.x];
-        if (!__syncthreads_or(mine)) {
-            tc::pdl_launch_dependents();
-            return;
-        }
-    }
+    const uint32_t crank = a.csize > 1 ? tc::cluster_ctarank() : 0;
+    const uint16_t cmask = (uint16_t)((1u << a.csize) - 1u);
 
     auto full = [&](int s) { return tc::smem_u32(bars + s); };
     auto empty = [&](int s) { return tc::smem_u32(bars + kStages + s); };
@@ -94,7 +95,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             tc::mbar_init(full(s), 1);
-            tc::mbar_init(empty(s), 1);
+            tc::mbar_init(empty(s), a.csize);   // one MMA commit per CTA of the cluster
         }
         for (int b = 0; b < 2; ++b) {
             tc::mbar_init(afull(b), 1);
@@ -112,9 +113,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc::prefetch_tmap(&mapT);
     }
     tc::tc_fence_before();
-    __syncthreads();
+    // every CTA's barriers are initialised before any multicast reaches them
+    if (a.csize > 1)
+        tc::cluster_sync();
+    else
+        __syncthreads();
     tc::tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    // the codes are rewritten by the previous Babai phase
+    tc::pdl_wait();
     tc::pdl_launch_dependents();
 
     if (warp == 0 && lane == 0) {
@@ -127,16 +134,23 @@ __global__ void __launch_bounds__(kThreads, 1)
                 break;
             }
             const int kx = h0 * a.g + c * 64;
+            // this CTA's full barrier counts the whole stage, including the
+            // digit tiles the other CTAs of the cluster multicast into it
             tc::mbar_expect_tx(full(s), kStage);
             tc::tma_load_2d(tileA(s), &mapC, full(s), kx, j0);
 #pragma unroll
-            for (int t = 0; t < 4; ++t)
-                tc::tma_load_2d(tileB(s, t), &mapT, full(s), kx, t * a.d_pad + m0);
+            for (int t = 0; t < 4; ++t) {
+                if (a.csize == 1)
+                    tc::tma_load_2d(tileB(s, t), &mapT, full(s), kx, t * a.d_pad + m0);
+                else if (t % a.csize == (int)crank)
+                    tc::tma_load_2d_mc(tileB(s, t), &mapT, full(s), kx, t * a.d_pad + m0, cmask);
+            }
             issued = c + 1;
         }
-        // do not leave with copies in flight
+        // do not leave before every CTA of the cluster has consumed the
+        // stages this CTA filled: no copy or commit is in flight afterwards
         for (int c = issued > kStages ? issued - kStages : 0; c < issued; ++c)
-            if (!tc::mbar_wait(full(c % kStages), (c / kStages) & 1)) *abort_flag = 1;
+            if (!tc::mbar_wait(empty(c % kStages), (c / kStages) & 1)) *abort_flag = 1;
     } else if (warp == 1 && lane == 0) {
         // ---------------- MMA issuer: one unit per group h
         for (int u = 0; u < nseg && !*abort_flag; ++u) {
@@ -157,13 +171,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                 for (int sub = 0; sub < 4; ++sub) {
                     const uint64_t ad = tc::sdesc_sw128(tileA(s)) + 2 * sub;
-#pragma unroll
-                    for (int t = 0; t < 4; ++t) {
-                        const uint64_t bd = tc::sdesc_sw128(tileB(s, t)) + 2 * sub;
-                        tc::mma_bf16(tmem + b * 256 + t * 64, ad, bd, kIdesc, (kc | sub) != 0);
-                    }
+                    const uint64_t bd = tc::sdesc_sw128(tileB(s, 0)) + 2 * sub;
+                    tc::mma_bf16(tmem + b * 256, ad, bd, kIdesc, (kc | sub) != 0);
                 }
-                tc::mma_commit(empty(s));
+                if (a.csize > 1)
+                    tc::mma_commit_mc(empty(s), cmask);
+                else
+                    tc::mma_commit(empty(s));
             }
             tc::mma_commit(afull(b));
         }
@@ -244,7 +258,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     }
     tc::tc_fence_before();
-    __syncthreads();
+    __syncwarp();
+    // no CTA leaves while another may still write to its shared memory
+    if (a.csize > 1)
+        tc::cluster_sync();
+    else
+        __syncthreads();
     if (warp == 1) {
         tc::tc_fence_after();
         tc::tmem_dealloc(tmem, 512);
@@ -276,9 +295,12 @@ cudaError_t launch_tc_target(const CUtensorMap &mapC, const CUtensorMap &mapT, f
         attr_set = true;
     }
     const int per = (G + nsplit - 1) / nsplit;
-    TargetArgs a{out_hi, out_lo, S, expoT, active, status, p, p_pad, d_pad, g, G, i, per};
-    dim3 grid(p_pad / 128, g / 64, nsplit);
-    return launch_pdl(tc_target_kernel, grid, dim3(kThreads), (size_t)kSmem, s, mapC, mapT, a);
+    const int tiles = p_pad / 128;
+    const int csize = tiles % 4 == 0 ? 4 : tiles % 2 == 0 ? 2 : 1;
+    TargetArgs a{out_hi, out_lo, S, expoT, active, status, p, p_pad, d_pad, g, G, i, per, csize};
+    dim3 grid(tiles, g / 64, nsplit);
+    return launch_pdl_cluster(tc_target_kernel, grid, dim3(kThreads), (size_t)kSmem, s, csize,
+                              mapC, mapT, a);
 }
 
 }  // namespace jarq
