@@ -148,8 +148,17 @@ __global__ void __launch_bounds__(32 * kMaxWarps) babai_kernel(BabaiArgs a) {
             y[t] = y[t] / s;
             u[t] = y[t];
         }
-        // back substitution by jumps (Eq. babai_update)
+        // back substitution by jumps (Eq. babai_update).  Rounding to the
+        // nearest even integer adds and subtracts 1.5 * 2^23 (exact for
+        // |x| < 2^22; beyond that the clamp to [0, qmax] gives the same code
+        // as rintf), and small integers travel in float bits: v + 2^23 has
+        // the bit pattern 0x4B000000 | v for 0 <= v < 2^23.
         const float qmaxf = (float)a.qmax;
+        constexpr float kRound = 12582912.0f;      // 1.5 * 2^23
+        constexpr float kBias = 8388864.0f;        // 2^23 + 256
+        uint32_t pos[NT];                          // (l + 1) << 9 of this lane's coordinates
+#pragma unroll
+        for (int t = 0; t < NT; ++t) pos[t] = (uint32_t)(l0 + t + 1) << 9;
         int hi = g - 1;
         bool any = false;
         while (true) {
@@ -159,14 +168,16 @@ __global__ void __launch_bounds__(32 * kMaxWarps) babai_kernel(BabaiArgs a) {
             uint32_t key = 0;
 #pragma unroll
             for (int t = 0; t < NT; ++t) {
-                const float q = fminf(fmaxf(rintf(fmaf(u[t], rd[t], qc[t])), 0.f), qmaxf);
-                if (l0 + t <= hi && q != qc[t])
-                    key = ((uint32_t)(l0 + t + 1) << 9) | (uint32_t)((int)(q - qc[t]) + 256);
+                const float x = fmaf(u[t], rd[t], qc[t]);
+                const float r = __fsub_rn(__fadd_rn(x, kRound), kRound);
+                const float q = fminf(fmaxf(r, 0.f), qmaxf);
+                const uint32_t kt = pos[t] | (__float_as_uint(__fadd_rn(q - qc[t], kBias)) & 511u);
+                if (l0 + t <= hi && q != qc[t]) key = kt;
             }
             const uint32_t best = __reduce_max_sync(0xffffffffu, key);
             if (!best) break;
             const int lstar = (int)(best >> 9) - 1;
-            const float fd = (float)((int)(best & 511u) - 256);
+            const float fd = __uint_as_float((best & 511u) | 0x4B000000u) - kBias;
 #pragma unroll
             for (int t = 0; t < NT; ++t)
                 if (l0 + t == lstar) qn[t] = qc[t] + fd;

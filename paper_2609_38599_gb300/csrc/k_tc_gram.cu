@@ -17,7 +17,9 @@
 // G + 1 blocks.
 //
 // Roles: warp 0 TMA producer; warp 1 TMEM allocation and MMA issuer;
-// warps 2..5 epilogue (TMEM lanes 32 (w % 4) ..).  One unit of work is
+// warps 2..9 epilogue: warp w reads TMEM lanes 32 (w % 4) .. and 32 of the
+// 64 columns of a unit; the two warps of a lane quarter add their partial
+// dots through shared memory at the end of each block.  One unit of work is
 // (h, column half of group i): 4 accumulators of 64 columns (one per digit
 // plane), double-buffered in 512 TMEM columns.
 #include "tc_common.cuh"
@@ -30,7 +32,9 @@ constexpr int kTileB = 64 * 64 * 2;    // 64 H rows x 64 K, one digit plane (fp1
 constexpr int kStage = kTileA + 4 * kTileB;
 constexpr int kStages = 3;
 constexpr int kCodesBytes = 128 * 128 * 2;  // int16 codes of group i for the tile
-constexpr int kSmem = 1024 + kStages * kStage + kCodesBytes + 256;
+constexpr int kPartBytes = 2 * 4 * 128 * 8;  // int64 partial dots, double-buffered
+constexpr int kSmem = 1024 + kStages * kStage + kCodesBytes + kPartBytes + 256;
+constexpr int kThreads = 320;
 // one MMA covers the four digit planes: they are consecutive 64-row tiles
 // in shared memory, and their accumulators consecutive 64-column blocks
 constexpr uint32_t kIdesc = tc::idesc_f16_f32(128, 256);
@@ -54,13 +58,14 @@ __device__ __forceinline__ int exact_int(float x) {
 // integer dots; otherwise |c| <= 15, |D_t| < 2^20 and every partial dot of
 // 8 terms fits in 32 bits.
 template <bool WIDE>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(kThreads, 1)
     tc_gram_kernel(const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapS,
                    GramArgs a) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     int16_t *codes = (int16_t *)(smem + kStages * kStage);   // [128 rows][128]
-    uint64_t *bars = (uint64_t *)(smem + kStages * kStage + kCodesBytes);
+    long long *part = (long long *)(smem + kStages * kStage + kCodesBytes);   // [2][4][128]
+    uint64_t *bars = (uint64_t *)(smem + kStages * kStage + kCodesBytes + kPartBytes);
     uint32_t *tmem_slot = (uint32_t *)(bars + 2 * kStages + 4);
     volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -103,7 +108,7 @@ __global__ void __launch_bounds__(192, 1)
         }
         for (int b = 0; b < 2; ++b) {
             tc::mbar_init(afull(b), 1);
-            tc::mbar_init(aempty(b), 4);
+            tc::mbar_init(aempty(b), 8);
         }
         *abort_flag = 0;
         tc::fence_barrier_init();
@@ -172,50 +177,55 @@ __global__ void __launch_bounds__(192, 1)
         }
     } else if (warp >= 2) {
         // ---------------- epilogue: exact integer dots with the codes of group i
-        const int q = warp & 3;
+        const int q = warp & 3, cw = (warp - 2) >> 2;   // lane quarter, 32-column slice
         const int rl = 32 * q + lane;           // row within the tile
         const int row = j0 + rl;
-        int cur_g = -1;
+        int cur_g = -1, par = 0;
+        bool dead = false;                      // a wait gave up: skip work, keep the pair barriers
         long long acc[4] = {0, 0, 0, 0};
         for (int u = 0; u < nunits; ++u) {
             int gi, h, half;
             unit(u, gi, h, half);
             if (gi != cur_g) {
-                // stage this tile's codes of group gi (row rl written by its own thread)
+                // stage this warp's columns of group gi (row rl written by its own thread)
                 __syncwarp();
-                if (row < a.p) {
-                    const int zz = a.Z[(size_t)row * G + gi];
-                    const uint4 *src = reinterpret_cast<const uint4 *>(a.Q + (size_t)row * a.d + gi * g);
-                    for (int m16 = 0; m16 < g / 16; ++m16) {
-                        const uint4 v = src[m16];
-                        const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+                for (int hf = 0; hf < nhalf; ++hf) {
+                    const int c0 = hf * 64 + cw * 32;
+                    if (row < a.p) {
+                        const int zz = a.Z[(size_t)row * G + gi];
+                        const uint4 *src = reinterpret_cast<const uint4 *>(a.Q + (size_t)row * a.d + gi * g + c0);
+                        for (int m16 = 0; m16 < 2; ++m16) {
+                            const uint4 v = src[m16];
+                            const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-                        for (int k = 0; k < 16; ++k)
-                            codes[rl * 128 + m16 * 16 + k] =
-                                (int16_t)((int)((w4[k >> 2] >> (8 * (k & 3))) & 0xFFu) - zz);
+                            for (int k = 0; k < 16; ++k)
+                                codes[rl * 128 + c0 + m16 * 16 + k] =
+                                    (int16_t)((int)((w4[k >> 2] >> (8 * (k & 3))) & 0xFFu) - zz);
+                        }
+                    } else {
+                        for (int m = 0; m < 32; ++m) codes[rl * 128 + c0 + m] = 0;
                     }
-                } else {
-                    for (int m = 0; m < g; ++m) codes[rl * 128 + m] = 0;
                 }
                 __syncwarp();
                 cur_g = gi;
             }
             const int b = u & 1;
-            bool w = tc::mbar_wait(afull(b), (u >> 1) & 1);
-            w = __shfl_sync(0xffffffffu, w && !*abort_flag, 0);
-            tc::tc_fence_after();
-            if (!w) {
-                *abort_flag = 1;
-                break;
+            if (!dead) {
+                bool w = tc::mbar_wait(afull(b), (u >> 1) & 1);
+                w = __shfl_sync(0xffffffffu, w && !*abort_flag, 0);
+                tc::tc_fence_after();
+                if (!w) {
+                    *abort_flag = 1;
+                    dead = true;
+                }
             }
-            const uint32_t base = tmem + ((uint32_t)(32 * q) << 16) + b * 256;
-            const int16_t *crow = codes + rl * 128 + half * 64;
-#pragma unroll 1
-            for (int hb = 0; hb < 64; hb += 32) {
+            if (!dead) {
+                const uint32_t base = tmem + ((uint32_t)(32 * q) << 16) + b * 256 + cw * 32;
+                const int16_t *crow = codes + rl * 128 + half * 64 + cw * 32;
                 int cr[32];
 #pragma unroll
                 for (int e = 0; e < 32; e += 8) {
-                    const int4 pk = *reinterpret_cast<const int4 *>(crow + hb + e);
+                    const int4 pk = *reinterpret_cast<const int4 *>(crow + e);
                     const int w4[4] = {pk.x, pk.y, pk.z, pk.w};
 #pragma unroll
                     for (int k = 0; k < 4; ++k) {
@@ -226,9 +236,15 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
                 for (int t = 0; t < 4; ++t) {
                     uint32_t v0[16], v1[16];
-                    tc::tmem_ld16(base + t * 64 + hb, v0);
-                    tc::tmem_ld16(base + t * 64 + hb + 16, v1);
+                    tc::tmem_ld16(base + t * 64, v0);
+                    tc::tmem_ld16(base + t * 64 + 16, v1);
                     tc::tmem_wait_ld();
+                    if (t == 3) {
+                        // every digit of this unit is in registers
+                        tc::tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) tc::mbar_arrive(aempty(b));
+                    }
                     if (WIDE) {
                         long long p0 = 0, p1 = 0, p2 = 0, p3 = 0;
 #pragma unroll
@@ -252,11 +268,17 @@ __global__ void __launch_bounds__(192, 1)
                     }
                 }
             }
-            tc::tc_fence_before();
-            __syncwarp();
-            if (lane == 0) tc::mbar_arrive(aempty(b));
             if (half == nhalf - 1) {
-                if (row < a.p) {
+                // the pair of warps of this lane quarter adds its partial dots
+                long long *pp = part + (size_t)par * 4 * 128;
+                if (cw == 1) {
+#pragma unroll
+                    for (int t = 0; t < 4; ++t) pp[t * 128 + rl] = acc[t];
+                }
+                asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory");
+                if (cw == 0 && row < a.p && !dead) {
+#pragma unroll
+                    for (int t = 0; t < 4; ++t) acc[t] += pp[t * 128 + rl];
                     const int E = a.expo[gi * G + h];
                     const double v = ldexp((double)acc[0] + ldexp((double)acc[1], -10) +
                                                ldexp((double)acc[2], -20) + ldexp((double)acc[3], -30),
@@ -267,6 +289,7 @@ __global__ void __launch_bounds__(192, 1)
                 }
 #pragma unroll
                 for (int t = 0; t < 4; ++t) acc[t] = 0;
+                par ^= 1;
             }
         }
     }
@@ -411,9 +434,9 @@ cudaError_t launch_tc_gram(const CUtensorMap &mapC, const CUtensorMap &mapS, con
     GramArgs a{Q, Z, expo, active, gram, status, p, d, g, G, d_pad};
     dim3 grid(p_pad / 128, (G + 1) / 2, 1);
     if (bits <= 4)
-        tc_gram_kernel<false><<<grid, 192, kSmem, s>>>(mapC, mapS, a);
+        tc_gram_kernel<false><<<grid, kThreads, kSmem, s>>>(mapC, mapS, a);
     else
-        tc_gram_kernel<true><<<grid, 192, kSmem, s>>>(mapC, mapS, a);
+        tc_gram_kernel<true><<<grid, kThreads, kSmem, s>>>(mapC, mapS, a);
     return cudaGetLastError();
 }
 
