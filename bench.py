@@ -35,16 +35,19 @@ PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 SM_COUNT = 152
 FP32_LANES_PER_SM = 128
 SM_MAX_MHZ = 2070.0
-DTYPE = "f32 (bf16x3 split products on tensor cores; integer-digit Gram and projection)"
+DTYPE = "f32 (integer-digit fp16/bf16 tensor-core products with exact partial sums, double-float accumulation)"
 
 # DRAM bytes (read + write) per launch from one ncu capture of this workload
-# (profiles/ncu_*_q_proj_4096x4096_g128_w3.md), valid while the kernel's
-# source file is unchanged (first 12 hex digits of its SHA-1).
+# (profiles/ncu_refine_kernels_q_proj_4096x4096_g128_w3.md; the sweep kernels'
+# figures are those of the first phase), valid while the kernel's source file
+# is unchanged (first 12 hex digits of its SHA-1).
 TRAFFIC = {
-    "babai": ("k_babai.cu", "126ba525ab8f", 10.3488e6),
-    "hr_full": ("k_tc_hr.cu", "18cbbd861ee9", 816.96896e6 + 62.980608e6),
-    "phase_hr": ("k_tc_hr.cu", "18cbbd861ee9", 103.852544e6 + 3.142656e6),
-    "gram": ("k_tc_gram.cu", "09948d7fccb2", 159.193856e6 + 26.183936e6),
+    "target": ("k_tc_target.cu", "07c974948b9d", 38.300e6 + 0.043264e6),
+    "babai": ("k_babai.cu", "5ea8bbe0238f", 14.275e6 + 0.002560e6),
+    "gram": ("k_tc_gram.cu", "3160a3b4f82d", 163.402e6 + 27.876352e6),
+    "proj": ("k_tc_proj.cu", "391ad329f213", 1374.367e6 + 155.951104e6),
+    "ptilde": ("k_tc_proj.cu", "391ad329f213", 138.978e6 + 90.157056e6),
+    "scale_solve": ("k_solve.cu", "0b9a43feec9b", 35.256e6 + 0.001024e6),
 }
 
 
@@ -209,7 +212,7 @@ def run_reference(args, rank, world):
 def config_dict(lay, note=None):
     c = {"workload": lay.name, "din": lay.din, "dout": lay.dout, "group_size": lay.g,
          "bits": lay.bits, "K": lay.K, "early_stop": False, "host": "RTN",
-         "l2": "inputs larger than L2 (H, W, P, r: 64 MB each per step)"}
+         "l2": "inputs larger than L2 (per step: W, P and the folded P 64 MB each, digit planes of H 336 MB)"}
     if note:
         c["note"] = note
     return c
@@ -222,25 +225,29 @@ def config_dict(lay, note=None):
 def kernel_model(kernel, lay, nsplit_bytes=0):
     """Algorithmic work of one launch and the roofline that bounds the kernel.
 
-    Contractions count one MMA of useful work (2 x M x N x K); the split
-    products they issue (6 for H r, 4 digit planes for the Gram, 18 digit
-    pairs for the target projection) are reported separately as ``issued``.  Babai counts its dense triangular work, 2 g^2
-    flops per (row, group): the R^{-T} product and the back substitution.
-    Memory-bound kernels count the bytes they must move once.
+    Contractions count one MMA of useful work (2 x M x N x K); the digit
+    products they issue (4 digit planes for the phase target product and the
+    Gram, 18 digit pairs for the target projection) are reported separately
+    as ``issued``.  Babai counts its dense triangular back substitution,
+    g^2 flops per (row, group); the folded projection its g^2 / 2
+    multiply-adds per (row, group) in double-float.  Memory-bound kernels
+    count the bytes they must move once.
     """
     p, d, g, G = lay.dout, lay.din, lay.g, lay.din // lay.g
-    if kernel == "phase_hr":
-        return dict(bound="tensor", work=2.0 * p * g * d, issued=6 * 2.0 * p * g * d)
+    if kernel == "target":
+        return dict(bound="tensor", work=2.0 * p * g * d, issued=4 * 2.0 * p * g * d)
     if kernel == "hr_full":
         return dict(bound="tensor", work=2.0 * p * d * d, issued=6 * 2.0 * p * d * d)
     if kernel == "gram":
         blocks = G * (G + 1) / 2
         return dict(bound="tensor", work=2.0 * p * g * g * blocks, issued=4 * 2.0 * p * g * g * blocks)
     if kernel == "babai":
-        return dict(bound="alu", work=2.0 * g * g * p)
+        return dict(bound="alu", work=1.0 * g * g * p)
+    if kernel == "ptilde":
+        return dict(bound="alu", work=1.0 * p * d * g)
     if kernel == "scale_solve":
-        # Gram (f64) + gradient + scales in; scales and the residual (f32 + 3 bf16 planes) out
-        return dict(bound="hbm", work=p * (8.0 * G * G + 8 * G + 8 * G) + p * d * (1 + 4 + 4 + 10))
+        # Gram (f64), rhs (f64), wHw, L_prev and the scales in; scales and L out
+        return dict(bound="hbm", work=p * (8.0 * G * G + 8 * G + 8 + 8 + 4 * G + 4 * G + 8))
     if kernel == "grad":
         return dict(bound="hbm", work=p * d * (4 + 4 + 1) + p * G * 8)
     if kernel == "proj":

@@ -13,7 +13,7 @@ torch = pytest.importorskip("torch")
 pytestmark = [pytest.mark.gpu,
               pytest.mark.skipif(not torch.cuda.is_available(), reason="needs a CUDA GPU")]
 
-from oracle import Options, objective, prepare_hessian, refine_layer  # noqa: E402
+from oracle import Options, group_target, objective, prepare_hessian, refine_layer  # noqa: E402
 from synth import Layer, small_layer, tiny_layer  # noqa: E402
 from tests.parity import compare_final, gpu_refine, lockstep  # noqa: E402
 
@@ -98,6 +98,29 @@ def test_objective_entry_point(jarq):
     F2 = jarq.objective(hess, lay.W, lay.S0, lay.Q0, lay.Z, lay.bits)
     np.testing.assert_allclose(F2, F, rtol=0, atol=0)
     hess.close()
+
+
+@pytest.mark.parametrize("din,dout,g,bits", [(384, 77, 128, 3), (320, 130, 64, 4)])
+def test_residual_product_elementwise(jarq, din, dout, g, bits):
+    """The split-precision tensor-core product H r (Eq. conditional_residual's
+    (H r)_i for every group) against the oracle's float64 group slices, element
+    by element.  The kernel's residual is float32 and its bf16 x 3 products
+    drop terms below 2^-24, so the error is bounded relative to |H| |r|."""
+    lay = small_layer(din, dout, g, bits, seed=31)
+    prep = prepare_hessian(lay.H, lay.g)
+    C = lay.Q0.astype(np.float64) - np.repeat(lay.Z, g, axis=1)
+    r = lay.W.astype(np.float64) - np.repeat(lay.S0.astype(np.float64), g, axis=1) * C
+    ref = np.concatenate([group_target(prep, r, lay.S0[:, i], C[:, i * g:(i + 1) * g], i)[0]
+                          for i in range(din // g)], axis=1)
+    scale = np.abs(r) @ np.abs(prep.H)
+    dev = "cuda"
+    hess = jarq.prepare(torch.as_tensor(lay.H, device=dev), lay.g)
+    HR = jarq.residual_product(hess, torch.as_tensor(lay.W, device=dev),
+                               torch.as_tensor(lay.S0, device=dev), torch.as_tensor(lay.Q0, device=dev),
+                               torch.as_tensor(lay.Z, device=dev), lay.bits).cpu().numpy()
+    hess.close()
+    assert HR.shape == (dout, din)
+    assert np.all(np.abs(HR - ref) <= 4e-6 * scale + 1e-30)
 
 
 def test_host_buffers_match_device_buffers(jarq):
