@@ -412,12 +412,77 @@ def run_ours(args, rank, world):
     return 0
 
 
+BLOCK_WORKLOAD = "llama2_7b_block"
+
+
+def run_block(args, rank, world):
+    """The Llama-2-7B decoder block, timed end to end per block: the three
+    Hessians prepared and the seven layers refined (K = 10 each) per step."""
+    import torch
+    from paper_2609_38599_gb300 import jarq
+    from synth import block_layers
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    hs, layers = block_layers(device=dev)
+    states = [(lay.S0.clone(), lay.Q0.clone()) for _, lay in layers]
+
+    def step():
+        hess = {k: jarq.prepare(h, 128) for k, h in hs.items()}
+        for (hkey, lay), (S, Q) in zip(layers, states):
+            S.copy_(lay.S0)
+            Q.copy_(lay.Q0)
+            opts = jarq.default_options(max_iters=lay.K, early_stop=0)
+            jarq.refine(hess[hkey], lay.W, S, Q, lay.Z, lay.bits, options=opts, collect_stats=False)
+        for h in hess.values():
+            h.close()
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES", "")
+    gpu_index = vis.split(",")[local] if vis and vis.split(",")[0].isdigit() else local
+    sampler = ClockSampler(gpu_index)
+    n0 = jarq.launch_count()
+    sampler.start()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.steps):
+        step()
+    e1.record()
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    launches = jarq.launch_count() - n0
+    ms = e0.elapsed_time(e1) / args.steps
+    weights = sum(lay.din * lay.dout for _, lay in layers)
+    line = {
+        "metric": METRIC, "value": world * weights / (ms / 1e3), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "s_per_block": ms / 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": DTYPE,
+        "data": "synthetic (seeded Llama-2-7B-shaped block, RTN host)",
+        "config": {"workload": BLOCK_WORKLOAD, "layers": [lay.name for _, lay in layers],
+                   "group_size": 128, "bits": 3, "K": 10, "early_stop": False,
+                   "hessians_prepared_per_step": len(hs),
+                   "l2": "inputs larger than L2 (H of down_proj alone 485 MB)"},
+        "roofline": None, "gpu_launches": launches,
+        "launches_per_step": launches / args.steps, "clocks": clocks,
+    }
+    if rank == 0:
+        print(json.dumps(line))
+    return 0
+
+
 def main():
     args = parse_args()
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     if args.impl == "reference":
         return run_reference(args, rank, world)
+    if args.workload == BLOCK_WORKLOAD:
+        return run_block(args, rank, world)
     return run_ours(args, rank, world)
 
 

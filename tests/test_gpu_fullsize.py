@@ -78,3 +78,35 @@ def test_lockstep_sampled_rows(name, n):
 
     recs = lockstep(sub, lay.K, step)
     print(recs)
+
+
+def test_decoder_block_sampled_rows():
+    """The Llama-2-7B decoder block: three Hessians, each prepared once, and
+    the seven layers refined on them (q/k/v/gate/up share the attention-input
+    H); every layer is compared with the oracle on a seeded sample of rows."""
+    from paper_2609_38599_gb300 import jarq
+    from synth import block_layers
+    hs, layers = block_layers(device="cuda")
+    hess = {k: jarq.prepare(h, 128) for k, h in hs.items()}
+    preps = {}
+    for idx, (hkey, lay) in enumerate(layers):
+        S = lay.S0.clone()
+        Q = lay.Q0.clone()
+        st = jarq.refine(hess[hkey], lay.W, S, Q, lay.Z, lay.bits, max_iters=lay.K, early_stop=0)
+        torch.cuda.synchronize()
+        rows = sample_rows(lay.dout, 8, seed=200 + idx)
+        sub = sub_layer(to_np(lay), rows)
+        if hkey not in preps:
+            preps[hkey] = prepare_hessian(sub.H, sub.g)
+        prep = preps[hkey]
+        res = refine_layer(prep, sub.W, sub.S0, sub.Q0, sub.Z, sub.bits,
+                           Options(max_iters=lay.K, early_stop=False))
+        stats = {"L_host": st.L_host.cpu().numpy()[rows], "L_final": st.L_final.cpu().numpy()[rows]}
+        m = compare_final(sub, prep, res, S.cpu().numpy()[rows], Q.cpu().numpy()[rows], stats)
+        print(lay.name, m)
+        assert m["Lhost_rel"] <= 5e-5 and m["Lfinal_vs_oracle_state"] <= 5e-5, (lay.name, m)
+        assert m["S_rel_max_same_rows"] <= 1e-4 and m["F_rel_max_same_rows"] <= 1e-4, (lay.name, m)
+        assert m["gpu_no_worse_than_host"], (lay.name, m)
+        assert m["codes_same"] >= 0.999, (lay.name, m)
+    for h in hess.values():
+        h.close()
