@@ -373,6 +373,36 @@ def run_ours(args, rank, world):
                          "pass of the same K steps (the value pass runs without them)",
         "launches_per_step": launches / args.steps, "clocks": clocks, "kernels": kernels,
     }
+    # write-back post-passes on the refined layer (not part of the step): the
+    # returned weights cast to float16, the packed codes, canonicalisation
+    post = {}
+    if rank == 0:
+        pk2, _ = peaks()
+
+        def timed(fn, reps=5):
+            fn()
+            torch.cuda.synchronize()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            for _ in range(reps):
+                fn()
+            b.record()
+            torch.cuda.synchronize()
+            return a.elapsed_time(b) / reps
+
+        n_el = lay.dout * lay.din
+        G = lay.din // lay.g
+        S2, Q2, Z2 = S.clone(), Q.clone(), lay.Z.clone()
+        t_dq = timed(lambda: jarq.dequantize(S, Q, lay.Z, lay.g, lay.bits, "float16"))
+        t_pk = timed(lambda: jarq.pack_codes(Q, lay.bits))
+        t_cn = timed(lambda: jarq.canonicalize(S2, Q2, Z2, lay.g, lay.bits))
+        for name, ms_, by in (("dequantize_f16", t_dq, n_el * (1 + 2) + lay.dout * G * 8),
+                              ("pack_codes", t_pk, n_el * (1 + lay.bits / 8)),
+                              ("canonicalize", t_cn, n_el * 2 + lay.dout * G * 16)):
+            post[name] = {"ms": ms_, "bytes": by, "GB_s": by / (ms_ / 1e3) / 1e9,
+                          "hbm_frac": by / (ms_ / 1e3) / 1e9 / pk2["hbm_gbs"],
+                          "note": "includes the code validation pass and a synchronize"}
+        line["postpass"] = post
     # end to end through the C ABI with pinned host buffers
     if rank == 0 or True:
         pin = lambda t: t.cpu().pin_memory().numpy()

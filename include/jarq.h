@@ -74,7 +74,13 @@ typedef struct jarq_options {
     float ridge;         /* lambda added when the Gram matrix is nearly singular (1e-4) */
     float rcond;         /* r_cond of the near-singularity test (1e-10)           */
     float eps;           /* eps_fp: FP32 machine epsilon; small-scale skip threshold */
+    int   ridge_accept;  /* 1: keep a ridge-stabilised solve only if it does not raise F_j,
+                            else keep the previous scales (App. G Remark ridge-acceptance);
+                            0 (default): keep every solve, as the paper's runs do */
 } jarq_options;
+
+/* Element types of jarq_dequantize's output. */
+typedef enum jarq_dtype { JARQ_F32 = 0, JARQ_F16 = 1, JARQ_BF16 = 2 } jarq_dtype;
 
 /* Per-row statistics.  Every pointer may be NULL (not collected) and may be
  * host or device memory; arrays have dout entries.
@@ -94,7 +100,7 @@ typedef struct jarq_stats {
 } jarq_stats;
 
 /* Default options: K = 3, early stop on, tau = 1e-5, ridge 1e-4,
- * rcond 1e-10, eps = FLT_EPSILON (App. E). */
+ * rcond 1e-10, eps = FLT_EPSILON (App. E), ridge acceptance off. */
 jarq_options jarq_default_options(void);
 
 /* Prepare a Hessian for refinement (Sec. 3.3.2, Eq. group_qr; App. G.7
@@ -149,6 +155,32 @@ jarq_status jarq_objective(jarq_hessian *h, const float *W, const float *S, cons
 jarq_status jarq_residual_product(jarq_hessian *h, const float *W, const float *S,
                                   const uint8_t *Q, const int32_t *Z, int dout, int bits,
                                   float *HR, void *stream);
+
+/* ---- write-back of a refined layer (device memory only) ----
+ * These post-passes act on a layer already in device memory; host pointers
+ * return JARQ_ERR_ARG.  They allocate nothing and return after their work
+ * has finished.  Codes and zero points must lie in [0, 2^bits - 1]
+ * (JARQ_ERR_ARG otherwise, before any change). */
+
+/* Negative-scale canonicalisation (App. E "Representing Negative Scales",
+ * Eq. canonicalization): for every group with s < 0, s' = -s,
+ * q' = qmax - q, z' = qmax - z, which leaves s (q - z) unchanged.
+ *   S [dout][G] float32, Q [dout][din] uint8, Z [dout][G] int32: in place. */
+jarq_status jarq_canonicalize(float *S, uint8_t *Q, int32_t *Z, int dout, int din,
+                              int group_size, int bits, void *stream);
+
+/* The returned weights what = s (q - z) (Sec. 3.1, Eq. quantized_group),
+ * exact before one round-to-nearest-even to `dtype`, written to
+ * W_out [dout][din] (App. E: the refined weights are cast to the model's
+ * weight dtype). */
+jarq_status jarq_dequantize(const float *S, const uint8_t *Q, const int32_t *Z, int dout, int din,
+                            int group_size, int bits, jarq_dtype dtype, void *W_out, void *stream);
+
+/* b-bit codes packed per row into a little-endian bit stream: code k of a
+ * row occupies bits [k b, k b + b), cut into 32-bit words, the last word
+ * zero-padded.  packed [dout][ceil(din * bits / 32)] uint32. */
+jarq_status jarq_pack_codes(const uint8_t *Q, int dout, int din, int bits, uint32_t *packed,
+                            void *stream);
 
 /* Per-row objective without any device allocation.  The paper has no
  * counterpart: this entry point exists for callers that cannot allocate

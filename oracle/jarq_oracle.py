@@ -44,6 +44,9 @@ Readings of the paper that this oracle takes where the text is silent:
    objective, the Babai recursion and the acceptance test then run in
    float64 on those float32 scales.  ``fp32_scales=False`` keeps float64
    scales, for the paper's exact worked examples.
+8. ``Options.ridge_accept`` (off by default, as in the paper's runs) keeps a
+   ridge-stabilised solve only when it does not increase F_j, and the
+   previous scales otherwise (App. G, Remark ridge-acceptance).
 
 Parity status: every function here is pinned by ``tests/test_oracle_*.py``
 against the paper's worked examples (App. G, Props. grid-staleness and
@@ -75,6 +78,7 @@ class Options:
     rcond: float = 1e-10        # spectrum test threshold
     eps: float = FP32_EPS       # eps_fp
     fp32_scales: bool = True    # store each solved scale as float32 (reading 7)
+    ridge_accept: bool = False  # Remark ridge-acceptance: keep a ridge solve only if F does not rise
 
 
 @dataclasses.dataclass
@@ -330,7 +334,15 @@ def refine_layer(prep: Prepared, W, S0, Q0, Z, bits: int, opt: Options = None,
                 status[j] = ROW_NUMERICAL
                 active[j] = False
                 continue
+            s_old = S[j].copy()
             S[j] = s.astype(np.float32) if opt.fp32_scales else s
+            if used_ridge and opt.ridge_accept:
+                # Remark ridge-acceptance: the ridge solution is kept only when
+                # it does not increase F_j; otherwise the previous scales stay
+                F_new = objective(prep, W[j:j + 1], S[j:j + 1], Q[j:j + 1], Z[j:j + 1])[0]
+                F_old = objective(prep, W[j:j + 1], s_old[None], Q[j:j + 1], Z[j:j + 1])[0]
+                if not F_new <= F_old:
+                    S[j] = s_old
         rows = np.nonzero(active)[0]
         iters[rows] = k
         L = np.full(p, np.nan)

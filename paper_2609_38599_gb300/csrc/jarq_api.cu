@@ -302,6 +302,7 @@ jarq_options jarq_default_options(void) {
     o.ridge = 1e-4f;
     o.rcond = 1e-10f;
     o.eps = FLT_EPSILON;
+    o.ridge_accept = 0;
     return o;
 }
 

@@ -18,7 +18,9 @@
 //     float64), and stores s_new rounded to float32;
 //  4. evaluates L^{(k)} = F(s_new) = wHw - 2 s_new^T rhs + s_new^T Gram s_new
 //     at the stored float32 scales and applies the early stop of Eq.
-//     strict_stopping against L^{(k-1)}.
+//     strict_stopping against L^{(k-1)}; with the ridge-acceptance option a
+//     ridge-stabilised s_new that would raise F is dropped (App. G Remark
+//     ridge-acceptance).
 // In evaluation mode it only writes F(s) of the current state, for every
 // row.
 #include <float.h>
@@ -202,14 +204,19 @@ __global__ void scale_solve_kernel(SolveArgs a) {
         t1 += (double)y[r0] * rj[r0];
         t2 += (double)y[r0] * gs;
     }
-    const double L_new = a.wHw[j] - 2.0 * warp_sum(t1) + warp_sum(t2);
+    double L_new = a.wHw[j] - 2.0 * warp_sum(t1) + warp_sum(t2);
+    // Remark ridge-acceptance (optional): a ridge-stabilised solve that would
+    // raise F_j is dropped and the previous scales stay
+    const bool keep_old = used_ridge && a.o.ridge_accept && !(L_new <= F_old);
+    if (keep_old) L_new = F_old;
     bool stop = false;
     if (a.o.early_stop && a.k >= 2) {
         const double dec = a.L_prev[j] - L_new;
         const double den = fmax(fabs(a.L_prev[j]), (double)a.o.eps);
         stop = (dec / den <= (double)a.o.tau_rel) || (fabs(dec) <= (double)a.o.tau_abs);
     }
-    for (int t = lane; t < G; t += 32) a.S[(size_t)j * G + t] = y[t];
+    if (!keep_old)
+        for (int t = lane; t < G; t += 32) a.S[(size_t)j * G + t] = y[t];
     if (lane == 0) {
         a.L_prev[j] = L_new;
         a.iters[j] = a.k;

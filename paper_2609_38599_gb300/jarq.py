@@ -30,7 +30,8 @@ EXPORTS = ("jarq_default_options", "jarq_prepare_hessian", "jarq_refine_layer",
            "jarq_objective", "jarq_hessian_din", "jarq_hessian_group_size",
            "jarq_hessian_destroy", "jarq_status_string", "jarq_profile_enable",
            "jarq_profile_reset", "jarq_profile_read", "jarq_launch_count",
-           "jarq_objective_noalloc", "jarq_residual_product")
+           "jarq_objective_noalloc", "jarq_residual_product", "jarq_canonicalize",
+           "jarq_dequantize", "jarq_pack_codes")
 
 
 class JarqError(RuntimeError):
@@ -43,7 +44,7 @@ class Options(ctypes.Structure):
     _fields_ = [("max_iters", ctypes.c_int), ("early_stop", ctypes.c_int),
                 ("tau_rel", ctypes.c_float), ("tau_abs", ctypes.c_float),
                 ("ridge", ctypes.c_float), ("rcond", ctypes.c_float),
-                ("eps", ctypes.c_float)]
+                ("eps", ctypes.c_float), ("ridge_accept", ctypes.c_int)]
 
 
 class Stats(ctypes.Structure):
@@ -71,6 +72,12 @@ def _load():
     lib.jarq_objective_noalloc.argtypes = [vp, vp, vp, vp, vp, ci, ci, vp, vp]
     lib.jarq_residual_product.restype = ci
     lib.jarq_residual_product.argtypes = [vp, vp, vp, vp, vp, ci, ci, vp, vp]
+    lib.jarq_canonicalize.restype = ci
+    lib.jarq_canonicalize.argtypes = [vp, vp, vp, ci, ci, ci, ci, vp]
+    lib.jarq_dequantize.restype = ci
+    lib.jarq_dequantize.argtypes = [vp, vp, vp, ci, ci, ci, ci, ci, vp, vp]
+    lib.jarq_pack_codes.restype = ci
+    lib.jarq_pack_codes.argtypes = [vp, ci, ci, ci, vp, vp]
     lib.jarq_hessian_din.restype = ci
     lib.jarq_hessian_din.argtypes = [vp]
     lib.jarq_hessian_group_size.restype = ci
@@ -263,6 +270,53 @@ def residual_product(hess: Hessian, W, S, Q, Z, bits: int, out=None):
                                         _ptr(out, np.float32), _stream(W, S, Q, Z))
     if status != JARQ_OK:
         raise JarqError(status, "jarq_residual_product")
+    return out
+
+
+JARQ_F32, JARQ_F16, JARQ_BF16 = 0, 1, 2
+
+
+def _dev_stream(*ts):
+    import torch
+    return ctypes.c_void_p(torch.cuda.current_stream(ts[0].device).cuda_stream)
+
+
+def canonicalize(S, Q, Z, group_size: int, bits: int):
+    """``jarq_canonicalize``: negative scales to the equivalent positive form,
+    in place on device tensors (S float32, Q uint8, Z int32)."""
+    dout, din = int(Q.shape[0]), int(Q.shape[1])
+    status = _lib.jarq_canonicalize(_ptr(S, np.float32), _ptr(Q, np.uint8), _ptr(Z, np.int32),
+                                    dout, din, int(group_size), int(bits), _dev_stream(S))
+    if status != JARQ_OK:
+        raise JarqError(status, "jarq_canonicalize")
+
+
+def dequantize(S, Q, Z, group_size: int, bits: int, dtype: str = "float16"):
+    """``jarq_dequantize``: s (q - z) in float32, float16 or bfloat16 (device tensors)."""
+    import torch
+    code = {"float32": JARQ_F32, "float16": JARQ_F16, "bfloat16": JARQ_BF16}[dtype]
+    tdt = {"float32": torch.float32, "float16": torch.float16, "bfloat16": torch.bfloat16}[dtype]
+    dout, din = int(Q.shape[0]), int(Q.shape[1])
+    out = torch.empty(dout, din, dtype=tdt, device=Q.device)
+    status = _lib.jarq_dequantize(_ptr(S, np.float32), _ptr(Q, np.uint8), _ptr(Z, np.int32), dout,
+                                  din, int(group_size), int(bits), code,
+                                  ctypes.c_void_p(out.data_ptr()), _dev_stream(S))
+    if status != JARQ_OK:
+        raise JarqError(status, "jarq_dequantize")
+    return out
+
+
+def pack_codes(Q, bits: int):
+    """``jarq_pack_codes``: b-bit codes packed per row (int32 storage of the
+    uint32 words, [dout][ceil(din b / 32)])."""
+    import torch
+    dout, din = int(Q.shape[0]), int(Q.shape[1])
+    nw = (din * int(bits) + 31) // 32
+    out = torch.empty(dout, nw, dtype=torch.int32, device=Q.device)
+    status = _lib.jarq_pack_codes(_ptr(Q, np.uint8), dout, din, int(bits),
+                                  ctypes.c_void_p(out.data_ptr()), _dev_stream(Q))
+    if status != JARQ_OK:
+        raise JarqError(status, "jarq_pack_codes")
     return out
 
 
