@@ -6,10 +6,12 @@ baseline of ``bench.py`` use this package.  The product path never imports it.
 from .jarq_oracle import (FP32_EPS, Options, Prepared, Result, babai_proposal, canonicalize,
                           code_sweep, dequantize, group_target, objective, prepare_hessian,
                           refine_layer, scale_system, solve_scales)
+from .jarq_hessian import accumulate_hessian, augmented_hessian
 from .jarq_format import (dequantize_cast, pack_codes, packed_words, round_to_bfloat16,
                           unpack_codes)
 
 __all__ = ["FP32_EPS", "Options", "Prepared", "Result", "babai_proposal", "canonicalize",
            "code_sweep", "dequantize", "group_target", "objective", "prepare_hessian",
            "refine_layer", "scale_system", "solve_scales", "dequantize_cast", "pack_codes",
-           "packed_words", "round_to_bfloat16", "unpack_codes"]
+           "packed_words", "round_to_bfloat16", "unpack_codes", "accumulate_hessian",
+           "augmented_hessian"]
