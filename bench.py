@@ -49,6 +49,7 @@ TRAFFIC = {
     "ptilde": ("k_tc_proj.cu", "391ad329f213", 138.978e6 + 90.157056e6),
     "scale_solve": ("k_solve.cu", "0b9a43feec9b", 35.256e6 + 0.001024e6),
 }
+HESSIAN_WORKLOAD = "llama2_7b_attn_in_4096_n262144"
 
 
 def traffic_for(kernel):
@@ -72,6 +73,8 @@ def parse_args():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default=WORKLOAD)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--tokens", type=int, default=None,
+                    help="calibration tokens of the Hessian workload (default: 128 x 2048)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="target CPU time of the oracle baseline sample")
     return ap.parse_args()
@@ -403,6 +406,8 @@ def run_ours(args, rank, world):
                           "hbm_frac": by / (ms_ / 1e3) / 1e9 / pk2["hbm_gbs"],
                           "note": "includes the code validation pass and a synchronize"}
         line["postpass"] = post
+    if rank == 0:
+        line["hessian"] = hessian_leg(args, jarq, dev)
     # end to end through the C ABI with pinned host buffers
     if rank == 0 or True:
         pin = lambda t: t.cpu().pin_memory().numpy()
@@ -439,6 +444,90 @@ def run_ours(args, rank, world):
         print(json.dumps(line))
     if dist:
         dist.destroy_process_group()
+    return 0
+
+
+def hessian_leg(args, jarq, dev, standalone=False):
+    """The calibration Hessian H = X^T X of the q/k/v/gate/up input of a
+    Llama-2-7B block (d = 4096) over 128 x 2048 fp16 tokens, one
+    ``jarq_accumulate_hessian`` call: the step before refinement.  Timed by
+    the library's CUDA event pair on its stream (kernel) and around the call
+    (which synchronises).  Algorithmic work counts each unordered feature
+    pair once: n d (d + 1) flops; the kernel issues whole 128 x 256 tiles
+    meeting the upper triangle."""
+    import torch
+    from synth import ACT_CONFIGS, config_activations
+    X = config_activations(HESSIAN_WORKLOAD, device=dev, tokens=args.tokens)
+    n, d = X.shape
+    H = torch.zeros(d, d, device=dev)
+    for _ in range(max(3, args.warmup)):
+        jarq.accumulate_hessian(X, H)
+    torch.cuda.synchronize()
+    reps = max(1, args.steps) if standalone else 5
+    jarq.profile_reset()
+    jarq.profile_enable(True)
+    t0 = time.perf_counter()
+    for _ in range(reps):
+        jarq.accumulate_hessian(X, H)
+    call_ms = (time.perf_counter() - t0) / reps * 1e3
+    jarq.profile_enable(False)
+    nl, tot = jarq.profile_read("syrk")
+    k_ms = tot / max(1, nl)
+    pk, peak_kind = peaks()
+    work = float(n) * d * (d + 1)
+    rt, ct = (d + 127) // 128, (d + 255) // 256
+    tiles = sum(min(rt, 2 * cj + 2) for cj in range(ct))
+    issued = tiles * 2.0 * 128 * 256 * (-(-n // 64) * 64)
+    achieved = work / (k_ms / 1e3) / 1e12
+    peak = pk["bf16_tflops"]
+    out = {"workload": HESSIAN_WORKLOAD, "tokens": n, "din": d, "call_ms": call_ms,
+           "kernel_ms": k_ms, "tokens_per_s": n / (k_ms / 1e3),
+           "roofline": {"kernel": "syrk", "bound": "tensor", "achieved": achieved, "peak": peak,
+                        "unit": "TFLOP/s", "frac": achieved / peak,
+                        "issued_frac": issued / (k_ms / 1e3) / 1e12 / peak,
+                        "traffic": traffic_for("syrk"),
+                        "peak_note": f"fp16 dense = bf16 dense rate, burst ({peak_kind})"},
+           "l2": f"X is {n * d * 2 / 2**20:.0f} MiB, larger than the 129 MB L2",
+           "data": "synthetic fp16 activations (rank-64 correlated + outlier channels)"}
+    del X, H
+    torch.cuda.empty_cache()
+    if not args.no_cpu_baseline:
+        from oracle import accumulate_hessian
+        from synth import activations_np
+        c = ACT_CONFIGS[HESSIAN_WORKLOAD]
+        ns = 4096
+        Xs = activations_np(ns, d, rank=c["rank"], n_out=c["n_out"], out_scale=c["out_scale"],
+                            D_lo=c["D_lo"], seed=c["seed"])
+        t0 = time.perf_counter()
+        accumulate_hessian(Xs)
+        t = time.perf_counter() - t0
+        out["cpu_baseline"] = {"value": ns / t, "unit": "tokens/s", "cores": os.cpu_count(),
+                               "kind": "oracle",
+                               "sample": f"{ns} of {n} tokens, d={d}, float64, {t:.2f} s"}
+    return out
+
+
+def run_hessian(args, rank, world):
+    """``--workload llama2_7b_attn_in_4096_n262144``: the Hessian step alone,
+    one line of its own (tokens/s)."""
+    import torch
+    from paper_2609_38599_gb300 import jarq
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", "0")))
+    torch.cuda.set_device(dev)
+    n0 = jarq.launch_count()
+    h = hessian_leg(args, jarq, dev, standalone=True)
+    line = {"metric": "calibration Hessian X^T X, tokens/s", "value": world * h["tokens_per_s"],
+            "unit": "tokens/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": h["kernel_ms"], "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "fp16 products, f32 sums", "data": h["data"],
+            "config": {"workload": HESSIAN_WORKLOAD, "tokens": h["tokens"], "din": h["din"],
+                       "l2": h["l2"]},
+            "roofline": h["roofline"], "gpu_launches": jarq.launch_count() - n0,
+            "call_ms": h["call_ms"]}
+    if "cpu_baseline" in h:
+        line["cpu_baseline"] = h["cpu_baseline"]
+    if rank == 0:
+        print(json.dumps(line))
     return 0
 
 
@@ -513,6 +602,8 @@ def main():
         return run_reference(args, rank, world)
     if args.workload == BLOCK_WORKLOAD:
         return run_block(args, rank, world)
+    if args.workload == HESSIAN_WORKLOAD:
+        return run_hessian(args, rank, world)
     return run_ours(args, rank, world)
 
 

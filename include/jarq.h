@@ -182,6 +182,33 @@ jarq_status jarq_dequantize(const float *S, const uint8_t *Q, const int32_t *Z, 
 jarq_status jarq_pack_codes(const uint8_t *Q, int dout, int din, int bits, uint32_t *packed,
                             void *stream);
 
+/* ---- calibration Hessian (device memory only) ----
+ * H <- H + scale * X^T X, the activation part of the Hessian H = A^T A of
+ * the augmented design A = [X~; nu I] (Sec. 3.2, Eq. strict_target; the
+ * paper writes H = X~^T X~ + nu^2 I out in its appendix on
+ * propagation-corrected targets).  nu^2 I is added by jarq_prepare_hessian.
+ * Called once per batch of calibration tokens, it accumulates H over an
+ * activation stream.
+ *   X     : device, float16 [n][d] row-major, one token per row (the layer's
+ *           inputs as the preceding quantized layers produce them), 16-byte
+ *           aligned; d a multiple of 8, 8 <= d <= 65536.  Not modified.
+ *   n     : tokens in this batch, >= 0 (0: nothing to do, H untouched).
+ *   scale : finite multiplier of the batch's product (1 for the paper's H).
+ *   H     : device, float32 [d][d] row-major, read and written in place;
+ *           every element, both triangles, becomes
+ *           fl(H[i][j] + scale * sum_t X[t][i] X[t][j]), so a symmetric H
+ *           stays exactly symmetric.  Must not overlap X.
+ * Precision: the fp16 products are exact (the paper forms its products from
+ * FP16 activations in FP32, App. "Metrics"); they are summed in float32 on
+ * the tensor cores over blocks of 512 tokens, the block sums in float32,
+ * and the result is added to H with one rounding.
+ * Errors: JARQ_ERR_ARG (sizes, a non-finite scale, null, host or misaligned
+ * pointers; nothing enqueued), JARQ_ERR_TIMEOUT (a bounded device wait gave
+ * up; H is then unspecified), JARQ_ERR_CUDA.  Returns after the update has
+ * finished. */
+jarq_status jarq_accumulate_hessian(const void *X, int n, int d, float scale, float *H,
+                                    void *stream);
+
 /* Per-row objective without any device allocation.  The paper has no
  * counterpart: this entry point exists for callers that cannot allocate
  * device memory when they need the objective -- code running while a CUDA
@@ -223,7 +250,8 @@ const char *jarq_status_string(jarq_status s);
  * kernel launch it makes; durations are accumulated per kernel name when the
  * enclosing call synchronises.  Names: "validate", "residual", "init_rows",
  * "hr_full", "grad", "gram", "scale_solve", "phase_hr", "babai",
- * "symmetrize", "group_factor", "slices".  Not thread-safe. */
+ * "symmetrize", "group_factor", "slices", "slice_rows", "proj", "whw", "rhs",
+ * "htilde", "ptilde", "target", "syrk".  Not thread-safe. */
 void jarq_profile_enable(int on);
 void jarq_profile_reset(void);
 /* Accumulated launches and total device milliseconds of one kernel name since

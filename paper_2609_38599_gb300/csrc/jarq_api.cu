@@ -16,38 +16,7 @@
 
 #include "jarq_internal.cuh"
 
-using namespace jarq;
-
-namespace {
-
-jarq_status cuda_fail(cudaError_t e) {
-    return e == cudaErrorMemoryAllocation ? JARQ_ERR_NOMEM : JARQ_ERR_CUDA;
-}
-
-#define CK(x)                                  \
-    do {                                       \
-        cudaError_t e_ = (x);                  \
-        if (e_ != cudaSuccess) {               \
-            (void)cudaGetLastError();          \
-            return cuda_fail(e_);              \
-        }                                      \
-    } while (0)
-
-// Launch `call` (which enqueues `n` kernels) under the profiling scope `name`.
-#define RUN(name, n, call)              \
-    do {                                \
-        ProfScope ps_(name, st);        \
-        CK(call);                       \
-        ps_.done();                     \
-        count_launches(n);              \
-    } while (0)
-
-template <class T>
-cudaError_t dalloc(T **p, size_t n) {
-    *p = nullptr;
-    if (n == 0) n = 1;
-    return cudaMalloc((void **)p, n * sizeof(T));
-}
+namespace jarq {
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
                                   const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
@@ -87,6 +56,41 @@ cudaError_t make_tmap_bf16(CUtensorMap *m, const void *base, uint64_t rows, uint
 cudaError_t make_tmap_f16(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols,
                           uint32_t box_rows) {
     return make_tmap_2b(m, base, rows, cols, box_rows, CU_TENSOR_MAP_DATA_TYPE_FLOAT16);
+}
+
+}  // namespace jarq
+
+using namespace jarq;
+
+namespace {
+
+jarq_status cuda_fail(cudaError_t e) {
+    return e == cudaErrorMemoryAllocation ? JARQ_ERR_NOMEM : JARQ_ERR_CUDA;
+}
+
+#define CK(x)                                  \
+    do {                                       \
+        cudaError_t e_ = (x);                  \
+        if (e_ != cudaSuccess) {               \
+            (void)cudaGetLastError();          \
+            return cuda_fail(e_);              \
+        }                                      \
+    } while (0)
+
+// Launch `call` (which enqueues `n` kernels) under the profiling scope `name`.
+#define RUN(name, n, call)              \
+    do {                                \
+        ProfScope ps_(name, st);        \
+        CK(call);                       \
+        ps_.done();                     \
+        count_launches(n);              \
+    } while (0)
+
+template <class T>
+cudaError_t dalloc(T **p, size_t n) {
+    *p = nullptr;
+    if (n == 0) n = 1;
+    return cudaMalloc((void **)p, n * sizeof(T));
 }
 
 // Split-K factor of the phase product: enough CTAs to cover the SMs.

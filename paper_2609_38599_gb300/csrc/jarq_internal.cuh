@@ -225,6 +225,19 @@ cudaError_t launch_init_rows(int *active, int *iters, int *accepted, int *ridge,
 
 int num_sms();
 
+// True for device (or managed) memory of the current context.
+bool on_device(const void *p);
+
+// 2D tensor map of 2-byte elements (bf16 or fp16) over [rows][cols]
+// (pitch = cols elements), box_rows x 64 boxes, 128-byte swizzle,
+// out-of-range elements read as zero.
+cudaError_t make_tmap_2b(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols,
+                         uint32_t box_rows, CUtensorMapDataType dtype);
+cudaError_t make_tmap_bf16(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols,
+                           uint32_t box_rows);
+cudaError_t make_tmap_f16(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols,
+                          uint32_t box_rows);
+
 // ---- instrumentation (prof.cu) ----
 void count_launches(int n);
 void prof_collect();

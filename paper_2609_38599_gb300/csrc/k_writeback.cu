@@ -72,15 +72,6 @@ __global__ void pack_codes_kernel(const uint8_t *__restrict__ Q, uint32_t *__res
     }
 }
 
-bool on_device(const void *p) {
-    cudaPointerAttributes at;
-    if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
-        (void)cudaGetLastError();
-        return false;
-    }
-    return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
-}
-
 int grid_for(size_t n) {
     size_t b = (n + 255) / 256;
     const size_t cap = (size_t)8 * num_sms();
@@ -119,6 +110,16 @@ jarq_status checked_run(const uint8_t *Q, const int32_t *Z, int p, int d, int G,
 }
 
 }  // namespace
+
+bool on_device(const void *p) {
+    cudaPointerAttributes at;
+    if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return false;
+    }
+    return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
+}
+
 }  // namespace jarq
 
 using namespace jarq;

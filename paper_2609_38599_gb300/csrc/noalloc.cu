@@ -64,15 +64,6 @@ bool encode_planes_map(CUtensorMap *m, void *base, uint64_t rows, uint64_t cols)
            CUDA_SUCCESS;
 }
 
-bool on_device(const void *p) {
-    cudaPointerAttributes at;
-    if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
-        (void)cudaGetLastError();
-        return false;
-    }
-    return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
-}
-
 }  // namespace
 }  // namespace jarq
 

@@ -31,7 +31,7 @@ EXPORTS = ("jarq_default_options", "jarq_prepare_hessian", "jarq_refine_layer",
            "jarq_hessian_destroy", "jarq_status_string", "jarq_profile_enable",
            "jarq_profile_reset", "jarq_profile_read", "jarq_launch_count",
            "jarq_objective_noalloc", "jarq_residual_product", "jarq_canonicalize",
-           "jarq_dequantize", "jarq_pack_codes")
+           "jarq_dequantize", "jarq_pack_codes", "jarq_accumulate_hessian")
 
 
 class JarqError(RuntimeError):
@@ -78,6 +78,8 @@ def _load():
     lib.jarq_dequantize.argtypes = [vp, vp, vp, ci, ci, ci, ci, ci, vp, vp]
     lib.jarq_pack_codes.restype = ci
     lib.jarq_pack_codes.argtypes = [vp, ci, ci, ci, vp, vp]
+    lib.jarq_accumulate_hessian.restype = ci
+    lib.jarq_accumulate_hessian.argtypes = [vp, ci, ci, cf, vp, vp]
     lib.jarq_hessian_din.restype = ci
     lib.jarq_hessian_din.argtypes = [vp]
     lib.jarq_hessian_group_size.restype = ci
@@ -108,7 +110,7 @@ def library():
 
 KERNELS = ("validate", "residual", "init_rows", "hr_full", "grad", "gram", "scale_solve",
            "phase_hr", "babai", "symmetrize", "group_factor", "slices", "slice_rows", "proj",
-           "whw", "rhs", "htilde", "ptilde", "target")
+           "whw", "rhs", "htilde", "ptilde", "target", "syrk")
 
 
 def profile_enable(on: bool = True):
@@ -318,6 +320,23 @@ def pack_codes(Q, bits: int):
     if status != JARQ_OK:
         raise JarqError(status, "jarq_pack_codes")
     return out
+
+
+def accumulate_hessian(X, H=None, scale: float = 1.0):
+    """``jarq_accumulate_hessian``: ``H + scale * X^T X`` for a float16 device
+    tensor X [tokens][din]; H (float32 [din][din], device) is updated in place
+    and returned (a zero matrix when H is None)."""
+    import torch
+    if not (_is_torch(X) and X.is_cuda and X.dtype == torch.float16 and X.is_contiguous()):
+        raise TypeError("X must be a contiguous float16 CUDA tensor [tokens][din]")
+    n, d = int(X.shape[0]), int(X.shape[1])
+    if H is None:
+        H = torch.zeros(d, d, dtype=torch.float32, device=X.device)
+    status = _lib.jarq_accumulate_hessian(ctypes.c_void_p(X.data_ptr()), n, d, float(scale),
+                                          _ptr(H, np.float32), _dev_stream(X))
+    if status != JARQ_OK:
+        raise JarqError(status, "jarq_accumulate_hessian")
+    return H
 
 
 def objective(hess: Hessian, W, S, Q, Z, bits: int, out=None):
