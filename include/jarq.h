@@ -194,7 +194,8 @@ jarq_status jarq_pack_codes(const uint8_t *Q, int dout, int din, int bits, uint3
  *           aligned; d a multiple of 8, 8 <= d <= 65536.  Not modified.
  *   n     : tokens in this batch, >= 0 (0: nothing to do, H untouched).
  *   scale : finite multiplier of the batch's product (1 for the paper's H).
- *   H     : device, float32 [d][d] row-major, read and written in place;
+ *   H     : device, float32 [d][d] row-major, 16-byte aligned, read and
+ *           written in place;
  *           every element, both triangles, becomes
  *           fl(H[i][j] + scale * sum_t X[t][i] X[t][j]), so a symmetric H
  *           stays exactly symmetric.  Must not overlap X.

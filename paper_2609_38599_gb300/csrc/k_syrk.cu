@@ -21,9 +21,10 @@
 //               M128 x N256 x K16 MMA per 16 tokens
 //   warps 2..9  drain: every 512 tokens the TMEM accumulator (restarted at
 //               zero, two of them alternate) is added into float32
-//               registers.  At the end the tile goes through shared memory
-//               and is added to H with coalesced stores, once as H[row][col]
-//               and once mirrored as H[col][row].
+//               registers.  At the end the tile is added to H twice with
+//               coalesced accesses: mirrored, H[col][row], straight from the
+//               registers (a warp's 32 rows are contiguous there), and as
+//               H[row][col] in float4 through shared memory.
 // Each unordered pair {i, j} belongs to exactly one tile element with
 // col >= row, so every element of H is written exactly once.
 #include <math.h>
@@ -82,6 +83,54 @@ __device__ __forceinline__ void tile_of(int t, int rt, int ct, int &ri, int &cj)
         t -= m;
     }
     ri = t;
+}
+
+// One pass of the tile update H += scale * T over 256 threads, as float4
+// read-modify-writes of H with 8 loads in flight per thread.  MIRROR false:
+// H[r0+i][c0+j] for c0+j >= r0+i (float4 along j, 128 rows x 64); MIRROR
+// true: H[c0+j][r0+i] for c0+j > r0+i (float4 along i, 256 rows x 32).  A
+// float4 that straddles the diagonal updates its own elements only.
+template <bool MIRROR>
+__device__ __forceinline__ void add_tile_pass(const SyrkArgs &a, const float *T, int t, int r0,
+                                              int c0) {
+    constexpr int kSh = MIRROR ? 5 : 6;           // float4 per H row segment: 32 or 64
+#pragma unroll 1
+    for (int k0 = 0; k0 < 32; k0 += 8) {
+        float4 h[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const int idx = t + 256 * (k0 + k);
+            const int u = idx >> kSh, v4 = 4 * (idx & ((1 << kSh) - 1));
+            const int hr = MIRROR ? c0 + u : r0 + u, hc = MIRROR ? r0 + v4 : c0 + v4;
+            // all four elements on the kept side of the diagonal
+            const bool full = hr < a.d && hc < a.d && (MIRROR ? hr > hc + 3 : hc >= hr);
+            h[k] = full ? *reinterpret_cast<const float4 *>(a.H + (size_t)hr * a.d + hc)
+                        : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const int idx = t + 256 * (k0 + k);
+            const int u = idx >> kSh, v4 = 4 * (idx & ((1 << kSh) - 1));
+            const int hr = MIRROR ? c0 + u : r0 + u, hc = MIRROR ? r0 + v4 : c0 + v4;
+            if (hr >= a.d || hc >= a.d) continue;
+            // tile element of H[hr][hc + m]
+            auto tv = [&](int m) {
+                return MIRROR ? T[(v4 + m) * kTld + u] : T[u * kTld + v4 + m];
+            };
+            float *hp = a.H + (size_t)hr * a.d + hc;
+            if (MIRROR ? hr > hc + 3 : hc >= hr) {
+                float4 v = h[k];
+                v.x = fmaf(a.scale, tv(0), v.x);
+                v.y = fmaf(a.scale, tv(1), v.y);
+                v.z = fmaf(a.scale, tv(2), v.z);
+                v.w = fmaf(a.scale, tv(3), v.w);
+                *reinterpret_cast<float4 *>(hp) = v;
+            } else {
+                for (int m = 0; m < 4; ++m)
+                    if (MIRROR ? hr > hc + m : hc + m >= hr) hp[m] = fmaf(a.scale, tv(m), hp[m]);
+            }
+        }
+    }
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -222,8 +271,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             __syncwarp();
             if (lane == 0) tc::mbar_arrive(aempty(b));
         }
-        // the stage ring is idle once the last accumulator has been read
-        // (or the CTA gives up); stage the tile as T[row][col]
+        // the stage ring is idle once the last accumulator has been read:
+        // stage the tile as T[row][col]
         float *T = (float *)smem;
         if (!*abort_flag) {
             const int i = 32 * q + lane;
@@ -233,24 +282,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         asm volatile("bar.sync 1, 256;" ::: "memory");
         if (!*abort_flag) {
             const int t = threadIdx.x - 64;
-            // H[row][col] for col >= row: consecutive threads, consecutive columns
-            for (int idx = t; idx < 128 * 256; idx += 256) {
-                const int i = idx >> 8, j = idx & 255;
-                const int row = r0 + i, col = c0 + j;
-                if (row < a.d && col < a.d && col >= row) {
-                    float *h = a.H + (size_t)row * a.d + col;
-                    *h = fmaf(a.scale, T[i * kTld + j], *h);
-                }
-            }
-            // H[col][row] for col > row: consecutive threads, consecutive rows
-            for (int idx = t; idx < 128 * 256; idx += 256) {
-                const int j = idx >> 7, i = idx & 127;
-                const int row = r0 + i, col = c0 + j;
-                if (row < a.d && col < a.d && col > row) {
-                    float *h = a.H + (size_t)col * a.d + row;
-                    *h = fmaf(a.scale, T[i * kTld + j], *h);
-                }
-            }
+            // H[row][col] for col >= row: a tile row is 64 float4 of H's row
+            add_tile_pass<false>(a, T, t, r0, c0);
+            // H[col][row] for col > row: a tile column is 32 float4 of H's row `col`
+            add_tile_pass<true>(a, T, t, r0, c0);
         }
     }
     tc::tc_fence_before();
@@ -278,7 +313,7 @@ using namespace jarq;
 extern "C" jarq_status jarq_accumulate_hessian(const void *X, int n, int d, float scale, float *H,
                                                void *stream) {
     if (n < 0 || d < 8 || d % 8 || d > 65536 || !isfinite(scale)) return JARQ_ERR_ARG;
-    if (!H || !on_device(H)) return JARQ_ERR_ARG;
+    if (!H || !on_device(H) || ((uintptr_t)H & 15)) return JARQ_ERR_ARG;
     if (n == 0) return JARQ_OK;
     if (!X || !on_device(X) || ((uintptr_t)X & 15)) return JARQ_ERR_ARG;
     cudaStream_t st = (cudaStream_t)stream;

@@ -99,6 +99,12 @@ def test_zero_tokens_and_bad_arguments(jarq):
         jarq.accumulate_hessian(Xm, H)
     assert ei.value.status == JARQ_ERR_ARG
     assert bool((H == 3.0).all())
+    # H not 16-byte aligned
+    hbuf = torch.zeros(d * d + 1, device="cuda")
+    with pytest.raises(JarqError) as ei:
+        jarq.accumulate_hessian(torch.ones(16, d, dtype=torch.float16, device="cuda"),
+                                hbuf[1:].view(d, d))
+    assert ei.value.status == JARQ_ERR_ARG
     # host H
     Hh = np.zeros((d, d), np.float32)
     Xd = torch.ones(16, d, dtype=torch.float16, device="cuda")
