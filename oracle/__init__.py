@@ -7,6 +7,7 @@ from .jarq_oracle import (FP32_EPS, Options, Prepared, Result, babai_proposal, c
                           code_sweep, dequantize, group_target, objective, prepare_hessian,
                           refine_layer, scale_system, solve_scales)
 from .jarq_hessian import accumulate_hessian, augmented_hessian
+from .jarq_qep import corrected_weights, mu_constant, refine_mu, target_energy
 from .jarq_format import (dequantize_cast, pack_codes, packed_words, round_to_bfloat16,
                           unpack_codes)
 
@@ -14,4 +15,4 @@ __all__ = ["FP32_EPS", "Options", "Prepared", "Result", "babai_proposal", "canon
            "code_sweep", "dequantize", "group_target", "objective", "prepare_hessian",
            "refine_layer", "scale_system", "solve_scales", "dequantize_cast", "pack_codes",
            "packed_words", "round_to_bfloat16", "unpack_codes", "accumulate_hessian",
-           "augmented_hessian"]
+           "augmented_hessian", "corrected_weights", "mu_constant", "refine_mu", "target_energy"]

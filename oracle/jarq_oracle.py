@@ -297,7 +297,7 @@ class Result:
 
 
 def refine_layer(prep: Prepared, W, S0, Q0, Z, bits: int, opt: Options = None,
-                 trace=None) -> Result:
+                 trace=None, const=None) -> Result:
     """JARQ's alternating refinement of one layer (Sec. 3.3; App. E).
 
     For ``k = 1..K`` each active row (i) refits all G scales jointly for its
@@ -305,6 +305,12 @@ def refine_layer(prep: Prepared, W, S0, Q0, Z, bits: int, opt: Options = None,
     stop of Eq. strict_stopping for ``k >= 2``, then (ii) runs one bounded
     Babai sweep over its groups on the new scales (Sec. 3.3.2).  Rows are
     independent (Sec. 3.3, "separates over output columns").
+
+    ``const`` (optional, per row) is a constant added to every objective
+    value L: a target outside the range of A contributes the orthogonal
+    residual c_j, which Algorithm 1 carries in its objective (App.
+    "Propagation-Corrected Targets and QEP"); it moves the early-stop test and
+    the reported L, never a scale or a code.
     """
     opt = opt or Options()
     W = np.asarray(W, dtype=np.float64)
@@ -314,7 +320,8 @@ def refine_layer(prep: Prepared, W, S0, Q0, Z, bits: int, opt: Options = None,
     p = W.shape[0]
     if Q.min(initial=0) < 0 or Q.max(initial=0) > (1 << bits) - 1:
         raise ValueError("codes outside the b-bit range")
-    L_host = objective(prep, W, S, Q, Z)
+    c = np.zeros(p) if const is None else np.asarray(const, dtype=np.float64)
+    L_host = objective(prep, W, S, Q, Z) + c
     active = np.ones(p, dtype=bool)
     iters = np.zeros(p, dtype=np.int64)
     accepted = np.zeros(p, dtype=np.int64)
@@ -346,7 +353,7 @@ def refine_layer(prep: Prepared, W, S0, Q0, Z, bits: int, opt: Options = None,
         rows = np.nonzero(active)[0]
         iters[rows] = k
         L = np.full(p, np.nan)
-        L[rows] = objective(prep, W[rows], S[rows], Q[rows], Z[rows])
+        L[rows] = objective(prep, W[rows], S[rows], Q[rows], Z[rows]) + c[rows]
         L_hist.append(L.copy())
         if trace is not None:
             trace.append(dict(kind="scale", k=k, rows=rows.copy(), S=S[rows].copy(), L=L[rows].copy()))
@@ -363,7 +370,7 @@ def refine_layer(prep: Prepared, W, S0, Q0, Z, bits: int, opt: Options = None,
         if trace is not None:
             trace.append(dict(kind="sweep", k=k, rows=rows.copy(),
                               F=objective(prep, W[rows], S[rows], Q[rows], Z[rows])))
-    L_final = objective(prep, W, S, Q, Z)
+    L_final = objective(prep, W, S, Q, Z) + c
     return Result(S=S, Q=Q, L_host=L_host, L_final=L_final, iters=iters,
                   accepted=accepted, ridge_hits=ridge_hits, row_status=status,
                   L_hist=L_hist)
