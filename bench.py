@@ -411,6 +411,7 @@ def run_ours(args, rank, world):
         line["postpass"] = post
     if rank == 0:
         line["hessian"] = hessian_leg(args, jarq, dev)
+        line["mu_target"] = mu_target_leg(args, jarq, dev, lay.name)
     # end to end through the C ABI with pinned host buffers
     if rank == 0 or True:
         pin = lambda t: t.cpu().pin_memory().numpy()
@@ -507,6 +508,46 @@ def hessian_leg(args, jarq, dev, standalone=False):
         out["cpu_baseline"] = {"value": ns / t, "unit": "tokens/s", "cores": os.cpu_count(),
                                "kind": "oracle",
                                "sample": f"{ns} of {n} tokens, d={d}, float64, {t:.2f} s"}
+    return out
+
+
+def mu_target_leg(args, jarq, dev, name):
+    """The same layer shape refined on the propagation-corrected target
+    (mu = 0.5; H, K = X~^T X and XX = X^T X from 128 x 2048 drifted fp16
+    tokens) against the main target (mu = 1) on the same H: per-layer time
+    of each, CUDA events on the launching stream, five timed calls after
+    three warm-up calls."""
+    import torch
+    from synth.qep import mu_config_layer
+    lay, K, XX, nu2 = mu_config_layer(name, device=dev)
+    hess = jarq.prepare(lay.H, lay.g)
+    opts = jarq.default_options(max_iters=lay.K, early_stop=0)
+    S, Q = lay.S0.clone(), lay.Q0.clone()
+
+    def run(mu):
+        S.copy_(lay.S0)
+        Q.copy_(lay.Q0)
+        jarq.refine_mu(hess, lay.W, S, Q, lay.Z, lay.bits, K, XX, mu, nu2, options=opts,
+                       collect_stats=False)
+
+    out = {}
+    for mu in (0.5, 1.0):
+        for _ in range(3):
+            run(mu)
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(5):
+            run(mu)
+        b.record()
+        torch.cuda.synchronize()
+        out[f"ms_per_layer_mu_{mu}"] = a.elapsed_time(b) / 5
+    out["extra_ms"] = out["ms_per_layer_mu_0.5"] - out["ms_per_layer_mu_1.0"]
+    out["weights_per_s_mu_0.5"] = lay.din * lay.dout / (out["ms_per_layer_mu_0.5"] / 1e3)
+    out["workload"] = name + " on the mu = 0.5 target (drift 0.05)"
+    hess.close()
+    del lay, K, XX
+    torch.cuda.empty_cache()
     return out
 
 

@@ -139,6 +139,33 @@ jarq_status jarq_refine_layer(jarq_hessian *h, const float *W, float *S, uint8_t
                               const int32_t *Z, int dout, int bits,
                               const jarq_options *opt, jarq_stats *stats, void *stream);
 
+/* Refinement on the propagation-corrected target (App. "Propagation-
+ * Corrected Targets and QEP", Eq. mu-target): the activation part of the
+ * target becomes Y*(mu) = (1 - mu) X W + mu X~ W, with X the layer's
+ * full-precision inputs and X~ the inputs after the quantized preceding
+ * layers; mu = 1 is the main target (this call is then jarq_refine_layer and
+ * K, XX are not read).  Equivalently (Eq. w-corr) the main problem on
+ * W_corr = W + (1 - mu) H^{-1} X~^T (X - X~) W plus a per-row constant; the
+ * library never forms H^{-1}: it replaces H w by H w_corr = mu H w +
+ * (1 - mu)(K w + nu2 w) and w^T H w by ||y(mu)||^2, both from exact
+ * tensor-core projections, and runs the same loop.  S, Q and the reported
+ * objectives (stats L_host, L_final) are those of the mu-target, constant
+ * included; early stopping uses them.
+ *   h, W, S, Q, Z, dout, bits, opt, stats, stream : as jarq_refine_layer; h
+ *        must be prepared from H = X~^T X~ + nu2 I.
+ *   K    : float32 [din][din], host or device: X~^T X, normalised like H.
+ *   XX   : float32 [din][din], host or device: X^T X, normalised like H.
+ *   mu   : in [0, 1].
+ *   nu2  : the nu^2 contained in the prepared H, >= 0 and finite.
+ * The first call with mu < 1 allocates the handle's digit planes for K and
+ * XX (6 din^2 bf16, kept until the handle is destroyed).  Errors as
+ * jarq_refine_layer; mu outside [0, 1], a non-finite or negative nu2, or a
+ * NULL K or XX with mu < 1 return JARQ_ERR_ARG. */
+jarq_status jarq_refine_layer_mu(jarq_hessian *h, const float *W, float *S, uint8_t *Q,
+                                 const int32_t *Z, int dout, int bits, const float *K,
+                                 const float *XX, float mu, float nu2, const jarq_options *opt,
+                                 jarq_stats *stats, void *stream);
+
 /* Per-row objective F_j = r_j^T H r_j, r_j = w_j - D_{s_j}(q_j - z_j)
  * (Sec. 3.2, Eq. bbmils_columns), written as double to F_per_row[dout]
  * (host or device).  Same layouts and checks as jarq_refine_layer. */
@@ -252,7 +279,7 @@ const char *jarq_status_string(jarq_status s);
  * enclosing call synchronises.  Names: "validate", "residual", "init_rows",
  * "hr_full", "grad", "gram", "scale_solve", "phase_hr", "babai",
  * "symmetrize", "group_factor", "slices", "slice_rows", "proj", "whw", "rhs",
- * "htilde", "ptilde", "target", "syrk".  Not thread-safe. */
+ * "htilde", "ptilde", "target", "syrk", "mu_combine".  Not thread-safe. */
 void jarq_profile_enable(int on);
 void jarq_profile_reset(void);
 /* Accumulated launches and total device milliseconds of one kernel name since

@@ -126,6 +126,7 @@ void free_ws(Workspace &w) {
     cudaFree(w.Phi);
     cudaFree(w.Plo);
     cudaFree(w.wHw);
+    cudaFree(w.aux);
     cudaFree(w.L_prev);
     cudaFree(w.L_host);
     cudaFree(w.L_final);
@@ -175,6 +176,7 @@ cudaError_t ensure_ws(jarq_hessian *h, int p) {
     if ((e = dalloc(&w.Phi, (size_t)p * d)) != cudaSuccess) return e;
     if ((e = dalloc(&w.Plo, (size_t)p * d)) != cudaSuccess) return e;
     if ((e = dalloc(&w.wHw, (size_t)p)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.aux, (size_t)p)) != cudaSuccess) return e;
     if ((e = dalloc(&w.L_prev, (size_t)p)) != cudaSuccess) return e;
     if ((e = dalloc(&w.L_host, (size_t)p)) != cudaSuccess) return e;
     if ((e = dalloc(&w.L_final, (size_t)p)) != cudaSuccess) return e;
@@ -293,6 +295,59 @@ bool layer_args_ok(const jarq_hessian *h, const void *W, const void *S, const vo
     return true;
 }
 
+// Inputs of the propagation-corrected target (App. "Propagation-Corrected
+// Targets and QEP"): K = X~^T X and XX = X^T X, float32 [d][d] with the
+// normalisation of the prepared H, and mu, nu^2.
+struct MuTarget {
+    const float *K, *XX;
+    float mu, nu2;
+};
+
+jarq_status refine_impl(jarq_hessian *h, const float *W, float *S, uint8_t *Q, const int32_t *Z,
+                        int dout, int bits, const jarq_options *opt, jarq_stats *stats,
+                        void *stream, const MuTarget *mt);
+
+// Digits of a d x d float32 matrix M (host or device) into the handle's
+// mu-target planes, then its target projection W M^T into (out_hi, out_lo).
+jarq_status project_by(jarq_hessian *h, const float *M, int p, float *out_hi, float *out_lo,
+                       cudaStream_t st) {
+    Workspace &w = h->ws;
+    const int d = h->din, g = h->g;
+    if (!h->qdig) {
+        CK(dalloc(&h->qdig, (size_t)6 * h->d_pad * h->d_pad));
+        CK(cudaMemset(h->qdig, 0, (size_t)6 * h->d_pad * h->d_pad * 2));
+        CK(dalloc(&h->qexp, (size_t)h->G * h->G));
+        CK(make_tmap_bf16(&h->mapQ, h->qdig, (uint64_t)6 * h->d_pad, h->d_pad, 64));
+    }
+    const float *Md = M;
+    if (!is_device_ptr(M)) {
+        if (!h->qstage) CK(dalloc(&h->qstage, (size_t)d * d));
+        CK(cudaMemcpyAsync(h->qstage, M, (size_t)d * d * sizeof(float), cudaMemcpyHostToDevice, st));
+        Md = h->qstage;
+    }
+    RUN("slices", 2, launch_slices8(Md, h->qexp, h->qdig, d, h->d_pad, g, st));
+    RUN("proj", 1, launch_tc_proj(w.mapWd, h->mapQ, out_hi, out_lo, w.wexp, h->qexp, p, w.p_pad,
+                                  d, h->d_pad, g, h->dstatus, st));
+    return JARQ_OK;
+}
+
+// H w_corr and ||y(mu)||^2 in place of H w and w^T H w (Eqs. mu-target,
+// w-corr): w^T XX w from the projection by XX, then the projection by K
+// and the combination.
+jarq_status mu_projection(jarq_hessian *h, const float *Wd, int p, const MuTarget &t,
+                          cudaStream_t st) {
+    Workspace &w = h->ws;
+    const int d = h->din;
+    jarq_status rc = project_by(h, t.XX, p, w.Pt_hi, w.Pt_lo, st);
+    if (rc != JARQ_OK) return rc;
+    RUN("whw", 1, launch_whw(Wd, w.Pt_hi, w.Pt_lo, w.aux, p, d, st));
+    rc = project_by(h, t.K, p, w.Pt_hi, w.Pt_lo, st);
+    if (rc != JARQ_OK) return rc;
+    RUN("mu_combine", 1, launch_mu_combine(w.Phi, w.Plo, w.Pt_hi, w.Pt_lo, Wd, w.aux, w.wHw, p, d,
+                                           (double)t.mu, (double)t.nu2, st));
+    return JARQ_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -340,6 +395,9 @@ void jarq_hessian_destroy(jarq_hessian *h) {
     cudaFree(h->Rinv);
     cudaFree(h->Htdig);
     cudaFree(h->expoT);
+    cudaFree(h->qdig);
+    cudaFree(h->qexp);
+    cudaFree(h->qstage);
     cudaFree(h->dstatus);
     cudaFreeHost(h->hstatus);
     (void)cudaGetLastError();
@@ -464,6 +522,27 @@ jarq_status jarq_residual_product(jarq_hessian *h, const float *W, const float *
 jarq_status jarq_refine_layer(jarq_hessian *h, const float *W, float *S, uint8_t *Q,
                               const int32_t *Z, int dout, int bits, const jarq_options *opt,
                               jarq_stats *stats, void *stream) {
+    return refine_impl(h, W, S, Q, Z, dout, bits, opt, stats, stream, nullptr);
+}
+
+jarq_status jarq_refine_layer_mu(jarq_hessian *h, const float *W, float *S, uint8_t *Q,
+                                 const int32_t *Z, int dout, int bits, const float *K,
+                                 const float *XX, float mu, float nu2, const jarq_options *opt,
+                                 jarq_stats *stats, void *stream) {
+    if (!(mu >= 0.f && mu <= 1.f) || !(nu2 >= 0.f) || !isfinite(nu2)) return JARQ_ERR_ARG;
+    if (mu == 1.f) return refine_impl(h, W, S, Q, Z, dout, bits, opt, stats, stream, nullptr);
+    if (!K || !XX) return JARQ_ERR_ARG;
+    MuTarget t{K, XX, mu, nu2};
+    return refine_impl(h, W, S, Q, Z, dout, bits, opt, stats, stream, &t);
+}
+
+}  // extern "C"
+
+namespace {
+
+jarq_status refine_impl(jarq_hessian *h, const float *W, float *S, uint8_t *Q, const int32_t *Z,
+                        int dout, int bits, const jarq_options *opt, jarq_stats *stats,
+                        void *stream, const MuTarget *mt) {
     if (!layer_args_ok(h, W, S, Q, Z, dout, bits)) return JARQ_ERR_ARG;
     jarq_options o = opt ? *opt : jarq_default_options();
     if (o.max_iters < 0 || !(o.ridge >= 0.f) || !(o.rcond >= 0.f) || !(o.eps >= 0.f))
@@ -483,6 +562,13 @@ jarq_status jarq_refine_layer(jarq_hessian *h, const float *W, float *S, uint8_t
     RUN("proj", 1, launch_tc_proj(w.mapWd, h->mapD8, w.Phi, w.Plo, w.wexp, h->expo, p, w.p_pad, d,
                                   h->d_pad, g, h->dstatus, st));
     RUN("whw", 1, launch_whw(la.W, w.Phi, w.Plo, w.wHw, p, d, st));
+    if (mt) {
+        // mu-target: P <- H w_corr and w^T H w <- ||y(mu)||^2 from the two
+        // extra projections W XX and W K^T (Pt's buffers hold them until
+        // the folded projection is formed)
+        rc = mu_projection(h, la.W, p, *mt, st);
+        if (rc != JARQ_OK) return rc;
+    }
     RUN("ptilde", 1, launch_ptilde(w.Phi, w.Plo, h->Rinv, w.Pt_hi, w.Pt_lo, p, d, g, st));
     for (int k = 1; k <= o.max_iters; ++k) {
         RUN("gram", 1, launch_tc_gram(w.mapC, h->mapD10, la.Q, la.Z, h->expo, w.active, w.gram, p,
@@ -529,4 +615,4 @@ jarq_status jarq_refine_layer(jarq_hessian *h, const float *W, float *S, uint8_t
     return status_from_bits(sb);
 }
 
-}  // extern "C"
+}  // namespace

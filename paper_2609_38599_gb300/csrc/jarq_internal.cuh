@@ -82,7 +82,8 @@ struct Workspace {
     float *Plo = nullptr;        // [p][d]
     float *Pt_hi = nullptr;      // [p][d]  folded projection Pt_i = R_i^{-T} P_i
     float *Pt_lo = nullptr;      // [p][d]
-    double *wHw = nullptr;       // [p]  w_j^T H w_j
+    double *wHw = nullptr;       // [p]  w_j^T H w_j (||y_j(mu)||^2 for the mu-target)
+    double *aux = nullptr;       // [p]  w_j^T XX w_j of the mu-target
     double *L_prev = nullptr;    // [p]  L^{(k-1)} of the early stop
     double *L_host = nullptr;    // [p]
     double *L_final = nullptr;   // [p]
@@ -119,6 +120,12 @@ struct jarq_hessian {
     __half *Htdig = nullptr;      // [4][d_pad][d_pad] fp16 digits, |digit| <= 512
     int *expoT = nullptr;         // [G][G] block exponents of Ht
     CUtensorMap mapHt;            // tensor map of Htdig, 64 x 64 boxes
+    // mu-target (allocated on first use): digits of K or XX, base 2^8, six
+    // planes, with a symmetric block-exponent map; staging for host K / XX
+    __nv_bfloat16 *qdig = nullptr;     // [6][d_pad][d_pad]
+    int *qexp = nullptr;               // [G][G]
+    float *qstage = nullptr;           // [d][d]
+    CUtensorMap mapQ;                  // tensor map of qdig, 64 x 64 boxes
     int *dstatus = nullptr;       // device status word
     int *hstatus = nullptr;       // pinned host mirror
     jarq::Workspace ws;
@@ -155,6 +162,11 @@ cudaError_t launch_tc_gram(const CUtensorMap &mapC, const CUtensorMap &mapS, con
                            const int32_t *Z, const int *expo, const int *active, double *gram,
                            int p, int p_pad, int d, int d_pad, int g, int bits, int *status,
                            cudaStream_t s);
+cudaError_t launch_slices8(const float *M, int *expo, __nv_bfloat16 *dig8, int d, int d_pad,
+                           int g, cudaStream_t s);
+cudaError_t launch_mu_combine(float *Phi, float *Plo, const float *Khi, const float *Klo,
+                              const float *W, const double *wXXw, double *wHw, int p, int d,
+                              double mu, double nu2, cudaStream_t s);
 cudaError_t launch_slice_rows(const float *W, __nv_bfloat16 *planes, int *wexp, int p, int d,
                               int d_pad, int p_pad, int g, cudaStream_t s);
 cudaError_t launch_tc_proj(const CUtensorMap &mapW, const CUtensorMap &mapH, float *Phi,

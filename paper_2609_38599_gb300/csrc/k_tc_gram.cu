@@ -302,14 +302,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0 && *abort_flag) atomicOr(a.status, ST_TIMEOUT);
 }
 
-// Per g x g block of the symmetric H: E = the exponent with max |H_blk| <= 2^E.
+// Per g x g block of H: E = the exponent with max |H_blk| <= 2^E.  With
+// `sym` the maximum also runs over the mirrored block (bh, bi), so that the
+// exponent map is symmetric for a matrix that is not (the target projection
+// reads the exponent of block (k, n) for the digits of entry (n, k)).
 __global__ void block_exponent_kernel(const float *__restrict__ Hs, int *__restrict__ expo, int d,
-                                      int g) {
+                                      int g, int sym) {
     const int G = d / g, bi = blockIdx.y, bh = blockIdx.x;
     float mx = 0.f;
     for (int idx = threadIdx.x; idx < g * g; idx += blockDim.x) {
         const int r = idx / g, c = idx % g;
         mx = fmaxf(mx, fabsf(Hs[(size_t)(bi * g + r) * d + bh * g + c]));
+        if (sym) mx = fmaxf(mx, fabsf(Hs[(size_t)(bh * g + r) * d + bi * g + c]));
     }
     for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
     __shared__ float wm[32];
@@ -350,6 +354,7 @@ __global__ void slice_kernel(const float *__restrict__ Hs, const int *__restrict
             dig8[t * plane + off] = __float2bfloat16_rn(dgt);
             x = (x - dgt) * 256.f;
         }
+        if (!dig10) continue;
         x = ldexpf(Hs[idx], 9 - E);
 #pragma unroll
         for (int t = 0; t < 4; ++t) {
@@ -393,7 +398,7 @@ __global__ void slice10_kernel(const float *__restrict__ hi, const float *__rest
 cudaError_t launch_slice10(const float *hi, const float *lo, int *expo, __half *dig, int d,
                            int d_pad, int g, cudaStream_t s) {
     const int G = d / g;
-    block_exponent_kernel<<<dim3(G, G), 256, 0, s>>>(hi, expo, d, g);
+    block_exponent_kernel<<<dim3(G, G), 256, 0, s>>>(hi, expo, d, g, 0);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     size_t n = (size_t)d * d;
@@ -406,13 +411,26 @@ cudaError_t launch_slice10(const float *hi, const float *lo, int *expo, __half *
 cudaError_t launch_slices(const float *Hs, int *expo, __nv_bfloat16 *dig8, __half *dig10, int d,
                           int d_pad, int g, cudaStream_t s) {
     const int G = d / g;
-    block_exponent_kernel<<<dim3(G, G), 256, 0, s>>>(Hs, expo, d, g);
+    block_exponent_kernel<<<dim3(G, G), 256, 0, s>>>(Hs, expo, d, g, 0);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     size_t n = (size_t)d * d;
     int blocks = (int)((n + 255) / 256);
     if (blocks > 16 * num_sms()) blocks = 16 * num_sms();
     slice_kernel<<<blocks, 256, 0, s>>>(Hs, expo, dig8, dig10, d, d_pad, g);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_slices8(const float *M, int *expo, __nv_bfloat16 *dig8, int d, int d_pad,
+                           int g, cudaStream_t s) {
+    const int G = d / g;
+    block_exponent_kernel<<<dim3(G, G), 256, 0, s>>>(M, expo, d, g, 1);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    size_t n = (size_t)d * d;
+    int blocks = (int)((n + 255) / 256);
+    if (blocks > 16 * num_sms()) blocks = 16 * num_sms();
+    slice_kernel<<<blocks, 256, 0, s>>>(M, expo, dig8, nullptr, d, d_pad, g);
     return cudaGetLastError();
 }
 

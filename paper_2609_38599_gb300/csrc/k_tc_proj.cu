@@ -376,6 +376,47 @@ __global__ void whw_kernel(const float *__restrict__ W, const float *__restrict_
     if (lane == 0) out[j] = (double)sh + (double)sl;
 }
 
+// Propagation-corrected target (App. "Propagation-Corrected Targets and
+// QEP", Eqs. mu-target, w-corr).  With H = X~^T X~ + nu^2 I and K = X~^T X,
+// the projection of the corrected weights needs no inverse of H:
+//   H w_corr = A^T y(mu) = mu H w + (1 - mu) (K w + nu^2 w),
+// and the target energy that replaces w^T H w in the objective is
+//   ||y(mu)||^2 = (1-mu)^2 w^T XX w + 2 mu (1-mu) w^T K w
+//                 + mu^2 (w^T H w - nu^2 w^T w) + nu^2 w^T w.
+// On entry P = Phi + Plo holds H w, PK = Khi + Klo holds K w (rows of the
+// target projection with K in place of H), wHw[j] = w^T H w and
+// wXXw[j] = w^T XX w; on exit P holds H w_corr and wHw[j] ||y_j(mu)||^2.
+// One warp per row, float64 arithmetic.
+__global__ void mu_combine_kernel(float *__restrict__ Phi, float *__restrict__ Plo,
+                                  const float *__restrict__ Khi, const float *__restrict__ Klo,
+                                  const float *__restrict__ W, const double *__restrict__ wXXw,
+                                  double *__restrict__ wHw, int p, int d, double mu, double nu2) {
+    const int j = (int)(((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+    const int lane = threadIdx.x & 31;
+    if (j >= p) return;
+    const size_t off = (size_t)j * d;
+    double wKw = 0.0, ww = 0.0;
+    for (int k = lane; k < d; k += 32) {
+        const double P = (double)Phi[off + k] + (double)Plo[off + k];
+        const double PK = (double)Khi[off + k] + (double)Klo[off + k];
+        const double w = W[off + k];
+        const double r = mu * P + (1.0 - mu) * fma(nu2, w, PK);
+        const float hi = __double2float_rn(r);
+        Phi[off + k] = hi;
+        Plo[off + k] = __double2float_rn(r - (double)hi);
+        wKw = fma(w, PK, wKw);
+        ww = fma(w, w, ww);
+    }
+    for (int o = 16; o; o >>= 1) {
+        wKw += __shfl_xor_sync(0xffffffffu, wKw, o);
+        ww += __shfl_xor_sync(0xffffffffu, ww, o);
+    }
+    if (lane == 0) {
+        const double a = 1.0 - mu;
+        wHw[j] = a * a * wXXw[j] + 2.0 * mu * a * wKw + mu * mu * (wHw[j] - nu2 * ww) + nu2 * ww;
+    }
+}
+
 // Folded target projection Pt_j[grp i] = R_i^{-T} P_j[grp i], i.e.
 // Pt[j, i g + a] = sum_{b <= a} Rinv_i[b][a] P[j, i g + b], in double-float
 // from the float64 inverse and the double-float P.  One CTA per (64 rows,
@@ -487,6 +528,14 @@ cudaError_t launch_tc_proj(const CUtensorMap &mapW, const CUtensorMap &mapH, flo
 cudaError_t launch_whw(const float *W, const float *Phi, const float *Plo, double *out, int p,
                        int d, cudaStream_t s) {
     whw_kernel<<<(unsigned)(((long long)p * 32 + 255) / 256), 256, 0, s>>>(W, Phi, Plo, out, p, d);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_mu_combine(float *Phi, float *Plo, const float *Khi, const float *Klo,
+                              const float *W, const double *wXXw, double *wHw, int p, int d,
+                              double mu, double nu2, cudaStream_t s) {
+    mu_combine_kernel<<<(unsigned)(((long long)p * 32 + 255) / 256), 256, 0, s>>>(
+        Phi, Plo, Khi, Klo, W, wXXw, wHw, p, d, mu, nu2);
     return cudaGetLastError();
 }
 

@@ -11,7 +11,7 @@ namespace {
 const char *const kNames[] = {"validate", "residual", "init_rows", "hr_full", "grad", "gram",
                               "scale_solve", "phase_hr", "babai", "symmetrize", "group_factor",
                               "slices", "slice_rows", "proj", "whw", "rhs", "htilde", "ptilde",
-                              "target", "syrk"};
+                              "target", "syrk", "mu_combine"};
 constexpr int kNumNames = sizeof(kNames) / sizeof(kNames[0]);
 
 struct Pending {

@@ -31,7 +31,8 @@ EXPORTS = ("jarq_default_options", "jarq_prepare_hessian", "jarq_refine_layer",
            "jarq_hessian_destroy", "jarq_status_string", "jarq_profile_enable",
            "jarq_profile_reset", "jarq_profile_read", "jarq_launch_count",
            "jarq_objective_noalloc", "jarq_residual_product", "jarq_canonicalize",
-           "jarq_dequantize", "jarq_pack_codes", "jarq_accumulate_hessian")
+           "jarq_dequantize", "jarq_pack_codes", "jarq_accumulate_hessian",
+           "jarq_refine_layer_mu")
 
 
 class JarqError(RuntimeError):
@@ -66,6 +67,9 @@ def _load():
     lib.jarq_refine_layer.restype = ci
     lib.jarq_refine_layer.argtypes = [vp, vp, vp, vp, vp, ci, ci, ctypes.POINTER(Options),
                                       ctypes.POINTER(Stats), vp]
+    lib.jarq_refine_layer_mu.restype = ci
+    lib.jarq_refine_layer_mu.argtypes = [vp, vp, vp, vp, vp, ci, ci, vp, vp, cf, cf,
+                                         ctypes.POINTER(Options), ctypes.POINTER(Stats), vp]
     lib.jarq_objective.restype = ci
     lib.jarq_objective.argtypes = [vp, vp, vp, vp, vp, ci, ci, vp, vp]
     lib.jarq_objective_noalloc.restype = ci
@@ -110,7 +114,7 @@ def library():
 
 KERNELS = ("validate", "residual", "init_rows", "hr_full", "grad", "gram", "scale_solve",
            "phase_hr", "babai", "symmetrize", "group_factor", "slices", "slice_rows", "proj",
-           "whw", "rhs", "htilde", "ptilde", "target", "syrk")
+           "whw", "rhs", "htilde", "ptilde", "target", "syrk", "mu_combine")
 
 
 def profile_enable(on: bool = True):
@@ -254,6 +258,36 @@ def refine(hess: Hessian, W, S, Q, Z, bits: int, options: Options = None,
         st.status = status
     if raise_on_error and status not in (JARQ_OK,):
         raise JarqError(status, "jarq_refine_layer")
+    return st if st is not None else status
+
+
+def refine_mu(hess: Hessian, W, S, Q, Z, bits: int, K, XX, mu: float, nu2: float,
+              options: Options = None, collect_stats: bool = True, raise_on_error: bool = True,
+              **opt):
+    """``jarq_refine_layer_mu``: refinement on the propagation-corrected target
+    (K = X~^T X, XX = X^T X, normalised like the prepared H = X~^T X~ + nu2 I);
+    S and Q in place; returns RefineStats with the mu-objective."""
+    o = options if options is not None else default_options(**opt)
+    dout = int(W.shape[0])
+    st = None
+    stats = None
+    if collect_stats:
+        st = RefineStats(*(_alloc_like(W, dout, t) for t in
+                           (np.float64, np.float64, np.int32, np.int32, np.int32, np.int32)),
+                         status=0)
+        stats = Stats(*(_ptr(x, t) for x, t in zip(
+            (st.L_host, st.L_final, st.iters, st.accepted, st.ridge_hits, st.row_status),
+            (np.float64, np.float64, np.int32, np.int32, np.int32, np.int32))))
+    status = _lib.jarq_refine_layer_mu(hess.handle, _ptr(W, np.float32), _ptr(S, np.float32),
+                                       _ptr(Q, np.uint8), _ptr(Z, np.int32), dout, int(bits),
+                                       _ptr(K, np.float32), _ptr(XX, np.float32), float(mu),
+                                       float(nu2), ctypes.byref(o),
+                                       ctypes.byref(stats) if stats else None,
+                                       _stream(W, S, Q, Z))
+    if st is not None:
+        st.status = status
+    if raise_on_error and status not in (JARQ_OK,):
+        raise JarqError(status, "jarq_refine_layer_mu")
     return st if st is not None else status
 
 

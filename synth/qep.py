@@ -77,3 +77,63 @@ def mu_layer(din, dout, g, bits, K_iters=3, tokens=None, drift=0.05, damp=0.01, 
     S0, Q0, Z = rtn_host_np(W, bits, g)
     return MuLayer(f"mu_{dout}x{din}_g{g}_w{bits}_s{seed}", W, H, K, XX, nu2, S0, Q0, Z, bits,
                    g, K_iters, Xq if keep_activations else None, Xf if keep_activations else None)
+
+
+def mu_grams_torch(din, tokens, rank, n_out, out_scale, D_lo, seed, device, drift=0.05,
+                   damp=0.01, chunk=8192):
+    """Full-size (H, K, XX, nu2) on ``device``: X~ drawn chunk by chunk with the
+    activation recipe and X = X~ + drift (a rank-4 channel mix of X~ plus
+    noise, scaled per channel), both rounded to float16; each chunk's
+    products formed in float32 (no TF32) and summed in float64; normalised
+    by the token count; returned as float32 matrices."""
+    import math
+
+    import torch
+    gen = torch.Generator(device=device)
+    gen.manual_seed(seed)
+    L = torch.randn(din, rank, generator=gen, device=device) * (2.0 / math.sqrt(rank))
+    D = torch.rand(din, generator=gen, device=device) * (1.0 - D_lo) + D_lo
+    col = torch.ones(din, device=device)
+    if n_out:
+        idx = torch.randperm(din, generator=gen, device=device)[:n_out]
+        col[idx] = out_scale
+    sd = torch.sqrt((L * L).sum(1) + D) * col          # per-channel spread of X~
+    M = (torch.randn(din, 4, generator=gen, device=device)
+         @ torch.randn(4, din, generator=gen, device=device)) / (2.0 * math.sqrt(din))
+    sqD = D.sqrt()
+    H0 = torch.zeros(din, din, dtype=torch.float64, device=device)
+    K = torch.zeros_like(H0)
+    XX = torch.zeros_like(H0)
+    prev = torch.get_float32_matmul_precision()
+    torch.set_float32_matmul_precision("highest")
+    try:
+        done = 0
+        while done < tokens:
+            m = min(chunk, tokens - done)
+            U = torch.randn(m, rank, generator=gen, device=device)
+            E = torch.randn(m, din, generator=gen, device=device)
+            Xq = ((U @ L.T + E * sqD) * col).half().float()
+            N = torch.randn(m, din, generator=gen, device=device)
+            Xf = (Xq + drift * ((Xq / sd) @ M + 0.5 * N) * sd).half().float()
+            H0 += (Xq.T @ Xq).double()
+            K += (Xq.T @ Xf).double()
+            XX += (Xf.T @ Xf).double()
+            done += m
+    finally:
+        torch.set_float32_matmul_precision(prev)
+    H0 /= tokens
+    K /= tokens
+    XX /= tokens
+    nu2 = float(torch.tensor(damp * H0.diagonal().mean().item()).float())
+    H = H0 + nu2 * torch.eye(din, dtype=torch.float64, device=device)
+    return H.float(), K.float(), XX.float(), nu2
+
+
+def mu_config_layer(name, device="cuda", drift=0.05):
+    """A named full-size layer of ``layers.CONFIGS`` with mu-target inputs:
+    (Layer, K, XX, nu2); the Layer's H is X~^T X~ / n + nu2 I."""
+    from .layers import CONFIGS, config_layer
+    c = CONFIGS[name]
+    H, K, XX, nu2 = mu_grams_torch(c["din"], c["tokens"], c["rank"], c["n_out"], c["out_scale"],
+                                   c["D_lo"], 500 + c["seed"], device, drift=drift)
+    return config_layer(name, device=device, H=H), K, XX, nu2
