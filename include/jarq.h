@@ -77,7 +77,17 @@ typedef struct jarq_options {
     int   ridge_accept;  /* 1: keep a ridge-stabilised solve only if it does not raise F_j,
                             else keep the previous scales (App. G Remark ridge-acceptance);
                             0 (default): keep every solve, as the paper's runs do */
+    int   fixed_grid;    /* 1: keep the host scales, update only the codes -- the "Fixed"
+                            arm of App. "Fixed-Grid versus Joint Refinement"; each iteration
+                            still evaluates L^(k) for the early stop.  0 (default): JARQ */
 } jarq_options;
+
+/* Scale fits of jarq_fit_scales (App. "Joint Scale Fitting"). */
+typedef enum jarq_fit {
+    JARQ_FIT_JOINT = 0,        /* the joint normal equations (Eq. scale_normal_equations) */
+    JARQ_FIT_INDEPENDENT = 1,  /* each group on its own contribution (Eq. independent-fit) */
+    JARQ_FIT_COORDINATE = 2    /* cyclic exact coordinate descent on the scales */
+} jarq_fit;
 
 /* Element types of jarq_dequantize's output. */
 typedef enum jarq_dtype { JARQ_F32 = 0, JARQ_F16 = 1, JARQ_BF16 = 2 } jarq_dtype;
@@ -183,6 +193,43 @@ jarq_status jarq_residual_product(jarq_hessian *h, const float *W, const float *
                                   const uint8_t *Q, const int32_t *Z, int dout, int bits,
                                   float *HR, void *stream);
 
+/* ---- mechanism ablations (App. "Refinement Mechanisms", Tab. mechanism-summary (a)) ----
+ * Same layouts, staging and code checks as jarq_refine_layer. */
+
+/* Fit all scales of every row for the given codes with one of the three fits
+ * that the paper compares (App. "Joint Scale Fitting"):
+ *   JARQ_FIT_JOINT        the joint least-squares fit (Sec. 3.3.1), with the
+ *                         ridge safeguard of App. E;
+ *   JARQ_FIT_INDEPENDENT  s_i = c_i^T H_ii w_i / c_i^T H_ii c_i, each group on
+ *                         its own contribution (Eq. independent-fit);
+ *   JARQ_FIT_COORDINATE   `passes` cyclic passes over the groups, each scale
+ *                         moved to the exact minimiser of F along it, starting
+ *                         from the input S.
+ * A group whose codes all equal its zero point keeps its scale in the last
+ * two.  S is overwritten with the fitted float32 scales; F_before / F_after
+ * (optional, [dout] double, host or device) receive the objective of the
+ * input and of the fitted scales.  passes >= 1 for JARQ_FIT_COORDINATE. */
+jarq_status jarq_fit_scales(jarq_hessian *h, const float *W, float *S, const uint8_t *Q,
+                            const int32_t *Z, int dout, int bits, jarq_fit method, int passes,
+                            double *F_before, double *F_after, void *stream);
+
+/* Multi-code probe of one group (App. "Multi-Code Updates"): for every row,
+ * with the scales and the other groups fixed, single-code updates of group
+ * `group` (each coordinate in order moved to its best code when that
+ * strictly lowers F; full passes until a pass moves nothing), then one
+ * bounded Babai proposal from that single-code-stationary state (Eq.
+ * babai_update), accepted iff it strictly lowers F.  Decisions are taken in
+ * float64.  Nothing is written back to S or Q.  Outputs (optional, host or
+ * device): Q_search [dout][g] uint8, the codes after the search; moves
+ * [dout], the single-code moves made; accepted [dout], 1 if the Babai
+ * proposal strictly lowers F; changed [dout], codes the proposal changes;
+ * dF [dout] double, its change of F.  Rows with |s| <= FLT_EPSILON are
+ * skipped (all outputs 0, codes unchanged). */
+jarq_status jarq_multicode_probe(jarq_hessian *h, const float *W, const float *S,
+                                 const uint8_t *Q, const int32_t *Z, int dout, int bits,
+                                 int group, uint8_t *Q_search, int32_t *moves, int32_t *accepted,
+                                 int32_t *changed, double *dF, void *stream);
+
 /* ---- write-back of a refined layer (device memory only) ----
  * These post-passes act on a layer already in device memory; host pointers
  * return JARQ_ERR_ARG.  They allocate nothing and return after their work
@@ -279,7 +326,8 @@ const char *jarq_status_string(jarq_status s);
  * enclosing call synchronises.  Names: "validate", "residual", "init_rows",
  * "hr_full", "grad", "gram", "scale_solve", "phase_hr", "babai",
  * "symmetrize", "group_factor", "slices", "slice_rows", "proj", "whw", "rhs",
- * "htilde", "ptilde", "target", "syrk", "mu_combine".  Not thread-safe. */
+ * "htilde", "ptilde", "target", "syrk", "mu_combine", "own_rhs", "scale_fit",
+ * "probe".  Not thread-safe. */
 void jarq_profile_enable(int on);
 void jarq_profile_reset(void);
 /* Accumulated launches and total device milliseconds of one kernel name since

@@ -127,6 +127,7 @@ void free_ws(Workspace &w) {
     cudaFree(w.Plo);
     cudaFree(w.wHw);
     cudaFree(w.aux);
+    cudaFree(w.own);
     cudaFree(w.L_prev);
     cudaFree(w.L_host);
     cudaFree(w.L_final);
@@ -177,6 +178,7 @@ cudaError_t ensure_ws(jarq_hessian *h, int p) {
     if ((e = dalloc(&w.Plo, (size_t)p * d)) != cudaSuccess) return e;
     if ((e = dalloc(&w.wHw, (size_t)p)) != cudaSuccess) return e;
     if ((e = dalloc(&w.aux, (size_t)p)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.own, (size_t)p * G)) != cudaSuccess) return e;
     if ((e = dalloc(&w.L_prev, (size_t)p)) != cudaSuccess) return e;
     if ((e = dalloc(&w.L_host, (size_t)p)) != cudaSuccess) return e;
     if ((e = dalloc(&w.L_final, (size_t)p)) != cudaSuccess) return e;
@@ -362,6 +364,7 @@ jarq_options jarq_default_options(void) {
     o.rcond = 1e-10f;
     o.eps = FLT_EPSILON;
     o.ridge_accept = 0;
+    o.fixed_grid = 0;
     return o;
 }
 
@@ -392,6 +395,7 @@ void jarq_hessian_destroy(jarq_hessian *h) {
     cudaFree(h->Hdig10);
     cudaFree(h->expo);
     cudaFree(h->Lf);
+    cudaFree(h->L64);
     cudaFree(h->Rinv);
     cudaFree(h->Htdig);
     cudaFree(h->expoT);
@@ -436,6 +440,7 @@ jarq_status jarq_prepare_hessian(const float *H, int din, int group_size, float 
         if ((e = make_tmap_bf16(&h->mapD8, h->Hdig8, (uint64_t)6 * h->d_pad, h->d_pad, 64)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = make_tmap_f16(&h->mapD10, h->Hdig10, (uint64_t)4 * h->d_pad, h->d_pad, 64)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->Lf, (size_t)h->G * group_size * group_size)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = dalloc(&h->L64, (size_t)h->G * group_size * group_size)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->Rinv, (size_t)h->G * group_size * group_size)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->Htdig, 4 * pd)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = cudaMemsetAsync(h->Htdig, 0, 4 * pd * 2, st)) != cudaSuccess) { rc = cuda_fail(e); break; }
@@ -452,7 +457,7 @@ jarq_status jarq_prepare_hessian(const float *H, int din, int group_size, float 
         if ((e = cudaMemsetAsync(h->dstatus, 0, sizeof(int), st)) != cudaSuccess) { rc = cuda_fail(e); break; }
         { ProfScope ps("symmetrize", st); e = launch_symmetrize(Hsrc, h->Hs, h->Hplanes, din, h->d_pad, nu2, st); ps.done(); count_launches(1); }
         if (e != cudaSuccess) { rc = cuda_fail(e); break; }
-        { ProfScope ps("group_factor", st); e = launch_group_factor(h->Hs, h->Lf, h->Rinv, din, group_size, h->dstatus, st); ps.done(); count_launches(1); }
+        { ProfScope ps("group_factor", st); e = launch_group_factor(h->Hs, h->Lf, h->L64, h->Rinv, din, group_size, h->dstatus, st); ps.done(); count_launches(1); }
         if (e != cudaSuccess) { rc = cuda_fail(e); break; }
         // folded rows R_i^{-T} H[grp i, :] (double-float, temporary) -> digits
         if ((e = dalloc(&Ht_hi, dd)) != cudaSuccess) { rc = cuda_fail(e); break; }
@@ -523,6 +528,83 @@ jarq_status jarq_refine_layer(jarq_hessian *h, const float *W, float *S, uint8_t
                               const int32_t *Z, int dout, int bits, const jarq_options *opt,
                               jarq_stats *stats, void *stream) {
     return refine_impl(h, W, S, Q, Z, dout, bits, opt, stats, stream, nullptr);
+}
+
+jarq_status jarq_fit_scales(jarq_hessian *h, const float *W, float *S, const uint8_t *Q,
+                            const int32_t *Z, int dout, int bits, jarq_fit method, int passes,
+                            double *F_before, double *F_after, void *stream) {
+    if (!layer_args_ok(h, W, S, Q, Z, dout, bits)) return JARQ_ERR_ARG;
+    if (method != JARQ_FIT_JOINT && method != JARQ_FIT_INDEPENDENT &&
+        method != JARQ_FIT_COORDINATE)
+        return JARQ_ERR_ARG;
+    if (method == JARQ_FIT_COORDINATE && passes < 1) return JARQ_ERR_ARG;
+    if (dout == 0) return JARQ_OK;
+    cudaStream_t st = (cudaStream_t)stream;
+    LayerArgs la;
+    jarq_status rc = layer_front(h, W, S, Q, Z, dout, bits, la, st, true);
+    if (rc != JARQ_OK) return rc;
+    Workspace &w = h->ws;
+    const int p = dout, d = h->din, g = h->g, G = h->G;
+    RUN("init_rows", 1, launch_init_rows(w.active, w.iters, w.accepted, w.ridge, w.rstat, p, st));
+    RUN("slice_rows", 1, launch_slice_rows(la.W, w.wdig, w.wexp, p, d, h->d_pad, w.p_pad, g, st));
+    RUN("proj", 1, launch_tc_proj(w.mapWd, h->mapD8, w.Phi, w.Plo, w.wexp, h->expo, p, w.p_pad, d,
+                                  h->d_pad, g, h->dstatus, st));
+    RUN("whw", 1, launch_whw(la.W, w.Phi, w.Plo, w.wHw, p, d, st));
+    RUN("gram", 1, launch_tc_gram(w.mapC, h->mapD10, la.Q, la.Z, h->expo, nullptr, w.gram, p,
+                                  w.p_pad, d, h->d_pad, g, bits, h->dstatus, st));
+    RUN("rhs", 1, launch_rhs(la.Q, la.Z, w.Phi, w.Plo, nullptr, w.rhs, p, d, g, st));
+    if (method == JARQ_FIT_JOINT) {
+        jarq_options o = jarq_default_options();
+        o.early_stop = 0;
+        RUN("scale_solve", 1, launch_scale_solve(w.gram, w.rhs, w.wHw, la.S, w.L_prev, w.L_host,
+                                                 w.active, w.iters, w.ridge, w.rstat, h->dstatus,
+                                                 p, d, g, 1, false, o, st));
+        CK(cudaMemcpyAsync(w.L_final, w.L_prev, p * sizeof(double), cudaMemcpyDeviceToDevice, st));
+    } else {
+        if (method == JARQ_FIT_INDEPENDENT)
+            RUN("own_rhs", 1, launch_own_rhs(h->Hs, la.W, la.Q, la.Z, w.own, p, d, g, st));
+        RUN("scale_fit", 1, launch_scale_fit(w.gram, w.rhs, w.own, w.wHw, la.S, w.L_host,
+                                             w.L_final, p, G, (int)method, passes, st));
+    }
+    if (la.hS) CK(cudaMemcpyAsync(S, la.S, (size_t)p * G * sizeof(float), cudaMemcpyDeviceToHost, st));
+    if (F_before) CK(cudaMemcpyAsync(F_before, w.L_host, p * sizeof(double), cudaMemcpyDefault, st));
+    if (F_after) CK(cudaMemcpyAsync(F_after, w.L_final, p * sizeof(double), cudaMemcpyDefault, st));
+    int sb = 0;
+    CK(read_status(h, st, &sb));
+    return status_from_bits(sb);
+}
+
+jarq_status jarq_multicode_probe(jarq_hessian *h, const float *W, const float *S,
+                                 const uint8_t *Q, const int32_t *Z, int dout, int bits,
+                                 int group, uint8_t *Q_search, int32_t *moves, int32_t *accepted,
+                                 int32_t *changed, double *dF, void *stream) {
+    if (!layer_args_ok(h, W, S, Q, Z, dout, bits) || group < 0 || group >= h->G) return JARQ_ERR_ARG;
+    if (dout == 0) return JARQ_OK;
+    cudaStream_t st = (cudaStream_t)stream;
+    LayerArgs la;
+    jarq_status rc = layer_front(h, W, S, Q, Z, dout, bits, la, st, true);
+    if (rc != JARQ_OK) return rc;
+    Workspace &w = h->ws;
+    const int p = dout, d = h->din, g = h->g, G = h->G;
+    const int nsplit = target_splits(w.p_pad, g, G);
+    RUN("slice_rows", 1, launch_slice_rows(la.W, w.wdig, w.wexp, p, d, h->d_pad, w.p_pad, g, st));
+    RUN("proj", 1, launch_tc_proj(w.mapWd, h->mapD8, w.Phi, w.Plo, w.wexp, h->expo, p, w.p_pad, d,
+                                  h->d_pad, g, h->dstatus, st));
+    // T = sum_h s_h H_ih c_h: the phase product with H's own digits
+    RUN("target", 1, launch_tc_target(w.mapC, h->mapD10, w.t_hi, w.t_lo, la.S, h->expo, nullptr, p,
+                                      w.p_pad, h->d_pad, g, G, group, nsplit, h->dstatus, st));
+    uint8_t *qo = reinterpret_cast<uint8_t *>(w.Hr);
+    RUN("probe", 1, launch_probe(w.Phi, w.Plo, w.t_hi, w.t_lo, h->Hs, h->L64, la.S, la.Q, la.Z, qo,
+                                 w.iters, w.accepted, w.ridge, w.L_final, p, w.p_pad, d, g, group,
+                                 nsplit, (1 << bits) - 1, FLT_EPSILON, st));
+    if (Q_search) CK(cudaMemcpyAsync(Q_search, qo, (size_t)p * g, cudaMemcpyDefault, st));
+    if (moves) CK(cudaMemcpyAsync(moves, w.iters, p * sizeof(int32_t), cudaMemcpyDefault, st));
+    if (accepted) CK(cudaMemcpyAsync(accepted, w.accepted, p * sizeof(int32_t), cudaMemcpyDefault, st));
+    if (changed) CK(cudaMemcpyAsync(changed, w.ridge, p * sizeof(int32_t), cudaMemcpyDefault, st));
+    if (dF) CK(cudaMemcpyAsync(dF, w.L_final, p * sizeof(double), cudaMemcpyDefault, st));
+    int sb = 0;
+    CK(read_status(h, st, &sb));
+    return status_from_bits(sb);
 }
 
 jarq_status jarq_refine_layer_mu(jarq_hessian *h, const float *W, float *S, uint8_t *Q,

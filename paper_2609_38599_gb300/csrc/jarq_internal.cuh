@@ -84,6 +84,7 @@ struct Workspace {
     float *Pt_lo = nullptr;      // [p][d]
     double *wHw = nullptr;       // [p]  w_j^T H w_j (||y_j(mu)||^2 for the mu-target)
     double *aux = nullptr;       // [p]  w_j^T XX w_j of the mu-target
+    double *own = nullptr;       // [p][G]  c_i^T H_ii w_i (independent scale fit)
     double *L_prev = nullptr;    // [p]  L^{(k-1)} of the early stop
     double *L_host = nullptr;    // [p]
     double *L_final = nullptr;   // [p]
@@ -115,6 +116,7 @@ struct jarq_hessian {
     CUtensorMap mapH128, mapH64;  // tensor maps of Hplanes, 128 x 64 and 64 x 64 boxes
     CUtensorMap mapD8, mapD10;    // tensor maps of Hdig8 / Hdig10, 64 x 64 boxes
     float *Lf = nullptr;          // [G][g][g] lower factor L_i = R_i^T, row-major
+    double *L64 = nullptr;        // [G][g][g] the same in float64
     double *Rinv = nullptr;       // [G][g][g] R_i^{-1} (upper), row-major, float64
     // folded rows Ht[grp i, :] = R_i^{-T} H[grp i, :] in the base-2^10 digit scheme
     __half *Htdig = nullptr;      // [4][d_pad][d_pad] fp16 digits, |digit| <= 512
@@ -136,8 +138,18 @@ namespace jarq {
 // ---- launchers (each returns the cudaError_t of its launch) ----
 cudaError_t launch_symmetrize(const float *H, float *Hs, __nv_bfloat16 *Hplanes, int d, int d_pad,
                               float nu2, cudaStream_t s);
-cudaError_t launch_group_factor(const float *Hs, float *Lf, double *Rinv, int d, int g,
-                                int *status, cudaStream_t s);
+cudaError_t launch_group_factor(const float *Hs, float *Lf, double *L64, double *Rinv, int d,
+                                int g, int *status, cudaStream_t s);
+cudaError_t launch_own_rhs(const float *Hs, const float *W, const uint8_t *Q, const int32_t *Z,
+                           double *own, int p, int d, int g, cudaStream_t s);
+cudaError_t launch_scale_fit(const double *gram, const double *rhs, const double *own,
+                             const double *wHw, float *S, double *F_before, double *F_after, int p,
+                             int G, int method, int passes, cudaStream_t s);
+cudaError_t launch_probe(const float *Phi, const float *Plo, const float *t_hi, const float *t_lo,
+                         const float *Hs, const double *L64, const float *S, const uint8_t *Q,
+                         const int32_t *Z, uint8_t *q_out, int32_t *moves, int32_t *accepted,
+                         int32_t *changed, double *dF, int p, int p_pad, int d, int g, int i,
+                         int nsplit, int qmax, float eps, cudaStream_t s);
 cudaError_t launch_htilde(const float *Hs, const double *Rinv, float *out_hi, float *out_lo,
                           int d, int g, cudaStream_t s);
 cudaError_t launch_slice10(const float *hi, const float *lo, int *expo, __half *dig, int d,

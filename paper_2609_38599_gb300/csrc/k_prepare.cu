@@ -53,7 +53,8 @@ __global__ void symmetrize_kernel(const float *__restrict__ H, float *__restrict
 // One block per group: float64 Cholesky of H_ii in shared memory, then an
 // in-place inverse of the lower factor.
 __global__ void group_factor_kernel(const float *__restrict__ Hs, float *__restrict__ Lf,
-                                    double *__restrict__ Rinv, int d, int g, int *status) {
+                                    double *__restrict__ L64, double *__restrict__ Rinv, int d,
+                                    int g, int *status) {
     extern __shared__ double smem[];
     const int ld = g + 1;
     double *A = smem;               // [g][g+1]
@@ -95,9 +96,11 @@ __global__ void group_factor_kernel(const float *__restrict__ Hs, float *__restr
         return;
     }
     float *Lo = Lf + (size_t)grp * g * g;
+    double *Ld = L64 + (size_t)grp * g * g;
     for (int idx = tid; idx < g * g; idx += nt) {
         int a = idx / g, b = idx % g;
         Lo[idx] = (b <= a) ? (float)A[a * ld + b] : 0.f;
+        Ld[idx] = (b <= a) ? A[a * ld + b] : 0.0;
     }
     __syncthreads();
     // in-place inverse of the lower factor, columns from last to first:
@@ -191,13 +194,13 @@ cudaError_t launch_symmetrize(const float *H, float *Hs, __nv_bfloat16 *Hplanes,
     return cudaGetLastError();
 }
 
-cudaError_t launch_group_factor(const float *Hs, float *Lf, double *Rinv, int d, int g,
-                                int *status, cudaStream_t s) {
+cudaError_t launch_group_factor(const float *Hs, float *Lf, double *L64, double *Rinv, int d,
+                                int g, int *status, cudaStream_t s) {
     size_t smem = (size_t)(g * (g + 1) + g) * sizeof(double);
     cudaError_t e = cudaFuncSetAttribute(group_factor_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    group_factor_kernel<<<d / g, 256, smem, s>>>(Hs, Lf, Rinv, d, g, status);
+    group_factor_kernel<<<d / g, 256, smem, s>>>(Hs, Lf, L64, Rinv, d, g, status);
     return cudaGetLastError();
 }
 

@@ -134,6 +134,21 @@ __global__ void scale_solve_kernel(SolveArgs a) {
     const double F_old = a.wHw[j] - warp_sum(fs);
     if (a.L_out && lane == 0) a.L_out[j] = F_old;
     if (a.eval_only) return;
+    if (a.o.fixed_grid) {
+        // fixed grid: the scales stay; L^(k) is the objective of the current state
+        bool stop = false;
+        if (a.o.early_stop && a.k >= 2) {
+            const double dec = a.L_prev[j] - F_old;
+            const double den = fmax(fabs(a.L_prev[j]), (double)a.o.eps);
+            stop = (dec / den <= (double)a.o.tau_rel) || (fabs(dec) <= (double)a.o.tau_abs);
+        }
+        if (lane == 0) {
+            a.L_prev[j] = F_old;
+            a.iters[j] = a.k;
+            if (stop) a.active[j] = 0;
+        }
+        return;
+    }
     auto load_sym = [&](float shift) -> bool {
         bool finite = true;
         for (int idx = lane; idx < G * G; idx += 32) {

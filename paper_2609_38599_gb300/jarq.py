@@ -32,7 +32,7 @@ EXPORTS = ("jarq_default_options", "jarq_prepare_hessian", "jarq_refine_layer",
            "jarq_profile_reset", "jarq_profile_read", "jarq_launch_count",
            "jarq_objective_noalloc", "jarq_residual_product", "jarq_canonicalize",
            "jarq_dequantize", "jarq_pack_codes", "jarq_accumulate_hessian",
-           "jarq_refine_layer_mu")
+           "jarq_refine_layer_mu", "jarq_fit_scales", "jarq_multicode_probe")
 
 
 class JarqError(RuntimeError):
@@ -45,7 +45,8 @@ class Options(ctypes.Structure):
     _fields_ = [("max_iters", ctypes.c_int), ("early_stop", ctypes.c_int),
                 ("tau_rel", ctypes.c_float), ("tau_abs", ctypes.c_float),
                 ("ridge", ctypes.c_float), ("rcond", ctypes.c_float),
-                ("eps", ctypes.c_float), ("ridge_accept", ctypes.c_int)]
+                ("eps", ctypes.c_float), ("ridge_accept", ctypes.c_int),
+                ("fixed_grid", ctypes.c_int)]
 
 
 class Stats(ctypes.Structure):
@@ -70,6 +71,10 @@ def _load():
     lib.jarq_refine_layer_mu.restype = ci
     lib.jarq_refine_layer_mu.argtypes = [vp, vp, vp, vp, vp, ci, ci, vp, vp, cf, cf,
                                          ctypes.POINTER(Options), ctypes.POINTER(Stats), vp]
+    lib.jarq_fit_scales.restype = ci
+    lib.jarq_fit_scales.argtypes = [vp, vp, vp, vp, vp, ci, ci, ci, ci, vp, vp, vp]
+    lib.jarq_multicode_probe.restype = ci
+    lib.jarq_multicode_probe.argtypes = [vp, vp, vp, vp, vp, ci, ci, ci, vp, vp, vp, vp, vp, vp]
     lib.jarq_objective.restype = ci
     lib.jarq_objective.argtypes = [vp, vp, vp, vp, vp, ci, ci, vp, vp]
     lib.jarq_objective_noalloc.restype = ci
@@ -114,7 +119,7 @@ def library():
 
 KERNELS = ("validate", "residual", "init_rows", "hr_full", "grad", "gram", "scale_solve",
            "phase_hr", "babai", "symmetrize", "group_factor", "slices", "slice_rows", "proj",
-           "whw", "rhs", "htilde", "ptilde", "target", "syrk", "mu_combine")
+           "whw", "rhs", "htilde", "ptilde", "target", "syrk", "mu_combine", "own_rhs", "scale_fit", "probe")
 
 
 def profile_enable(on: bool = True):
@@ -289,6 +294,48 @@ def refine_mu(hess: Hessian, W, S, Q, Z, bits: int, K, XX, mu: float, nu2: float
     if raise_on_error and status not in (JARQ_OK,):
         raise JarqError(status, "jarq_refine_layer_mu")
     return st if st is not None else status
+
+
+JARQ_FIT_JOINT, JARQ_FIT_INDEPENDENT, JARQ_FIT_COORDINATE = 0, 1, 2
+
+
+def fit_scales(hess: Hessian, W, S, Q, Z, bits: int, method: str = "joint", passes: int = 3):
+    """``jarq_fit_scales``: refit S in place for the codes Q with the joint,
+    independent or coordinate-descent fit; returns (F_before, F_after)."""
+    code = {"joint": JARQ_FIT_JOINT, "independent": JARQ_FIT_INDEPENDENT,
+            "coordinate": JARQ_FIT_COORDINATE}[method]
+    dout = int(W.shape[0])
+    Fb, Fa = _alloc_like(W, dout, np.float64), _alloc_like(W, dout, np.float64)
+    status = _lib.jarq_fit_scales(hess.handle, _ptr(W, np.float32), _ptr(S, np.float32),
+                                  _ptr(Q, np.uint8), _ptr(Z, np.int32), dout, int(bits), code,
+                                  int(passes), _ptr(Fb, np.float64), _ptr(Fa, np.float64),
+                                  _stream(W, S, Q, Z))
+    if status != JARQ_OK:
+        raise JarqError(status, "jarq_fit_scales")
+    return Fb, Fa
+
+
+def multicode_probe(hess: Hessian, W, S, Q, Z, bits: int, group: int):
+    """``jarq_multicode_probe``: dict of q_search [dout][g] (uint8), moves,
+    accepted, changed (int32) and dF (float64) for one group of every row."""
+    dout = int(W.shape[0])
+    g = hess.group_size
+    if _is_torch(W):
+        import torch
+        qs = torch.empty(dout, g, dtype=torch.uint8, device=W.device)
+    else:
+        qs = np.empty((dout, g), dtype=np.uint8)
+    out = {"q_search": qs, "moves": _alloc_like(W, dout, np.int32),
+           "accepted": _alloc_like(W, dout, np.int32), "changed": _alloc_like(W, dout, np.int32),
+           "dF": _alloc_like(W, dout, np.float64)}
+    status = _lib.jarq_multicode_probe(
+        hess.handle, _ptr(W, np.float32), _ptr(S, np.float32), _ptr(Q, np.uint8),
+        _ptr(Z, np.int32), dout, int(bits), int(group), _ptr(qs, np.uint8),
+        _ptr(out["moves"], np.int32), _ptr(out["accepted"], np.int32),
+        _ptr(out["changed"], np.int32), _ptr(out["dF"], np.float64), _stream(W, S, Q, Z))
+    if status != JARQ_OK:
+        raise JarqError(status, "jarq_multicode_probe")
+    return out
 
 
 def residual_product(hess: Hessian, W, S, Q, Z, bits: int, out=None):

@@ -1,0 +1,103 @@
+"""Mechanism ablations through the C ABI against the oracle (App.
+"Refinement Mechanisms").
+
+* Scale fits (joint, independent, 3-pass coordinate descent) with the codes
+  fixed: float32 scales within relative 1e-6 of the oracle's float64 fits
+  rounded to float32 (both round a float64-accurate value), objectives
+  within relative 1e-6.
+* Multi-code probe: the codes after the single-code search, the acceptance
+  of the Babai proposal and the number of codes it changes are integers
+  decided in float64 on both sides; they must agree on >= 99.5 % of the
+  (row, group) cases, and every disagreement must sit at a float64
+  near-tie of the oracle's own values (|dF| tiny against F).
+* Fixed grid: the scales stay bit-identical, codes >= 99.9 % identical to
+  the oracle's fixed-grid sweeps, objective within 5e-5.
+"""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+pytestmark = [pytest.mark.gpu,
+              pytest.mark.skipif(not torch.cuda.is_available(), reason="needs a CUDA GPU")]
+
+from oracle import (coordinate_descent_scales, independent_scales, joint_scales,  # noqa: E402
+                    multicode_probe, objective, prepare_hessian, refine_fixed_grid)
+from synth import small_layer  # noqa: E402
+
+
+@pytest.fixture(scope="module")
+def jarq():
+    from paper_2609_38599_gb300 import jarq as mod
+    return mod
+
+
+@pytest.mark.parametrize("din,dout,g,bits", [(256, 96, 64, 3), (384, 130, 128, 4)])
+@pytest.mark.parametrize("method", ["joint", "independent", "coordinate"])
+def test_scale_fit_parity(jarq, din, dout, g, bits, method):
+    lay = small_layer(din, dout, g, bits, seed=din + dout + 1)
+    prep = prepare_hessian(lay.H, lay.g)
+    if method == "joint":
+        ref = joint_scales(prep, lay.W, lay.S0, lay.Q0, lay.Z)
+    elif method == "independent":
+        ref = independent_scales(prep, lay.W, lay.S0, lay.Q0, lay.Z)
+    else:
+        ref = coordinate_descent_scales(prep, lay.W, lay.S0, lay.Q0, lay.Z, passes=3)
+    ref32 = ref.astype(np.float32)
+    hess = jarq.prepare(lay.H, lay.g)
+    S = lay.S0.copy()
+    Fb, Fa = jarq.fit_scales(hess, lay.W, S, lay.Q0, lay.Z, lay.bits, method, 3)
+    hess.close()
+    rel = np.abs(S.astype(np.float64) - ref32) / np.maximum(np.abs(ref32), 1e-30)
+    print(method, "max rel scale diff", rel.max(), "identical", np.mean(S == ref32))
+    assert rel.max() <= 1e-6
+    F0 = objective(prep, lay.W, lay.S0, lay.Q0, lay.Z)
+    F1 = objective(prep, lay.W, ref32, lay.Q0, lay.Z)
+    np.testing.assert_allclose(Fb, F0, rtol=1e-6)
+    np.testing.assert_allclose(Fa, F1, rtol=1e-6)
+    if method != "independent":
+        assert np.all(Fa <= Fb * (1 + 1e-9))
+
+
+@pytest.mark.parametrize("din,dout,g,bits", [(256, 80, 64, 3), (384, 64, 128, 3), (256, 48, 64, 4)])
+def test_multicode_probe_parity(jarq, din, dout, g, bits):
+    lay = small_layer(din, dout, g, bits, seed=din + dout + 2)
+    prep = prepare_hessian(lay.H, lay.g)
+    hess = jarq.prepare(lay.H, lay.g)
+    agree = total = 0
+    for i in range(din // g):
+        ref = multicode_probe(prep, lay.W, lay.S0, lay.Q0, lay.Z, lay.bits, i)
+        out = jarq.multicode_probe(hess, lay.W, lay.S0, lay.Q0, lay.Z, lay.bits, i)
+        same = (np.all(out["q_search"] == ref["q_search"], axis=1)
+                & (out["accepted"] == ref["accepted"]) & (out["changed"] == ref["changed"])
+                & (out["moves"] == ref["moves"]))
+        agree += int(same.sum())
+        total += same.size
+        F = objective(prep, lay.W, lay.S0, lay.Q0, lay.Z)
+        for j in np.nonzero(~same)[0]:
+            # a disagreement must start at a float64 near-tie
+            assert abs(ref["dF"][j]) <= 1e-9 * F[j] or out["moves"][j] != ref["moves"][j], (i, j)
+        both = same & ref["accepted"]
+        if both.any():
+            np.testing.assert_allclose(out["dF"][both], ref["dF"][both], rtol=1e-6,
+                                       atol=1e-12 * F.max())
+    hess.close()
+    print("probe agreement", agree, "/", total)
+    assert agree >= 0.995 * total
+
+
+def test_fixed_grid_parity(jarq):
+    lay = small_layer(256, 96, 64, 3, seed=41)
+    prep = prepare_hessian(lay.H, lay.g)
+    Qo, hist = refine_fixed_grid(prep, lay.W, lay.S0, lay.Q0, lay.Z, lay.bits, 3)
+    hess = jarq.prepare(lay.H, lay.g)
+    S, Q = lay.S0.copy(), lay.Q0.copy()
+    o = jarq.default_options(max_iters=3, early_stop=0)
+    o.fixed_grid = 1
+    st = jarq.refine(hess, lay.W, S, Q, lay.Z, lay.bits, options=o)
+    hess.close()
+    assert np.array_equal(S, lay.S0)
+    assert np.mean(Q == Qo) >= 0.999
+    F_gpu_state = objective(prep, lay.W, S, Q, lay.Z)
+    assert np.max(np.abs(st.L_final - F_gpu_state) / F_gpu_state) <= 5e-5
+    np.testing.assert_allclose(F_gpu_state, hist[-1], rtol=1e-4)
