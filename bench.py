@@ -412,6 +412,7 @@ def run_ours(args, rank, world):
     if rank == 0:
         line["hessian"] = hessian_leg(args, jarq, dev)
         line["mu_target"] = mu_target_leg(args, jarq, dev, lay.name)
+        line["ablations"] = ablation_leg(args, jarq, dev, lay, hess, ms)
     # end to end through the C ABI with pinned host buffers
     if rank == 0 or True:
         pin = lambda t: t.cpu().pin_memory().numpy()
@@ -508,6 +509,95 @@ def hessian_leg(args, jarq, dev, standalone=False):
         out["cpu_baseline"] = {"value": ns / t, "unit": "tokens/s", "cores": os.cpu_count(),
                                "kind": "oracle",
                                "sample": f"{ns} of {n} tokens, d={d}, float64, {t:.2f} s"}
+    return out
+
+
+def ablation_leg(args, jarq, dev, lay, hess, joint_ms):
+    """Tab. mechanism-summary (a) on the bench layer, from its RTN host
+    state (App. "Refinement Mechanisms"):
+    * scale fits with the host codes: median over rows of the gap
+      100 (F_method - F_joint) / F_host of the independent fit and of 3-pass
+      coordinate descent, and the call times;
+    * multi-code probe of every (row, group): share of cases where one Babai
+      proposal still lowers F after single-code search stops, median codes
+      such a proposal changes;
+    * Fixed (host scales, code sweeps) against Joint at equal time: Joint is
+      the timed K = 10 step; Fixed gets the sweeps that fit in that time; both
+      final states are scored on a held-out Hessian (the same distribution,
+      other tokens): median over rows of 100 (F_fixed - F_joint) / F_fixed and
+      the share of rows Joint improves."""
+    import torch
+    from synth import CONFIGS
+    from synth.layers import hessian_torch
+    out = {}
+    ev = lambda: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+
+    def timed(fn):
+        fn()
+        torch.cuda.synchronize()
+        a, b = ev()
+        a.record()
+        r = fn()
+        b.record()
+        torch.cuda.synchronize()
+        return r, a.elapsed_time(b)
+
+    F = {}
+    tms = {}
+    for m in ("joint", "independent", "coordinate"):
+        S = lay.S0.clone()
+        (Fb, Fa), tms[m] = timed(lambda: jarq.fit_scales(hess, lay.W, S.copy_(lay.S0), lay.Q0,
+                                                         lay.Z, lay.bits, m, 3))
+        F[m], F["host"] = Fa.cpu().numpy(), Fb.cpu().numpy()
+    for m in ("independent", "coordinate"):
+        out[f"gap_{m}_pct_median"] = float(np.median(100.0 * (F[m] - F["joint"]) / F["host"]))
+    out["fit_ms"] = tms
+    out["coordinate_time_ratio"] = tms["coordinate"] / tms["joint"]
+    G = lay.din // lay.g
+    acc, chg, moves = [], [], []
+    t0 = time.perf_counter()
+    for i in range(G):
+        r = jarq.multicode_probe(hess, lay.W, lay.S0, lay.Q0, lay.Z, lay.bits, i)
+        a = r["accepted"].cpu().numpy().astype(bool)
+        acc.append(a)
+        chg.append(r["changed"].cpu().numpy()[a])
+        moves.append(r["moves"].cpu().numpy())
+    out["probe_ms_per_group"] = (time.perf_counter() - t0) / G * 1e3
+    acc = np.concatenate(acc)
+    chg = np.concatenate(chg)
+    out["babai_after_single_code_pct"] = 100.0 * float(acc.mean())
+    out["median_codes_changed"] = float(np.median(chg)) if chg.size else 0.0
+    out["median_single_code_moves"] = float(np.median(np.concatenate(moves)))
+    # Fixed vs Joint at equal time
+    S, Q = lay.S0.clone(), lay.Q0.clone()
+    o = jarq.default_options(max_iters=lay.K, early_stop=0)
+    o.fixed_grid = 1
+
+    def fixed(k):
+        o.max_iters = k
+        S.copy_(lay.S0)
+        Q.copy_(lay.Q0)
+        jarq.refine(hess, lay.W, S, Q, lay.Z, lay.bits, options=o, collect_stats=False)
+
+    _, t_fix = timed(lambda: fixed(lay.K))
+    k_fixed = max(1, int(lay.K * joint_ms / t_fix))
+    fixed(k_fixed)
+    torch.cuda.synchronize()
+    Sf, Qf = S.clone(), Q.clone()
+    Sj, Qj = lay.S0.clone(), lay.Q0.clone()
+    jarq.refine(hess, lay.W, Sj, Qj, lay.Z, lay.bits, max_iters=lay.K, early_stop=0,
+                collect_stats=False)
+    c = CONFIGS[lay.name]
+    H_ho = hessian_torch(c["din"], c["rank"], c["n_out"], c["out_scale"], c["tokens"] // 4,
+                         c["D_lo"], c["seed"], dev, token_seed=9000 + c["seed"])
+    h_ho = jarq.prepare(H_ho, lay.g)
+    Ff = jarq.objective(h_ho, lay.W, Sf, Qf, lay.Z, lay.bits).cpu().numpy()
+    Fj = jarq.objective(h_ho, lay.W, Sj, Qj, lay.Z, lay.bits).cpu().numpy()
+    h_ho.close()
+    out["fixed_sweeps_in_joint_time"] = k_fixed
+    out["joint_over_fixed_heldout_pct_median"] = float(np.median(100.0 * (Ff - Fj) / Ff))
+    out["rows_improved_by_joint"] = float(np.mean(Fj < Ff))
+    out["heldout"] = f"{c['tokens'] // 4} other tokens of the same distribution"
     return out
 
 

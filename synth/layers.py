@@ -191,11 +191,13 @@ def tiny_layer(return_X=False):
 # --------------------------------------------------------------------------
 
 def hessian_torch(din, rank, n_out, out_scale, tokens, D_lo, seed, device,
-                  chunk=8192, damp=0.01):
+                  chunk=8192, damp=0.01, token_seed=None):
     """``X^T X / n + damp*mean(diag)*I`` accumulated chunk by chunk.
 
     Each 8192-token chunk's product is formed in float32 (full-precision
-    matmul, no TF32) and summed in float64.
+    matmul, no TF32) and summed in float64.  With ``token_seed`` the
+    distribution (L, D, outlier channels) is the one of ``seed`` and the
+    tokens are drawn from ``token_seed``: a held-out calibration set.
     """
     import torch
     gen = torch.Generator(device=device)
@@ -207,6 +209,8 @@ def hessian_torch(din, rank, n_out, out_scale, tokens, D_lo, seed, device,
         idx = torch.randperm(din, generator=gen, device=device)[:n_out]
         col[idx] = out_scale
     sqD = D.sqrt()
+    if token_seed is not None:
+        gen.manual_seed(token_seed)
     H = torch.zeros(din, din, dtype=torch.float64, device=device)
     prev = torch.get_float32_matmul_precision()
     torch.set_float32_matmul_precision("highest")
