@@ -31,7 +31,9 @@ namespace jarq {
 namespace {
 
 // In-place lower Cholesky of a G x G matrix (row stride G+1) by one warp.
-// Fails when a pivot is not above `thr` or is not finite.
+// Fails when a pivot is not above `thr` or is not finite.  Each lane owns
+// the rows a = lane (mod 32) of the trailing update; A[b][k] is read by all
+// lanes at once (a broadcast) and the rows a differ in bank (stride G + 1).
 __device__ bool warp_cholesky(float *A, int G, float thr) {
     const int lane = threadIdx.x & 31, ld = G + 1;
     for (int k = 0; k < G; ++k) {
@@ -43,10 +45,9 @@ __device__ bool warp_cholesky(float *A, int G, float thr) {
         if (lane == 0) A[k * ld + k] = lkk;
         for (int a = k + 1 + lane; a < G; a += 32) A[a * ld + k] /= lkk;
         __syncwarp();
-        const int n = G - k - 1;
-        for (int idx = lane; idx < n * n; idx += 32) {
-            int a = k + 1 + idx / n, b = k + 1 + idx % n;
-            if (b <= a) A[a * ld + b] = fmaf(-A[a * ld + k], A[b * ld + k], A[a * ld + b]);
+        for (int a = k + 1 + lane; a < G; a += 32) {
+            const float lak = A[a * ld + k];
+            for (int b = k + 1; b <= a; ++b) A[a * ld + b] = fmaf(-lak, A[b * ld + k], A[a * ld + b]);
         }
     }
     __syncwarp();
@@ -117,7 +118,9 @@ __global__ void scale_solve_kernel(SolveArgs a) {
     double *inc = b + G;                                      // increment of the scales
     const double *gj = a.gram + (size_t)j * G * G;
     const double *rj = a.rhs + (size_t)j * G;
-    auto gsym = [&](int r0, int c0) { return gj[r0 * G + c0]; };
+    // the Gram matrix is exactly symmetric: entry (r0, c0) is read as
+    // (c0, r0), so that lanes with consecutive r0 read consecutive addresses
+    auto gsym = [&](int r0, int c0) { return gj[c0 * G + r0]; };
     for (int t = lane; t < G; t += 32) so[t] = a.S[(size_t)j * G + t];
     __syncwarp();
     // gradient g = rhs - Gram s_old and F(s_old) = wHw - s_old^T (rhs + g)
@@ -151,13 +154,13 @@ __global__ void scale_solve_kernel(SolveArgs a) {
     }
     auto load_sym = [&](float shift) -> bool {
         bool finite = true;
-        for (int idx = lane; idx < G * G; idx += 32) {
-            int r0 = idx / G, c0 = idx % G;
-            float v = (float)gsym(r0, c0);
-            if (r0 == c0) v += shift;
-            if (!isfinite(v)) finite = false;
-            A[r0 * ld + c0] = v;
-        }
+        for (int r0 = 0; r0 < G; ++r0)
+            for (int c0 = lane; c0 < G; c0 += 32) {
+                float v = (float)gj[r0 * G + c0];
+                if (r0 == c0) v += shift;
+                if (!isfinite(v)) finite = false;
+                A[r0 * ld + c0] = v;
+            }
         __syncwarp();
         return __all_sync(0xffffffffu, finite);
     };
