@@ -16,13 +16,12 @@
 // so the pre-round value of Eq. babai_update is
 //     z + x_l = q_l + (y_l - sum_{h>l} R_lh Delta_h) / R_ll,
 // Delta_h = q^cand_h - q_h.  The running vector u = y - R Delta changes only
-// where Delta != 0, so the back substitution proceeds by jumps: every still
-// undecided coordinate rounds its current value in parallel, the highest one
-// whose code changes is fixed, its column updates u below it, and the scan
-// continues beneath it (one warp-wide max reduction per step picks the
-// coordinate and carries its code change).  Every u_l receives exactly the
-// updates, in the order, of the one-coordinate-at-a-time recursion; the
-// number of serial steps is the number of changed codes plus one.
+// where Delta != 0.  The back substitution scans h = g-1 .. 0: the lane that
+// owns coordinate h rounds it, the change is broadcast, and only when it is
+// non-zero do the coordinates below take the column update (a warp-uniform
+// branch).  A row none of whose codes would change at u = y has no change
+// at all (the first coordinate's value is final and unchanged, and so on
+// down) and skips the scan.
 //
 // The change of the group objective (Eq. group_bils) is
 // dF = s^2 (||R Delta - y||^2 - ||y||^2) = s^2 sum_l (a_l - y_l)(a_l + y_l)
@@ -148,46 +147,45 @@ __global__ void __launch_bounds__(32 * kMaxWarps) babai_kernel(BabaiArgs a) {
             y[t] = y[t] / s;
             u[t] = y[t];
         }
-        // back substitution by jumps (Eq. babai_update).  Rounding to the
-        // nearest even integer adds and subtracts 1.5 * 2^23 (exact for
-        // |x| < 2^22; beyond that the clamp to [0, qmax] gives the same code
-        // as rintf), and small integers travel in float bits: v + 2^23 has
-        // the bit pattern 0x4B000000 | v for 0 <= v < 2^23.
+        // back substitution (Eq. babai_update).  Rounding to the nearest
+        // even integer adds and subtracts 1.5 * 2^23 (exact for |x| < 2^22;
+        // beyond that the clamp to [0, qmax] gives the same code as rintf).
         const float qmaxf = (float)a.qmax;
         constexpr float kRound = 12582912.0f;      // 1.5 * 2^23
-        constexpr float kBias = 8388864.0f;        // 2^23 + 256
-        uint32_t pos[NT];                          // (l + 1) << 9 of this lane's coordinates
-#pragma unroll
-        for (int t = 0; t < NT; ++t) pos[t] = (uint32_t)(l0 + t + 1) << 9;
-        int hi = g - 1;
         bool any = false;
-        while (true) {
-            // each lane: its highest still-undecided coordinate whose code
-            // changes, as the key (l + 1) << 9 | (delta + 256); the warp-wide
-            // maximum is the highest such coordinate of the row
-            uint32_t key = 0;
+        // does any code change at u = y?
+        int nchg = 0;
 #pragma unroll
-            for (int t = 0; t < NT; ++t) {
-                const float x = fmaf(u[t], rd[t], qc[t]);
-                const float r = __fsub_rn(__fadd_rn(x, kRound), kRound);
-                const float q = fminf(fmaxf(r, 0.f), qmaxf);
-                const uint32_t kt = pos[t] | (__float_as_uint(__fadd_rn(q - qc[t], kBias)) & 511u);
-                if (l0 + t <= hi && q != qc[t]) key = kt;
+        for (int t = 0; t < NT; ++t) {
+            const float x = fmaf(u[t], rd[t], qc[t]);
+            const float r = __fsub_rn(__fadd_rn(x, kRound), kRound);
+            nchg += fminf(fmaxf(r, 0.f), qmaxf) != qc[t];
+        }
+        if (__any_sync(0xffffffffu, nchg != 0)) {
+            // descending scan (Eq. babai_update), coordinate h = NT L + t
+            for (int L = 31; L >= 0; --L) {
+#pragma unroll
+                for (int t = NT - 1; t >= 0; --t) {
+                    const int h = NT * L + t;
+                    float dq = 0.f;
+                    if (lane == L) {
+                        const float x = fmaf(u[t], rd[t], qc[t]);
+                        const float r = __fsub_rn(__fadd_rn(x, kRound), kRound);
+                        const float q = fminf(fmaxf(r, 0.f), qmaxf);
+                        dq = q - qc[t];
+                        qn[t] = q;
+                    }
+                    dq = __shfl_sync(0xffffffffu, dq, L);
+                    if (dq != 0.f) {                      // warp-uniform
+                        any = true;
+                        float lr[NT];
+                        load_vec<NT>(Lg + h * g + l0, lr);   // R[l'][h] for l' = l0..
+#pragma unroll
+                        for (int tt = 0; tt < NT; ++tt)
+                            if (l0 + tt < h) u[tt] = fmaf(-lr[tt], dq, u[tt]);
+                    }
+                }
             }
-            const uint32_t best = __reduce_max_sync(0xffffffffu, key);
-            if (!best) break;
-            const int lstar = (int)(best >> 9) - 1;
-            const float fd = __uint_as_float((best & 511u) | 0x4B000000u) - kBias;
-#pragma unroll
-            for (int t = 0; t < NT; ++t)
-                if (l0 + t == lstar) qn[t] = qc[t] + fd;
-            any = true;
-            float lr[NT];
-            load_vec<NT>(Lg + lstar * g + l0, lr);   // R[l'][l*] for l' = l0..
-#pragma unroll
-            for (int t = 0; t < NT; ++t)
-                if (l0 + t < lstar) u[t] = fmaf(-lr[t], fd, u[t]);
-            hi = lstar - 1;
         }
         if (!any) continue;
         float acc = 0.f;
