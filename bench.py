@@ -44,11 +44,11 @@ DTYPE = "f32 (integer-digit fp16/bf16 tensor-core products with exact partial su
 # file is unchanged (first 12 hex digits of its SHA-1).
 TRAFFIC = {
     "target": ("k_tc_target.cu", "07c974948b9d", 38.300e6 + 0.043264e6),
-    "babai": ("k_babai.cu", "5ea8bbe0238f", 14.275e6 + 0.002560e6),
-    "gram": ("k_tc_gram.cu", "3160a3b4f82d", 163.402e6 + 27.876352e6),
-    "proj": ("k_tc_proj.cu", "391ad329f213", 1374.367e6 + 155.951104e6),
-    "ptilde": ("k_tc_proj.cu", "391ad329f213", 138.978e6 + 90.157056e6),
-    "scale_solve": ("k_solve.cu", "b1417ed940dd", 35.257e6 + 0.002560e6),
+    "babai": ("k_babai.cu", "d2d96a20da85", 14.274e6 + 0.001536e6),
+    "gram": ("k_tc_gram.cu", "03e045e2e481", 163.166e6 + 27.856384e6),
+    "proj": ("k_tc_proj.cu", "9a9de7b74f80", 1371.623e6 + 156.537856e6),
+    "ptilde": ("k_tc_proj.cu", "9a9de7b74f80", 138.444e6 + 89.543168e6),
+    "scale_solve": ("k_solve.cu", "f3195c119d2c", 35.257e6 + 0.0),
     # profiles/ncu_syrk_attn_in_4096_n32768.md, scaled from 32768 to 262144 tokens
     "syrk": ("k_syrk.cu", "3896afedc783", 8 * 537.171e6 + 40.712e6),
 }
