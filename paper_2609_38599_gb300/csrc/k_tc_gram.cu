@@ -22,6 +22,8 @@
 // dots through shared memory at the end of each block.  One unit of work is
 // (h, column half of group i): 4 accumulators of 64 columns (one per digit
 // plane), double-buffered in 512 TMEM columns.
+#include <type_traits>
+
 #include "tc_common.cuh"
 
 namespace jarq {
@@ -30,10 +32,20 @@ namespace {
 constexpr int kTileA = 128 * 64 * 2;   // 128 code rows x 64 K (fp16)
 constexpr int kTileB = 64 * 64 * 2;    // 64 H rows x 64 K, one digit plane (fp16)
 constexpr int kStage = kTileA + 4 * kTileB;
-constexpr int kStages = 3;
-constexpr int kCodesBytes = 128 * 128 * 2;  // int16 codes of group i for the tile
+// Codes of group i are staged per tile as int8 when they fit (|q - z| <= 127,
+// up to 7 bits; then the freed shared memory holds a fourth pipeline stage)
+// and as int16 otherwise.
+template <bool WIDE>
+struct GramCfg {
+    using code_t = typename std::conditional<WIDE, int16_t, int8_t>::type;
+    static constexpr int kStages = WIDE ? 3 : 4;
+    static constexpr int kCodesBytes = 128 * 128 * (int)sizeof(code_t);
+};
 constexpr int kPartBytes = 2 * 4 * 128 * 8;  // int64 partial dots, double-buffered
-constexpr int kSmem = 1024 + kStages * kStage + kCodesBytes + kPartBytes + 256;
+template <bool WIDE>
+constexpr int gram_smem() {
+    return 1024 + GramCfg<WIDE>::kStages * kStage + GramCfg<WIDE>::kCodesBytes + kPartBytes + 256;
+}
 constexpr int kThreads = 320;
 // one MMA covers the four digit planes: they are consecutive 64-row tiles
 // in shared memory, and their accumulators consecutive 64-column blocks
@@ -63,7 +75,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                    GramArgs a) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    int16_t *codes = (int16_t *)(smem + kStages * kStage);   // [128 rows][128]
+    using code_t = typename GramCfg<WIDE>::code_t;
+    constexpr int kStages = GramCfg<WIDE>::kStages;
+    constexpr int kCodesBytes = GramCfg<WIDE>::kCodesBytes;
+    code_t *codes = (code_t *)(smem + kStages * kStage);   // [128 rows][128]
     long long *part = (long long *)(smem + kStages * kStage + kCodesBytes);   // [2][4][128]
     uint64_t *bars = (uint64_t *)(smem + kStages * kStage + kCodesBytes + kPartBytes);
     uint32_t *tmem_slot = (uint32_t *)(bars + 2 * kStages + 4);
@@ -200,7 +215,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                             for (int k = 0; k < 16; ++k)
                                 codes[rl * 128 + c0 + m16 * 16 + k] =
-                                    (int16_t)((int)((w4[k >> 2] >> (8 * (k & 3))) & 0xFFu) - zz);
+                                    (code_t)((int)((w4[k >> 2] >> (8 * (k & 3))) & 0xFFu) - zz);
                         }
                     } else {
                         for (int m = 0; m < 32; ++m) codes[rl * 128 + c0 + m] = 0;
@@ -221,16 +236,27 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             if (!dead) {
                 const uint32_t base = tmem + ((uint32_t)(32 * q) << 16) + b * 256 + cw * 32;
-                const int16_t *crow = codes + rl * 128 + half * 64 + cw * 32;
+                const code_t *crow = codes + rl * 128 + half * 64 + cw * 32;
                 int cr[32];
+                if constexpr (WIDE) {
 #pragma unroll
-                for (int e = 0; e < 32; e += 8) {
-                    const int4 pk = *reinterpret_cast<const int4 *>(crow + e);
-                    const int w4[4] = {pk.x, pk.y, pk.z, pk.w};
+                    for (int e = 0; e < 32; e += 8) {
+                        const int4 pk = *reinterpret_cast<const int4 *>(crow + e);
+                        const int w4[4] = {pk.x, pk.y, pk.z, pk.w};
 #pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        cr[e + 2 * k] = (int)(int16_t)(w4[k] & 0xFFFF);
-                        cr[e + 2 * k + 1] = w4[k] >> 16;
+                        for (int k = 0; k < 4; ++k) {
+                            cr[e + 2 * k] = (int)(int16_t)(w4[k] & 0xFFFF);
+                            cr[e + 2 * k + 1] = w4[k] >> 16;
+                        }
+                    }
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 32; e += 16) {
+                        const int4 pk = *reinterpret_cast<const int4 *>(crow + e);
+                        const int w4[4] = {pk.x, pk.y, pk.z, pk.w};
+#pragma unroll
+                        for (int k = 0; k < 16; ++k)
+                            cr[e + k] = (int)(int8_t)((w4[k >> 2] >> (8 * (k & 3))) & 0xFF);
                     }
                 }
 #pragma unroll
@@ -441,10 +467,10 @@ cudaError_t launch_tc_gram(const CUtensorMap &mapC, const CUtensorMap &mapS, con
     static bool attr_set = false;
     if (!attr_set) {
         cudaError_t e = cudaFuncSetAttribute(tc_gram_kernel<false>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, gram_smem<false>());
         if (e == cudaSuccess)
             e = cudaFuncSetAttribute(tc_gram_kernel<true>,
-                                     cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, gram_smem<true>());
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
@@ -452,9 +478,9 @@ cudaError_t launch_tc_gram(const CUtensorMap &mapC, const CUtensorMap &mapS, con
     GramArgs a{Q, Z, expo, active, gram, status, p, d, g, G, d_pad};
     dim3 grid(p_pad / 128, (G + 1) / 2, 1);
     if (bits <= 4)
-        tc_gram_kernel<false><<<grid, kThreads, kSmem, s>>>(mapC, mapS, a);
+        tc_gram_kernel<false><<<grid, kThreads, gram_smem<false>(), s>>>(mapC, mapS, a);
     else
-        tc_gram_kernel<true><<<grid, kThreads, kSmem, s>>>(mapC, mapS, a);
+        tc_gram_kernel<true><<<grid, kThreads, gram_smem<true>(), s>>>(mapC, mapS, a);
     return cudaGetLastError();
 }
 

@@ -451,38 +451,44 @@ __global__ void __launch_bounds__(512) ptilde_kernel(const float *__restrict__ P
         pl[idx] = in ? Plo[o] : 0.f;
     }
     __syncthreads();
-    // each thread: one output column a and kRowsPer rows, independent chains
+    // each thread: the column pair (a, g-1-a), so that every thread (and every
+    // warp, hence every scheduler) does about the same g+1 steps of the
+    // triangle, and kRowsPer rows as independent chains
     constexpr int kRowsPer = 8;
-    const int a = tid % g, jstep = blockDim.x / g;
-    for (int jb = (tid / g) * kRowsPer; jb < kPtRows; jb += jstep * kRowsPer) {
-        float sh[kRowsPer], sl[kRowsPer];
-#pragma unroll
-        for (int r = 0; r < kRowsPer; ++r) {
-            sh[r] = 0.f;
-            sl[r] = 0.f;
-        }
-        for (int b = 0; b <= a; ++b) {
-            const float xh = rh[b * g + a], xl = rl[b * g + a];
+    const int npairs = g / 2, pair = tid % npairs, rstep = (blockDim.x / npairs) * kRowsPer;
+    for (int jb = (tid / npairs) * kRowsPer; jb < kPtRows; jb += rstep) {
+#pragma unroll 1
+        for (int side = 0; side < 2; ++side) {
+            const int a = side == 0 ? pair : g - 1 - pair;
+            float sh[kRowsPer], sl[kRowsPer];
 #pragma unroll
             for (int r = 0; r < kRowsPer; ++r) {
-                const float yh = ph[(jb + r) * g + b], yl = pl[(jb + r) * g + b];
-                const float m = xh * yh;
-                float e = fmaf(xh, yh, -m);
-                e = fmaf(xh, yl, fmaf(xl, yh, e));
-                float s2, e2;
-                two_sum(sh[r], m, s2, e2);
-                sh[r] = s2;
-                sl[r] += e2 + e;
+                sh[r] = 0.f;
+                sl[r] = 0.f;
             }
-        }
+            for (int b = 0; b <= a; ++b) {
+                const float xh = rh[b * g + a], xl = rl[b * g + a];
 #pragma unroll
-        for (int r = 0; r < kRowsPer; ++r) {
-            if (r0 + jb + r < p) {
-                float s2, e2;
-                two_sum(sh[r], sl[r], s2, e2);
-                const size_t o = (size_t)(r0 + jb + r) * d + (size_t)i * g + a;
-                out_hi[o] = s2;
-                out_lo[o] = e2;
+                for (int r = 0; r < kRowsPer; ++r) {
+                    const float yh = ph[(jb + r) * g + b], yl = pl[(jb + r) * g + b];
+                    const float m = xh * yh;
+                    float e = fmaf(xh, yh, -m);
+                    e = fmaf(xh, yl, fmaf(xl, yh, e));
+                    float s2, e2;
+                    two_sum(sh[r], m, s2, e2);
+                    sh[r] = s2;
+                    sl[r] += e2 + e;
+                }
+            }
+#pragma unroll
+            for (int r = 0; r < kRowsPer; ++r) {
+                if (r0 + jb + r < p) {
+                    float s2, e2;
+                    two_sum(sh[r], sl[r], s2, e2);
+                    const size_t o = (size_t)(r0 + jb + r) * d + (size_t)i * g + a;
+                    out_hi[o] = s2;
+                    out_lo[o] = e2;
+                }
             }
         }
     }

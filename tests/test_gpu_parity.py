@@ -61,6 +61,8 @@ def test_tiny_layer_parity(jarq, early_stop):
     (448, 33, 64, 3, 5),      # seven groups of 64
     (640, 129, 128, 3, 4),    # five groups of 128
     (1024, 300, 128, 4, 2),   # several K chunks per split
+    (256, 96, 64, 6, 3),      # 6-bit: codes beyond 4 bits (wide integer dots)
+    (384, 64, 128, 8, 2),     # 8-bit: codes need 16-bit staging
 ])
 def test_shapes_parity(jarq, din, dout, g, bits, K):
     lay = small_layer(din, dout, g, bits, K=K, seed=din + dout + g)
