@@ -30,3 +30,20 @@ def gather_rows(local, dout: int, group=None):
     outs = [torch.empty_like(pad) for _ in range(world)]
     dist.all_gather(outs, pad, group=group)
     return torch.cat([o[: b - a] for o, (a, b) in zip(outs, sizes)], dim=0)
+
+
+def token_range(n: int, rank: int, world: int):
+    """Contiguous [start, stop) of the calibration tokens a rank accumulates.
+
+    The Hessian H = X^T X + nu^2 I (Eq. strict_target) is a sum over tokens, so
+    the tokens shard across ranks with one exchange: each rank forms the
+    partial product of its tokens (``jarq_accumulate_hessian``) and the
+    partials are summed on every rank (``allreduce_hessian``)."""
+    return row_range(n, rank, world)
+
+
+def allreduce_hessian(H_local, group=None):
+    """Sum the ranks' partial Hessians in place (one all-reduce); returns H."""
+    import torch.distributed as dist
+    dist.all_reduce(H_local, op=dist.ReduceOp.SUM, group=group)
+    return H_local

@@ -73,3 +73,42 @@ def test_two_gloo_ranks_match_single_process():
     assert np.array_equal(Q, ref.Q)
     np.testing.assert_allclose(S, ref.S, rtol=0, atol=0)
     assert tmax == 2.0
+
+
+def _hessian_worker(rank, world, port, q):
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        from oracle import accumulate_hessian
+        from paper_2609_38599_gb300.shard import allreduce_hessian, token_range
+        from synth import integer_activations_np
+        X = integer_activations_np(1001, 24, amax=8, seed=5)
+        a, b = token_range(X.shape[0], rank, world)
+        H = torch.as_tensor(accumulate_hessian(X[a:b]))   # this rank's partial X^T X
+        allreduce_hessian(H)
+        if rank == 0:
+            q.put(H.numpy())
+    finally:
+        dist.destroy_process_group()
+
+
+def test_token_sharded_hessian_equals_single_process():
+    """Three gloo ranks accumulate disjoint token ranges and sum the partial
+    Hessians with one all-reduce; on integer activations the sum is exact,
+    so it must equal the single-process product bit for bit.  The oracle
+    stands in for each rank's GPU call."""
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_hessian_worker, args=(r, 3, port, q)) for r in range(3)]
+    for p in procs:
+        p.start()
+    H = q.get(timeout=300)
+    for p in procs:
+        p.join(timeout=120)
+        assert p.exitcode == 0
+    from oracle import accumulate_hessian
+    from synth import integer_activations_np
+    X = integer_activations_np(1001, 24, amax=8, seed=5)
+    np.testing.assert_array_equal(H, accumulate_hessian(X))
