@@ -27,9 +27,8 @@
 // The drain does about 19 float32 operations per output and group, hence
 // sixteen drain warps; the scale and block exponent of the next group are
 // loaded one group ahead.
-// The kernel is bound by moving tiles into shared memory, and the digit
-// tiles are the same for every row tile.  CTAs of consecutive row tiles
-// therefore form a cluster of C: each loads 4/C of the digit planes and
+// The digit tiles are the same for every row tile, so CTAs of consecutive
+// row tiles can form a cluster of C: each loads 4/C of the digit planes and
 // multicasts them to all C, cutting that traffic by C.  A stage is refilled
 // only after every CTA of the cluster has consumed it (its "empty" barrier
 // counts one MMA commit per CTA), and no CTA leaves before the others.
@@ -296,7 +295,11 @@ cudaError_t launch_tc_target(const CUtensorMap &mapC, const CUtensorMap &mapT, f
     }
     const int per = (G + nsplit - 1) / nsplit;
     const int tiles = p_pad / 128;
-    const int csize = tiles % 4 == 0 ? 4 : tiles % 2 == 0 ? 2 : 1;
+    // The kernel supports clusters of 2 or 4 row tiles multicasting the digit
+    // tiles (csize); on the q_proj workload single CTAs measured faster
+    // (35.3 against 37.2 us per launch with 4): the stage lockstep of a
+    // cluster costs more than the L2 traffic it saves.
+    const int csize = 1;
     TargetArgs a{out_hi, out_lo, S, expoT, active, status, p, p_pad, d_pad, g, G, i, per, csize};
     dim3 grid(tiles, g / 64, nsplit);
     return launch_pdl_cluster(tc_target_kernel, grid, dim3(kThreads), (size_t)kSmem, s, csize,
