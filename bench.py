@@ -43,11 +43,11 @@ DTYPE = "f32 (integer-digit fp16/bf16 tensor-core products with exact partial su
 # profiles/ncu_syrk_attn_in_4096_n32768.md), valid while the kernel's source
 # file is unchanged (first 12 hex digits of its SHA-1).
 TRAFFIC = {
-    "target": ("k_tc_target.cu", "07c974948b9d", 38.300e6 + 0.043264e6),
+    "target": ("k_tc_target.cu", "86cd9636faf0", 38.300e6 + 0.125e6),
     "babai": ("k_babai.cu", "d2d96a20da85", 14.274e6 + 0.001536e6),
-    "gram": ("k_tc_gram.cu", "03e045e2e481", 163.166e6 + 27.856384e6),
-    "proj": ("k_tc_proj.cu", "9a9de7b74f80", 1371.623e6 + 156.537856e6),
-    "ptilde": ("k_tc_proj.cu", "9a9de7b74f80", 138.444e6 + 89.543168e6),
+    "gram": ("k_tc_gram.cu", "c839a427ea94", 164.246e6 + 27.889664e6),
+    "proj": ("k_tc_proj.cu", "7fe129ae0adf", 1374.566e6 + 156.723968e6),
+    "ptilde": ("k_tc_proj.cu", "7fe129ae0adf", 138.449e6 + 90.958080e6),
     "scale_solve": ("k_solve.cu", "f3195c119d2c", 35.257e6 + 0.0),
     # profiles/ncu_syrk_attn_in_4096_n32768.md, scaled from 32768 to 262144 tokens
     "syrk": ("k_syrk.cu", "3896afedc783", 8 * 537.171e6 + 40.712e6),

@@ -101,3 +101,34 @@ def test_fixed_grid_parity(jarq):
     F_gpu_state = objective(prep, lay.W, S, Q, lay.Z)
     assert np.max(np.abs(st.L_final - F_gpu_state) / F_gpu_state) <= 5e-5
     np.testing.assert_allclose(F_gpu_state, hist[-1], rtol=1e-4)
+
+
+def test_full_size_scale_fits_and_probe_sampled_rows(jarq):
+    """The q_proj layer (4096 x 4096, g = 128, 3-bit) from its RTN state: the
+    three scale fits and the multi-code probe of two groups on the whole layer;
+    the oracle on 24 seeded rows."""
+    from synth import config_layer
+    lay = config_layer("llama2_7b_q_proj_4096x4096_g128_w3", device="cuda")
+    rng = np.random.Generator(np.random.PCG64(77))
+    rows = np.sort(rng.choice(lay.dout, 24, replace=False))
+    cpu = lambda t: t.cpu().numpy()
+    W, S0, Q0, Z = cpu(lay.W)[rows], cpu(lay.S0)[rows], cpu(lay.Q0)[rows], cpu(lay.Z)[rows]
+    prep = prepare_hessian(cpu(lay.H), lay.g)
+    hess = jarq.prepare(lay.H, lay.g)
+    for method, fit in (("joint", joint_scales), ("independent", independent_scales),
+                        ("coordinate", lambda *a: coordinate_descent_scales(*a, passes=3))):
+        S = lay.S0.clone()
+        jarq.fit_scales(hess, lay.W, S, lay.Q0, lay.Z, lay.bits, method, 3)
+        ref = fit(prep, W, S0, Q0, Z).astype(np.float32)
+        rel = np.abs(cpu(S)[rows].astype(np.float64) - ref) / np.maximum(np.abs(ref), 1e-30)
+        print(method, "max rel", rel.max())
+        assert rel.max() <= 1e-6, method
+    for i in (0, 17):
+        out = jarq.multicode_probe(hess, lay.W, lay.S0, lay.Q0, lay.Z, lay.bits, i)
+        ref = multicode_probe(prep, W, S0, Q0, Z, lay.bits, i)
+        same = (np.all(cpu(out["q_search"])[rows] == ref["q_search"], axis=1)
+                & (cpu(out["accepted"])[rows] == ref["accepted"])
+                & (cpu(out["changed"])[rows] == ref["changed"]))
+        print("group", i, "probe rows identical", int(same.sum()), "/", len(rows))
+        assert same.mean() >= 0.95
+    hess.close()

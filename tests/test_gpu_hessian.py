@@ -146,3 +146,27 @@ def test_full_size_attention_input_sampled(jarq):
     assert np.array_equal(Hn, Hn.T)
     del X, H
     torch.cuda.empty_cache()
+
+
+def test_full_size_down_proj_input_sampled(jarq):
+    """The down_proj input (d = 11008, 1892 tiles) over 64 x 2048 tokens, in
+    one call; 64 sampled features against the oracle."""
+    X = config_activations("llama2_7b_down_in_11008_n131072", device="cuda")
+    n, d = X.shape
+    H = jarq.accumulate_hessian(X)
+    torch.cuda.synchronize()
+    rng = np.random.Generator(np.random.PCG64(7))
+    idx = np.sort(np.concatenate([[0, d - 1], rng.choice(np.arange(1, d - 1), 62, replace=False)]))
+    it = torch.as_tensor(idx, device="cuda")
+    Xs = X.index_select(1, it).cpu().numpy()
+    ref = accumulate_hessian(Xs)
+    absdot = accumulate_hessian(np.abs(Xs))
+    Hs = H.index_select(0, it).index_select(1, it).cpu().numpy().astype(np.float64)
+    err = np.abs(Hs - ref)
+    bound = gamma(n) * absdot + 2.0 ** -24 * np.abs(ref)
+    print("down_in: max err / bound", float((err / bound).max()))
+    assert np.all(err <= bound)
+    Hn = H.cpu().numpy()
+    assert np.array_equal(Hn, Hn.T)
+    del X, H
+    torch.cuda.empty_cache()
