@@ -592,7 +592,8 @@ jarq_status jarq_multicode_probe(jarq_hessian *h, const float *W, const float *S
                                   h->d_pad, g, h->dstatus, st));
     // T = sum_h s_h H_ih c_h: the phase product with H's own digits
     RUN("target", 1, launch_tc_target(w.mapC, h->mapD10, w.t_hi, w.t_lo, la.S, h->expo, nullptr, p,
-                                      w.p_pad, h->d_pad, g, G, group, nsplit, h->dstatus, st));
+                                      w.p_pad, h->d_pad, g, G, group, nsplit, (1 << bits) - 1, h->dstatus,
+                                      st));
     uint8_t *qo = reinterpret_cast<uint8_t *>(w.Hr);
     RUN("probe", 1, launch_probe(w.Phi, w.Plo, w.t_hi, w.t_lo, h->Hs, h->L64, la.S, la.Q, la.Z, qo,
                                  w.iters, w.accepted, w.ridge, w.L_final, p, w.p_pad, d, g, group,
@@ -663,7 +664,7 @@ jarq_status refine_impl(jarq_hessian *h, const float *W, float *S, uint8_t *Q, c
         for (int i = 0; i < G; ++i) {
             RUN("target", 1, launch_tc_target(w.mapC, h->mapHt, w.t_hi, w.t_lo, la.S, h->expoT,
                                               w.active, p, w.p_pad, h->d_pad, g, G, i, nsplit,
-                                              h->dstatus, st));
+                                              qmax, h->dstatus, st));
             RUN("babai", 1, launch_babai(w.t_hi, w.t_lo, w.Pt_hi, w.Pt_lo, nsplit, h->Lf, la.S, la.Q,
                                          la.Z, rv, w.active, w.accepted, h->dstatus, p, g, i, qmax,
                                          o.eps, st));

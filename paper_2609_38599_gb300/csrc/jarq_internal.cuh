@@ -203,7 +203,7 @@ cudaError_t launch_ptilde(const float *Phi, const float *Plo, const double *Rinv
 int target_splits(int p_pad, int g, int G);
 cudaError_t launch_tc_target(const CUtensorMap &mapC, const CUtensorMap &mapT, float *out_hi,
                              float *out_lo, const float *S, const int *expoT, const int *active,
-                             int p, int p_pad, int d_pad, int g, int G, int i, int nsplit,
+                             int p, int p_pad, int d_pad, int g, int G, int i, int nsplit, int qmax,
                              int *status, cudaStream_t s);
 
 // Launch with programmatic stream serialization: the kernel may start while

@@ -24,7 +24,7 @@
 //   warp 1       TMEM allocation and the single-thread MMA issuer
 //   warps 2..17  drain: warp w reads TMEM lanes 32 (w % 4) and 16 columns
 // Four 64-column accumulators per group h, double-buffered (512 columns).
-// The drain does about 19 float32 operations per output and group, hence
+// The drain does 17 float32 operations per output and group, hence
 // sixteen drain warps; the scale and block exponent of the next group are
 // loaded one group ahead.
 // The digit tiles are the same for every row tile, so CTAs of consecutive
@@ -32,6 +32,8 @@
 // multicasts them to all C, cutting that traffic by C.  A stage is refilled
 // only after every CTA of the cluster has consumed it (its "empty" barrier
 // counts one MMA commit per CTA), and no CTA leaves before the others.
+#include <cmath>
+
 #include "tc_common.cuh"
 
 namespace jarq {
@@ -56,6 +58,7 @@ struct TargetArgs {
     int *status;
     int p, p_pad, d_pad, g, G, i, seg_per_split;
     int csize;                // CTAs per cluster (1, 2 or 4)
+    float round_c;            // 1.5 * 2^(23 - k): rounds to multiples of 2^-k
 };
 
 __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
@@ -229,10 +232,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
 #pragma unroll
                 for (int e = 0; e < 8; ++e) {
-                    // D_0 + D_1 2^-10 exactly as (vh, vl); the D_2, D_3 terms are
-                    // below 2^-20 of it and enter the low part
-                    float vh, vl, s2, e2;
-                    two_sum(__uint_as_float(v0[e]), __uint_as_float(v1[e]) * 0x1p-10f, vh, vl);
+                    // D_0 + D_1 2^-10 exactly as (vh, vl): the digit sums are
+                    // integers with |D_0| <= 128 qmax 512 and |D_1 2^-10| < 2^14;
+                    // t = D_1 2^-10 rounded to a multiple of 2^-k (by adding
+                    // and subtracting 1.5 2^(23-k)), with k chosen on the host
+                    // so that |D_0 + t| < 2^(24-k): then vh = D_0 + t and
+                    // vl = D_1 2^-10 - t (|vl| <= 2^-(k+1)) are exact.  The
+                    // D_2, D_3 terms are below 2^-20 of the sum and enter the
+                    // low part.
+                    float s2, e2;
+                    const float d1 = __uint_as_float(v1[e]);
+                    const float tq = __fsub_rn(__fmaf_rn(d1, 0x1p-10f, a.round_c), a.round_c);
+                    const float vh = __fadd_rn(__uint_as_float(v0[e]), tq);
+                    float vl = __fmaf_rn(d1, 0x1p-10f, -tq);
                     vl = fmaf(__uint_as_float(v2[e]), 0x1p-20f, vl);
                     vl = fmaf(__uint_as_float(v3[e]), 0x1p-30f, vl);
                     // (vh + vl) * scale, added to the accumulator
@@ -285,7 +297,7 @@ int target_splits(int p_pad, int g, int G) {
 cudaError_t launch_tc_target(const CUtensorMap &mapC, const CUtensorMap &mapT, float *out_hi,
                              float *out_lo, const float *S, const int *expoT, const int *active,
                              int p, int p_pad, int d_pad, int g, int G, int i, int nsplit,
-                             int *status, cudaStream_t s) {
+                             int qmax, int *status, cudaStream_t s) {
     static bool attr_set = false;
     if (!attr_set) {
         cudaError_t e = cudaFuncSetAttribute(tc_target_kernel,
@@ -300,7 +312,15 @@ cudaError_t launch_tc_target(const CUtensorMap &mapC, const CUtensorMap &mapT, f
     // (35.3 against 37.2 us per launch with 4): the stage lockstep of a
     // cluster costs more than the L2 traffic it saves.
     const int csize = 1;
-    TargetArgs a{out_hi, out_lo, S, expoT, active, status, p, p_pad, d_pad, g, G, i, per, csize};
+    // quantum 2^-k of the exact digit split: the largest k with
+    // 128 qmax 512 + 2^14 <= 2^(24-k)
+    if (qmax < 1 || qmax > 255 || g > 128) return cudaErrorInvalidValue;
+    const double bound = 128.0 * qmax * 512.0 + 16384.0;
+    int kq = 0;
+    while (kq < 7 && bound <= std::ldexp(1.0, 24 - (kq + 1))) ++kq;
+    const float round_c = (float)std::ldexp(1.5, 23 - kq);
+    TargetArgs a{out_hi, out_lo, S, expoT, active, status, p, p_pad, d_pad, g, G, i, per, csize,
+                 round_c};
     dim3 grid(tiles, g / 64, nsplit);
     return launch_pdl_cluster(tc_target_kernel, grid, dim3(kThreads), (size_t)kSmem, s, csize,
                               mapC, mapT, a);
