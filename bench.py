@@ -235,9 +235,9 @@ def kernel_model(kernel, lay, nsplit_bytes=0):
     products they issue (4 digit planes for the phase target product and the
     Gram, 18 digit pairs for the target projection) are reported separately
     as ``issued``.  Babai counts its dense triangular back substitution,
-    g^2 flops per (row, group); the folded projection its g^2 / 2
-    multiply-adds per (row, group) in double-float.  Memory-bound kernels
-    count the bytes they must move once.
+    g^2 flops per (row, group); the folded projection one MMA of its
+    block-diagonal product (2 x p x d x g; 21 digit pairs issued).
+    Memory-bound kernels count the bytes they must move once.
     """
     p, d, g, G = lay.dout, lay.din, lay.g, lay.din // lay.g
     if kernel == "target":
@@ -250,7 +250,7 @@ def kernel_model(kernel, lay, nsplit_bytes=0):
     if kernel == "babai":
         return dict(bound="alu", work=1.0 * g * g * p)
     if kernel == "ptilde":
-        return dict(bound="alu", work=1.0 * p * d * g)
+        return dict(bound="tensor", work=2.0 * p * d * g, issued=21 * 2.0 * p * d * g)
     if kernel == "scale_solve":
         # Gram (f64), rhs (f64), wHw, L_prev and the scales in; scales and L out
         return dict(bound="hbm", work=p * (8.0 * G * G + 8 * G + 8 + 8 + 4 * G + 4 * G + 8))

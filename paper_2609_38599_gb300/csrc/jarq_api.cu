@@ -160,9 +160,11 @@ cudaError_t ensure_ws(jarq_hessian *h, int p) {
     if ((e = cudaMemset(w.cplane, 0, (size_t)p_pad * h->d_pad * 2)) != cudaSuccess) return e;
     if ((e = make_tmap_f16(&w.mapC, w.cplane, (uint64_t)p_pad, h->d_pad, 128)) != cudaSuccess)
         return e;
-    if ((e = dalloc(&w.wdig, (size_t)4 * p_pad * h->d_pad)) != cudaSuccess) return e;
-    if ((e = cudaMemset(w.wdig, 0, (size_t)4 * p_pad * h->d_pad * 2)) != cudaSuccess) return e;
+    if ((e = dalloc(&w.wdig, (size_t)6 * p_pad * h->d_pad)) != cudaSuccess) return e;
+    if ((e = cudaMemset(w.wdig, 0, (size_t)6 * p_pad * h->d_pad * 2)) != cudaSuccess) return e;
     if ((e = make_tmap_bf16(&w.mapWd, w.wdig, (uint64_t)4 * p_pad, h->d_pad, 128)) != cudaSuccess)
+        return e;
+    if ((e = make_tmap_bf16(&w.mapPd, w.wdig, (uint64_t)6 * p_pad, h->d_pad, 128)) != cudaSuccess)
         return e;
     w.p_pad = p_pad;
     if ((e = dalloc(&w.Hr, (size_t)p * d)) != cudaSuccess) return e;
@@ -397,6 +399,8 @@ void jarq_hessian_destroy(jarq_hessian *h) {
     cudaFree(h->Lf);
     cudaFree(h->L64);
     cudaFree(h->Rinv);
+    cudaFree(h->rdig);
+    cudaFree(h->rexp);
     cudaFree(h->Htdig);
     cudaFree(h->expoT);
     cudaFree(h->qdig);
@@ -442,6 +446,9 @@ jarq_status jarq_prepare_hessian(const float *H, int din, int group_size, float 
         if ((e = dalloc(&h->Lf, (size_t)h->G * group_size * group_size)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->L64, (size_t)h->G * group_size * group_size)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->Rinv, (size_t)h->G * group_size * group_size)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = dalloc(&h->rdig, (size_t)6 * din * group_size)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = dalloc(&h->rexp, (size_t)h->G)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = make_tmap_bf16(&h->mapRi, h->rdig, (uint64_t)6 * din, group_size, 64)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->Htdig, 4 * pd)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = cudaMemsetAsync(h->Htdig, 0, 4 * pd * 2, st)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->expoT, (size_t)h->G * h->G)) != cudaSuccess) { rc = cuda_fail(e); break; }
@@ -458,6 +465,8 @@ jarq_status jarq_prepare_hessian(const float *H, int din, int group_size, float 
         { ProfScope ps("symmetrize", st); e = launch_symmetrize(Hsrc, h->Hs, h->Hplanes, din, h->d_pad, nu2, st); ps.done(); count_launches(1); }
         if (e != cudaSuccess) { rc = cuda_fail(e); break; }
         { ProfScope ps("group_factor", st); e = launch_group_factor(h->Hs, h->Lf, h->L64, h->Rinv, din, group_size, h->dstatus, st); ps.done(); count_launches(1); }
+        if (e != cudaSuccess) { rc = cuda_fail(e); break; }
+        { ProfScope ps("slices", st); e = launch_slice_rinv(h->Rinv, h->rdig, h->rexp, din, group_size, st); ps.done(); count_launches(1); }
         if (e != cudaSuccess) { rc = cuda_fail(e); break; }
         // folded rows R_i^{-T} H[grp i, :] (double-float, temporary) -> digits
         if ((e = dalloc(&Ht_hi, dd)) != cudaSuccess) { rc = cuda_fail(e); break; }
@@ -652,7 +661,8 @@ jarq_status refine_impl(jarq_hessian *h, const float *W, float *S, uint8_t *Q, c
         rc = mu_projection(h, la.W, p, *mt, st);
         if (rc != JARQ_OK) return rc;
     }
-    RUN("ptilde", 1, launch_ptilde(w.Phi, w.Plo, h->Rinv, w.Pt_hi, w.Pt_lo, p, d, g, st));
+    RUN("ptilde", 2, launch_ptilde(w.mapPd, h->mapRi, w.Phi, w.Plo, w.wdig, w.wexp, h->rexp, w.Pt_hi,
+                                   w.Pt_lo, p, w.p_pad, d, h->d_pad, g, h->dstatus, st));
     for (int k = 1; k <= o.max_iters; ++k) {
         RUN("gram", 1, launch_tc_gram(w.mapC, h->mapD10, la.Q, la.Z, h->expo, w.active, w.gram, p,
                                       w.p_pad, d, h->d_pad, g, bits, h->dstatus, st));

@@ -74,10 +74,12 @@ struct Workspace {
     __half *cplane = nullptr;          // [p_pad][d_pad] codes c = q - z
     CUtensorMap mapR;            // tensor map of rplanes, 128 x 64 boxes
     CUtensorMap mapC;            // tensor map of cplane, 128 x 64 boxes
-    // target projection P = W H (once per call)
-    __nv_bfloat16 *wdig = nullptr;     // [4][p_pad][d_pad] integer digits of W
-    int *wexp = nullptr;               // [p][G] exponents of the digits of W
-    CUtensorMap mapWd;                 // tensor map of wdig, 128 x 64 boxes
+    // target projection P = W H (once per call); after it the same buffers
+    // hold the six digit planes of P for the folded projection
+    __nv_bfloat16 *wdig = nullptr;     // [6][p_pad][d_pad] integer digits of W (4) or P (6)
+    int *wexp = nullptr;               // [p][G] exponents of those digits
+    CUtensorMap mapWd;                 // tensor map of wdig's first 4 planes, 128 x 64 boxes
+    CUtensorMap mapPd;                 // tensor map of all 6 planes, 128 x 64 boxes
     float *Phi = nullptr;        // [p][d]  P = Phi + Plo (double-float)
     float *Plo = nullptr;        // [p][d]
     float *Pt_hi = nullptr;      // [p][d]  folded projection Pt_i = R_i^{-T} P_i
@@ -118,6 +120,11 @@ struct jarq_hessian {
     float *Lf = nullptr;          // [G][g][g] lower factor L_i = R_i^T, row-major
     double *L64 = nullptr;        // [G][g][g] the same in float64
     double *Rinv = nullptr;       // [G][g][g] R_i^{-1} (upper), row-major, float64
+    // R_i^{-1} in six base-2^8 digit planes, transposed per block (row i g + a,
+    // column b: digit of R_i^{-1}[b][a]), one exponent per group
+    __nv_bfloat16 *rdig = nullptr;     // [6][d][g]
+    int *rexp = nullptr;               // [G]
+    CUtensorMap mapRi;                 // tensor map of rdig, 64 x 64 boxes
     // folded rows Ht[grp i, :] = R_i^{-T} H[grp i, :] in the base-2^10 digit scheme
     __half *Htdig = nullptr;      // [4][d_pad][d_pad] fp16 digits, |digit| <= 512
     int *expoT = nullptr;         // [G][G] block exponents of Ht
@@ -198,8 +205,12 @@ cudaError_t launch_babai(const float *t_hi, const float *t_lo, const float *pt_h
                          uint8_t *Q, const int32_t *Z, ResidualView rv, const int *active,
                          int *accepted, int *status, int p, int g, int i, int qmax, float eps,
                          cudaStream_t s);
-cudaError_t launch_ptilde(const float *Phi, const float *Plo, const double *Rinv, float *out_hi,
-                          float *out_lo, int p, int d, int g, cudaStream_t s);
+cudaError_t launch_slice_rinv(const double *Rinv, __nv_bfloat16 *rdig, int *rexp, int d, int g,
+                              cudaStream_t s);
+cudaError_t launch_ptilde(const CUtensorMap &mapPd, const CUtensorMap &mapR, const float *Phi,
+                          const float *Plo, __nv_bfloat16 *pdig, int *pexp, const int *rexp,
+                          float *out_hi, float *out_lo, int p, int p_pad, int d, int d_pad, int g,
+                          int *status, cudaStream_t s);
 int target_splits(int p_pad, int g, int G);
 cudaError_t launch_tc_target(const CUtensorMap &mapC, const CUtensorMap &mapT, float *out_hi,
                              float *out_lo, const float *S, const int *expoT, const int *active,

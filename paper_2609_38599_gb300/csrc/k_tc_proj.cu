@@ -35,9 +35,15 @@ namespace {
 constexpr int kWDig = 4, kHDig = 6, kLevels = 6;
 constexpr int kTileA = 128 * 64 * 2;   // one W digit plane, 128 rows x 64 K
 constexpr int kTileB = 64 * 64 * 2;    // one H digit plane, 64 rows x 64 K
-constexpr int kStage = kWDig * kTileA + kHDig * kTileB;
-constexpr int kStages = 2;
-constexpr int kSmem = 1024 + kStages * kStage + 256;
+// WDIG row-side digit planes (4 for W, 6 for the double-float P of the folded
+// projection); DIAG: only the K block of the tile's own column group (the
+// block-diagonal right-hand side R_i^{-1}), one stage of 144 KB.
+template <int WDIG, bool DIAG>
+struct ProjCfg {
+    static constexpr int kStage = WDIG * kTileA + kHDig * kTileB;
+    static constexpr int kStages = DIAG ? 1 : 2;
+    static constexpr int kSmem = 1024 + kStages * kStage + 256;
+};
 // For a W digit t the H digit planes u are consecutive 64-row tiles and the
 // levels t + u consecutive 64-column blocks, so one MMA covers up to four
 // planes (N = 64 per plane).
@@ -47,7 +53,7 @@ constexpr int kGroupRows = 8;
 struct ProjArgs {
     float *Phi, *Plo;    // [p][d] double-float result
     const int *wexp;     // [p][G] row-group exponents of W
-    const int *hexp;     // [G][G] block exponents of H
+    const int *hexp;     // [G][G] block exponents of H ([G] in the diagonal form)
     int *status;
     int p, d, g, G, w_plane, h_plane;   // rows between digit planes in the two maps
 };
@@ -59,9 +65,11 @@ __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
     e = (a - (s - bb)) + (b - bb);
 }
 
+template <int WDIG, bool DIAG>
 __global__ void __launch_bounds__(320, 1)
     tc_proj_kernel(const __grid_constant__ CUtensorMap mapW, const __grid_constant__ CUtensorMap mapH,
                    ProjArgs a) {
+    constexpr int kStage = ProjCfg<WDIG, DIAG>::kStage, kStages = ProjCfg<WDIG, DIAG>::kStages;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint64_t *bars = (uint64_t *)(smem + kStages * kStage);
@@ -76,9 +84,11 @@ __global__ void __launch_bounds__(320, 1)
     const int j0 = (band * kGroupRows + in_band % rows_in_band) * 128;
     const int n0 = (in_band / rows_in_band) * 64;
     const int nkc = a.g / 64;               // K chunks per group
-    const int nseg = a.G;                   // K segments = groups
-    const int nchunks = nseg * nkc;
     const int hblk = n0 / a.g;              // column group of the tile (a 64-wide tile lies in one)
+    // K segments = groups; in the diagonal form only the tile's own group
+    // (none for a padding tile)
+    const int nseg = DIAG ? (hblk < a.G ? 1 : 0) : a.G;
+    const int nchunks = nseg * nkc;
 
     auto full = [&](int s) { return tc::smem_u32(bars + s); };
     auto empty = [&](int s) { return tc::smem_u32(bars + kStages + s); };
@@ -86,7 +96,7 @@ __global__ void __launch_bounds__(320, 1)
     const uint32_t aempty = tc::smem_u32(bars + 2 * kStages + 1);
     auto tileA = [&](int s, int t) { return tc::smem_u32(smem + s * kStage + t * kTileA); };
     auto tileB = [&](int s, int u) {
-        return tc::smem_u32(smem + s * kStage + kWDig * kTileA + u * kTileB);
+        return tc::smem_u32(smem + s * kStage + WDIG * kTileA + u * kTileB);
     };
 
     if (threadIdx.x == 0) {
@@ -121,14 +131,17 @@ __global__ void __launch_bounds__(320, 1)
                 *abort_flag = 1;
                 break;
             }
-            const int k = c * 64;
+            // K offsets in the two maps: the right-hand side of the diagonal
+            // form holds only the g columns of each group's block
+            const int kw = DIAG ? hblk * a.g + c * 64 : c * 64;
+            const int kh = c * 64;
             tc::mbar_expect_tx(full(s), kStage);
 #pragma unroll
-            for (int t = 0; t < kWDig; ++t)
-                tc::tma_load_2d(tileA(s, t), &mapW, full(s), k, t * a.w_plane + j0);
+            for (int t = 0; t < WDIG; ++t)
+                tc::tma_load_2d(tileA(s, t), &mapW, full(s), kw, t * a.w_plane + j0);
 #pragma unroll
             for (int u = 0; u < kHDig; ++u)
-                tc::tma_load_2d(tileB(s, u), &mapH, full(s), k, u * a.h_plane + n0);
+                tc::tma_load_2d(tileB(s, u), &mapH, full(s), kh, u * a.h_plane + n0);
             issued = c + 1;
         }
         // do not leave with copies in flight
@@ -153,7 +166,7 @@ __global__ void __launch_bounds__(320, 1)
 #pragma unroll
                 for (int sub = 0; sub < 4; ++sub) {
 #pragma unroll
-                    for (int t = 0; t < kWDig; ++t) {
+                    for (int t = 0; t < WDIG; ++t) {
                         const uint64_t ad = tc::sdesc_sw128(tileA(s, t)) + 2 * sub;
                         // the products of W digit t with H digits u < kLevels - t,
                         // in runs of at most four planes; t = 0 opens every level
@@ -185,11 +198,11 @@ __global__ void __launch_bounds__(320, 1)
         // exponents of the next group, loaded one group ahead
         const int *wrow = a.wexp + (size_t)min(row, a.p - 1) * a.G;
         const int hb = min(hblk, a.G - 1);
-        int ew_next = wrow[0], eh_next = a.hexp[hb];
+        int ew_next = DIAG ? wrow[hb] : wrow[0], eh_next = a.hexp[hb];
         for (int sg = 0; sg < nseg; ++sg) {
             const int ew = row < a.p ? ew_next : 0;
             const int eh = hblk < a.G ? eh_next : 0;
-            if (sg + 1 < nseg) {
+            if (!DIAG && sg + 1 < nseg) {
                 ew_next = wrow[sg + 1];
                 eh_next = a.hexp[(sg + 1) * a.G + hb];
             }
@@ -417,93 +430,114 @@ __global__ void mu_combine_kernel(float *__restrict__ Phi, float *__restrict__ P
     }
 }
 
-// Folded target projection Pt_j[grp i] = R_i^{-T} P_j[grp i], i.e.
-// Pt[j, i g + a] = sum_{b <= a} Rinv_i[b][a] P[j, i g + b], in double-float
-// from the float64 inverse and the double-float P.  One CTA per (64 rows,
-// group i); Rinv_i and the rows' P slice in shared memory.
-constexpr int kPtRows = 64;
-
-__global__ void __launch_bounds__(512) ptilde_kernel(const float *__restrict__ Phi,
-                                                     const float *__restrict__ Plo,
-                                                     const double *__restrict__ Rinv,
-                                                     float *__restrict__ out_hi,
-                                                     float *__restrict__ out_lo, int p, int d,
-                                                     int g) {
-    extern __shared__ float psm[];
-    float *rh = psm;                   // [g][g] Rinv[b][a] at b * g + a
-    float *rl = rh + g * g;
-    float *ph = rl + g * g;            // [kPtRows][g]
-    float *pl = ph + kPtRows * g;
-    const int i = blockIdx.y, r0 = blockIdx.x * kPtRows;
-    const int tid = threadIdx.x;
-    const double *Ri = Rinv + (size_t)i * g * g;
-    for (int idx = tid; idx < g * g; idx += blockDim.x) {
-        const double v = Ri[idx];
-        const float hv = (float)v;
-        rh[idx] = hv;
-        rl[idx] = (float)(v - (double)hv);
+// Digits of the double-float P for the folded projection: per (row, group)
+// the exponent e with max |P| < 2^e, and six balanced base-256 digits of
+// P 2^(7-e) (|digit| <= 128, exact in bf16), taken from the float pair
+// (xh, xl) = (Phi, Plo) 2^(7-e) with exact float operations: the digit is
+// rint(xh), and the remainder (xh - digit) + xl is renormalised by an exact
+// two-sum before the next digit.  Six digits hold P to 2^-48 of its group
+// maximum (the pair itself carries about 48 bits).
+__global__ void slice_df_rows_kernel(const float *__restrict__ Phi, const float *__restrict__ Plo,
+                                     __nv_bfloat16 *__restrict__ planes, int *__restrict__ pexp,
+                                     int p, int d, int d_pad, int p_pad, int g) {
+    const int G = d / g;
+    const long long warp = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (warp >= (long long)p * G) return;
+    const int j = (int)(warp / G), h = (int)(warp % G);
+    const size_t src = (size_t)j * d + (size_t)h * g;
+    float mx = 0.f;
+    for (int m = lane; m < g; m += 32) mx = fmaxf(mx, fabsf(Phi[src + m]));
+    for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    int e = 0;
+    if (mx > 0.f) frexpf(mx, &e);
+    if (lane == 0) pexp[(size_t)j * G + h] = e;
+    const size_t plane = (size_t)p_pad * d_pad;
+    for (int m = lane; m < g; m += 32) {
+        float xh = ldexpf(Phi[src + m], 7 - e), xl = ldexpf(Plo[src + m], 7 - e);
+        const size_t off = (size_t)j * d_pad + (size_t)h * g + m;
+#pragma unroll
+        for (int t = 0; t < kHDig; ++t) {
+            const float dg = rintf(xh);
+            planes[t * plane + off] = __float2bfloat16_rn(dg);
+            float s2, e2;
+            two_sum(xh - dg, xl, s2, e2);
+            xh = s2 * 256.f;
+            xl = e2 * 256.f;
+        }
     }
-    for (int idx = tid; idx < kPtRows * g; idx += blockDim.x) {
-        const int jj = idx / g, b = idx % g;
-        const bool in = r0 + jj < p;
-        const size_t o = (size_t)(r0 + jj) * d + (size_t)i * g + b;
-        ph[idx] = in ? Phi[o] : 0.f;
-        pl[idx] = in ? Plo[o] : 0.f;
+}
+
+// Digits of the group inverses for the folded projection (once per prepared
+// Hessian): plane u, row i g + a, column b holds digit u of R_i^{-1}[b][a]
+// (zero below the diagonal), so that the 64 x 64 tiles of the projection
+// kernel read the transposed block; exponent E_i with max |R_i^{-1}| < 2^E_i,
+// six balanced base-256 digits of R_i^{-1} 2^(7-E_i) in float64.
+__global__ void slice_rinv_kernel(const double *__restrict__ Rinv, __nv_bfloat16 *__restrict__ rdig,
+                                  int *__restrict__ rexp, int d, int g) {
+    __shared__ double red[32];
+    const int i = blockIdx.x;
+    const double *Ri = Rinv + (size_t)i * g * g;
+    double mx = 0.0;
+    for (int idx = threadIdx.x; idx < g * g; idx += blockDim.x) mx = fmax(mx, fabs(Ri[idx]));
+    for (int o = 16; o; o >>= 1) mx = fmax(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = mx;
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        mx = threadIdx.x < (blockDim.x >> 5) ? red[threadIdx.x] : 0.0;
+        for (int o = 16; o; o >>= 1) mx = fmax(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+        if (threadIdx.x == 0) red[0] = mx;
     }
     __syncthreads();
-    // each thread: the column pair (a, g-1-a), so that every thread (and every
-    // warp, hence every scheduler) does about the same g+1 steps of the
-    // triangle, and kRowsPer rows as independent chains
-    constexpr int kRowsPer = 8;
-    const int npairs = g / 2, pair = tid % npairs, rstep = (blockDim.x / npairs) * kRowsPer;
-    for (int jb = (tid / npairs) * kRowsPer; jb < kPtRows; jb += rstep) {
-#pragma unroll 1
-        for (int side = 0; side < 2; ++side) {
-            const int a = side == 0 ? pair : g - 1 - pair;
-            float sh[kRowsPer], sl[kRowsPer];
+    mx = red[0];
+    int E = 0;
+    if (mx > 0.0) frexp(mx, &E);
+    if (threadIdx.x == 0) rexp[i] = E;
+    const size_t plane = (size_t)d * g;
+    for (int idx = threadIdx.x; idx < g * g; idx += blockDim.x) {
+        const int a = idx / g, b = idx % g;
+        double x = b <= a ? ldexp(Ri[(size_t)b * g + a], 7 - E) : 0.0;
+        const size_t off = ((size_t)i * g + a) * g + b;
 #pragma unroll
-            for (int r = 0; r < kRowsPer; ++r) {
-                sh[r] = 0.f;
-                sl[r] = 0.f;
-            }
-            for (int b = 0; b <= a; ++b) {
-                const float xh = rh[b * g + a], xl = rl[b * g + a];
-#pragma unroll
-                for (int r = 0; r < kRowsPer; ++r) {
-                    const float yh = ph[(jb + r) * g + b], yl = pl[(jb + r) * g + b];
-                    const float m = xh * yh;
-                    float e = fmaf(xh, yh, -m);
-                    e = fmaf(xh, yl, fmaf(xl, yh, e));
-                    float s2, e2;
-                    two_sum(sh[r], m, s2, e2);
-                    sh[r] = s2;
-                    sl[r] += e2 + e;
-                }
-            }
-#pragma unroll
-            for (int r = 0; r < kRowsPer; ++r) {
-                if (r0 + jb + r < p) {
-                    float s2, e2;
-                    two_sum(sh[r], sl[r], s2, e2);
-                    const size_t o = (size_t)(r0 + jb + r) * d + (size_t)i * g + a;
-                    out_hi[o] = s2;
-                    out_lo[o] = e2;
-                }
-            }
+        for (int u = 0; u < kHDig; ++u) {
+            const double dg = rint(x);
+            rdig[u * plane + off] = __float2bfloat16_rn((float)dg);
+            x = (x - dg) * 256.0;
         }
     }
 }
 
 }  // namespace
 
-cudaError_t launch_ptilde(const float *Phi, const float *Plo, const double *Rinv, float *out_hi,
-                          float *out_lo, int p, int d, int g, cudaStream_t s) {
-    const size_t smem = ((size_t)2 * g * g + (size_t)2 * kPtRows * g) * sizeof(float);
-    cudaError_t e = cudaFuncSetAttribute(ptilde_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
+cudaError_t launch_slice_rinv(const double *Rinv, __nv_bfloat16 *rdig, int *rexp, int d, int g,
+                              cudaStream_t s) {
+    slice_rinv_kernel<<<d / g, 256, 0, s>>>(Rinv, rdig, rexp, d, g);
+    return cudaGetLastError();
+}
+
+// Pt = the folded projection, Pt[j, i g + a] = sum_{b <= a} R_i^{-1}[b][a] P[j, i g + b]:
+// the six digit planes of P (into the row-digit workspace) and the
+// block-diagonal product with the digits of R_i^{-1} on the tensor cores.
+cudaError_t launch_ptilde(const CUtensorMap &mapPd, const CUtensorMap &mapR, const float *Phi,
+                          const float *Plo, __nv_bfloat16 *pdig, int *pexp, const int *rexp,
+                          float *out_hi, float *out_lo, int p, int p_pad, int d, int d_pad, int g,
+                          int *status, cudaStream_t s) {
+    const long long warps = (long long)p * (d / g);
+    slice_df_rows_kernel<<<(unsigned)((warps * 32 + 255) / 256), 256, 0, s>>>(
+        Phi, Plo, pdig, pexp, p, d, d_pad, p_pad, g);
+    cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    dim3 grid((p + kPtRows - 1) / kPtRows, d / g);
-    ptilde_kernel<<<grid, 512, smem, s>>>(Phi, Plo, Rinv, out_hi, out_lo, p, d, g);
+    using C = ProjCfg<kHDig, true>;
+    static bool attr_set = false;
+    if (!attr_set) {
+        e = cudaFuncSetAttribute(tc_proj_kernel<kHDig, true>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    ProjArgs a{out_hi, out_lo, pexp, rexp, status, p, d, g, d / g, p_pad, d};
+    dim3 grid(p_pad / 128, d_pad / 64, 1);
+    tc_proj_kernel<kHDig, true><<<grid, 320, C::kSmem, s>>>(mapPd, mapR, a);
     return cudaGetLastError();
 }
 
@@ -518,16 +552,17 @@ cudaError_t launch_slice_rows(const float *W, __nv_bfloat16 *planes, int *wexp, 
 cudaError_t launch_tc_proj(const CUtensorMap &mapW, const CUtensorMap &mapH, float *Phi,
                            float *Plo, const int *wexp, const int *hexp, int p, int p_pad, int d,
                            int d_pad, int g, int *status, cudaStream_t s) {
+    using C = ProjCfg<kWDig, false>;
     static bool attr_set = false;
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(tc_proj_kernel,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
+        cudaError_t e = cudaFuncSetAttribute(tc_proj_kernel<kWDig, false>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
     ProjArgs a{Phi, Plo, wexp, hexp, status, p, d, g, d / g, p_pad, d_pad};
     dim3 grid(p_pad / 128, d_pad / 64, 1);
-    tc_proj_kernel<<<grid, 320, kSmem, s>>>(mapW, mapH, a);
+    tc_proj_kernel<kWDig, false><<<grid, 320, C::kSmem, s>>>(mapW, mapH, a);
     return cudaGetLastError();
 }
 
