@@ -76,19 +76,38 @@ __global__ void __launch_bounds__(320, 1)
     uint32_t *tmem_slot = (uint32_t *)(bars + 2 * kStages + 2);
     volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    // grouped tile order: bands of kGroupRows row tiles sweep all column tiles
-    const int lin = blockIdx.y * gridDim.x + blockIdx.x;
-    const int per_band = kGroupRows * gridDim.y;
-    const int band = lin / per_band, in_band = lin % per_band;
-    const int rows_in_band = min(kGroupRows, (int)gridDim.x - band * kGroupRows);
-    const int j0 = (band * kGroupRows + in_band % rows_in_band) * 128;
-    const int n0 = (in_band / rows_in_band) * 64;
     const int nkc = a.g / 64;               // K chunks per group
-    const int hblk = n0 / a.g;              // column group of the tile (a 64-wide tile lies in one)
-    // K segments = groups; in the diagonal form only the tile's own group
-    // (none for a padding tile)
-    const int nseg = DIAG ? (hblk < a.G ? 1 : 0) : a.G;
+    // General form: one 128 x 64 tile per CTA in grouped order (bands of
+    // kGroupRows row tiles sweep all column tiles), one segment per group of
+    // K.  Diagonal form: the CTA loops over tiles, item blockIdx.x + v gridDim.x
+    // of (row tiles) x (d / 64 column tiles), one segment each: the K block of
+    // the tile's own column group.
+    int gj0 = 0, gn0 = 0;
+    if (!DIAG) {
+        const int lin = blockIdx.y * gridDim.x + blockIdx.x;
+        const int per_band = kGroupRows * gridDim.y;
+        const int band = lin / per_band, in_band = lin % per_band;
+        const int rows_in_band = min(kGroupRows, (int)gridDim.x - band * kGroupRows);
+        gj0 = (band * kGroupRows + in_band % rows_in_band) * 128;
+        gn0 = (in_band / rows_in_band) * 64;
+    }
+    const int nct = a.d / 64;
+    const int nitems = DIAG ? ((a.p + 127) / 128) * nct : 1;
+    const int nseg = DIAG ? ((int)blockIdx.x < nitems ? (nitems - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0)
+                          : a.G;
     const int nchunks = nseg * nkc;
+    // tile (first row, first column) of segment v; a 64-wide tile lies in
+    // one column group n0 / g
+    auto tile_of = [&](int v, int &j0, int &n0) {
+        if (DIAG) {
+            const int it = (int)blockIdx.x + v * (int)gridDim.x;
+            j0 = (it / nct) * 128;
+            n0 = (it % nct) * 64;
+        } else {
+            j0 = gj0;
+            n0 = gn0;
+        }
+    };
 
     auto full = [&](int s) { return tc::smem_u32(bars + s); };
     auto empty = [&](int s) { return tc::smem_u32(bars + kStages + s); };
@@ -131,10 +150,13 @@ __global__ void __launch_bounds__(320, 1)
                 *abort_flag = 1;
                 break;
             }
+            const int v = c / nkc, kc = c % nkc;
+            int j0, n0;
+            tile_of(v, j0, n0);
             // K offsets in the two maps: the right-hand side of the diagonal
             // form holds only the g columns of each group's block
-            const int kw = DIAG ? hblk * a.g + c * 64 : c * 64;
-            const int kh = c * 64;
+            const int kw = DIAG ? (n0 / a.g) * a.g + kc * 64 : c * 64;
+            const int kh = DIAG ? kc * 64 : c * 64;
             tc::mbar_expect_tx(full(s), kStage);
 #pragma unroll
             for (int t = 0; t < WDIG; ++t)
@@ -185,82 +207,180 @@ __global__ void __launch_bounds__(320, 1)
         }
     } else if (warp >= 2) {
         // ---------------- drain: levels -> double-float per group -> accumulator
-        const int q = warp & 3, half = (warp - 2) >> 2;
-        const int row = j0 + 32 * q + lane;
-        float hi[32], lo[32];
+        if constexpr (DIAG) {
+            // diagonal form: a tile per segment, written when it completes
+            const int q = warp & 3, half = (warp - 2) >> 2;
+            float hi[32], lo[32];
 #pragma unroll
-        for (int e = 0; e < 32; ++e) {
-            hi[e] = 0.f;
-            lo[e] = 0.f;
-        }
-        bool ok = true;
-        const uint32_t base = tmem + ((uint32_t)(32 * q) << 16) + half * 32;
-        // exponents of the next group, loaded one group ahead
-        const int *wrow = a.wexp + (size_t)min(row, a.p - 1) * a.G;
-        const int hb = min(hblk, a.G - 1);
-        int ew_next = DIAG ? wrow[hb] : wrow[0], eh_next = a.hexp[hb];
-        for (int sg = 0; sg < nseg; ++sg) {
-            const int ew = row < a.p ? ew_next : 0;
-            const int eh = hblk < a.G ? eh_next : 0;
-            if (!DIAG && sg + 1 < nseg) {
-                ew_next = wrow[sg + 1];
-                eh_next = a.hexp[(sg + 1) * a.G + hb];
+            for (int e = 0; e < 32; ++e) {
+                hi[e] = 0.f;
+                lo[e] = 0.f;
             }
-            bool w = tc::mbar_wait(afull, sg & 1);
-            w = __shfl_sync(0xffffffffu, w && !*abort_flag, 0);
-            tc::tc_fence_after();
-            if (!w) {
-                ok = false;
-                *abort_flag = 1;
-                break;
-            }
-            const float scale = ldexpf(1.0f, ew + eh - 14);
-            // value of the group = sum_l L_l 2^(-8 l), as (vh, vl), 32 columns
-            float vh[32], vl[32];
-#pragma unroll
-            for (int l = 0; l < kLevels; ++l) {
-                uint32_t x[32];
-                tc::tmem_ld32(base + l * 64, x);
-                tc::tmem_wait_ld();
-                if (l == kLevels - 1) {
-                    // every level is in registers: hand the columns back
-                    tc::tc_fence_before();
-                    __syncwarp();
-                    if (lane == 0) tc::mbar_arrive(aempty);
+            bool ok = true;
+            const uint32_t base = tmem + ((uint32_t)(32 * q) << 16) + half * 32;
+            // exponents of this thread's row and segment v: W's (row, K group)
+            // and H's block (K group, column group); loaded one segment ahead
+            auto seg_exp = [&](int v, int &ew, int &eh) {
+                int j0, n0;
+                tile_of(v, j0, n0);
+                const int row = j0 + 32 * q + lane, hb = n0 / a.g, kg = DIAG ? hb : v;
+                ew = row < a.p ? a.wexp[(size_t)row * a.G + kg] : 0;
+                eh = hb < a.G ? a.hexp[DIAG ? hb : kg * a.G + hb] : 0;
+            };
+            int ew_next = 0, eh_next = 0;
+            if (nseg > 0) seg_exp(0, ew_next, eh_next);
+            for (int sg = 0; sg < nseg; ++sg) {
+                const int ew = ew_next, eh = eh_next;
+                if (sg + 1 < nseg) seg_exp(sg + 1, ew_next, eh_next);
+                bool w = tc::mbar_wait(afull, sg & 1);
+                w = __shfl_sync(0xffffffffu, w && !*abort_flag, 0);
+                tc::tc_fence_after();
+                if (!w) {
+                    ok = false;
+                    *abort_flag = 1;
+                    break;
                 }
-                const float f = ldexpf(1.0f, -8 * l);
+                const float scale = ldexpf(1.0f, ew + eh - 14);
+                // value of the group = sum_l L_l 2^(-8 l), as (vh, vl), 32 columns
+                float vh[32], vl[32];
+#pragma unroll
+                for (int l = 0; l < kLevels; ++l) {
+                    uint32_t x[32];
+                    tc::tmem_ld32(base + l * 64, x);
+                    tc::tmem_wait_ld();
+                    if (l == kLevels - 1) {
+                        // every level is in registers: hand the columns back
+                        tc::tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) tc::mbar_arrive(aempty);
+                    }
+                    const float f = ldexpf(1.0f, -8 * l);
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) {
+                        const float v = __uint_as_float(x[e]) * f;   // exact (power of two)
+                        if (l == 0) {
+                            vh[e] = v;
+                            vl[e] = 0.f;
+                        } else {
+                            float s2, e2;
+                            two_sum(vh[e], v, s2, e2);
+                            vh[e] = s2;
+                            vl[e] += e2;
+                        }
+                    }
+                }
 #pragma unroll
                 for (int e = 0; e < 32; ++e) {
-                    const float v = __uint_as_float(x[e]) * f;   // exact (power of two)
-                    if (l == 0) {
-                        vh[e] = v;
-                        vl[e] = 0.f;
-                    } else {
-                        float s2, e2;
-                        two_sum(vh[e], v, s2, e2);
-                        vh[e] = s2;
-                        vl[e] += e2;
+                    float s2, e2;
+                    two_sum(hi[e], vh[e] * scale, s2, e2);
+                    hi[e] = s2;
+                    lo[e] += e2 + vl[e] * scale;
+                }
+                // the tile is complete after its last segment (every segment in
+                // the diagonal form)
+                if (DIAG || sg + 1 == nseg) {
+                    int j0, n0;
+                    tile_of(sg, j0, n0);
+                    const int row = j0 + 32 * q + lane, ncol = n0 + half * 32;
+                    if (row < a.p) {
+#pragma unroll
+                        for (int e = 0; e < 32; ++e) {
+                            const int col = ncol + e;
+                            if (col < a.d) {
+                                float s2, e2;
+                                two_sum(hi[e], lo[e], s2, e2);
+                                a.Phi[(size_t)row * a.d + col] = s2;
+                                a.Plo[(size_t)row * a.d + col] = e2;
+                            }
+                        }
+                    }
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) {
+                        hi[e] = 0.f;
+                        lo[e] = 0.f;
                     }
                 }
             }
+            (void)ok;
+        } else {
+            const int q = warp & 3, half = (warp - 2) >> 2;
+            const int j0 = gj0, n0 = gn0, hblk = n0 / a.g;
+            const int row = j0 + 32 * q + lane;
+            float hi[32], lo[32];
 #pragma unroll
             for (int e = 0; e < 32; ++e) {
-                float s2, e2;
-                two_sum(hi[e], vh[e] * scale, s2, e2);
-                hi[e] = s2;
-                lo[e] += e2 + vl[e] * scale;
+                hi[e] = 0.f;
+                lo[e] = 0.f;
             }
-        }
-        if (ok && row < a.p) {
-            const int ncol = n0 + half * 32;
+            bool ok = true;
+            const uint32_t base = tmem + ((uint32_t)(32 * q) << 16) + half * 32;
+            // exponents of the next group, loaded one group ahead
+            const int *wrow = a.wexp + (size_t)min(row, a.p - 1) * a.G;
+            const int hb = min(hblk, a.G - 1);
+            int ew_next = wrow[0], eh_next = a.hexp[hb];
+            for (int sg = 0; sg < nseg; ++sg) {
+                const int ew = row < a.p ? ew_next : 0;
+                const int eh = hblk < a.G ? eh_next : 0;
+                if (sg + 1 < nseg) {
+                    ew_next = wrow[sg + 1];
+                    eh_next = a.hexp[(sg + 1) * a.G + hb];
+                }
+                bool w = tc::mbar_wait(afull, sg & 1);
+                w = __shfl_sync(0xffffffffu, w && !*abort_flag, 0);
+                tc::tc_fence_after();
+                if (!w) {
+                    ok = false;
+                    *abort_flag = 1;
+                    break;
+                }
+                const float scale = ldexpf(1.0f, ew + eh - 14);
+                // value of the group = sum_l L_l 2^(-8 l), as (vh, vl), 32 columns
+                float vh[32], vl[32];
 #pragma unroll
-            for (int e = 0; e < 32; ++e) {
-                const int col = ncol + e;
-                if (col < a.d) {
+                for (int l = 0; l < kLevels; ++l) {
+                    uint32_t x[32];
+                    tc::tmem_ld32(base + l * 64, x);
+                    tc::tmem_wait_ld();
+                    if (l == kLevels - 1) {
+                        // every level is in registers: hand the columns back
+                        tc::tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) tc::mbar_arrive(aempty);
+                    }
+                    const float f = ldexpf(1.0f, -8 * l);
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) {
+                        const float v = __uint_as_float(x[e]) * f;   // exact (power of two)
+                        if (l == 0) {
+                            vh[e] = v;
+                            vl[e] = 0.f;
+                        } else {
+                            float s2, e2;
+                            two_sum(vh[e], v, s2, e2);
+                            vh[e] = s2;
+                            vl[e] += e2;
+                        }
+                    }
+                }
+#pragma unroll
+                for (int e = 0; e < 32; ++e) {
                     float s2, e2;
-                    two_sum(hi[e], lo[e], s2, e2);
-                    a.Phi[(size_t)row * a.d + col] = s2;
-                    a.Plo[(size_t)row * a.d + col] = e2;
+                    two_sum(hi[e], vh[e] * scale, s2, e2);
+                    hi[e] = s2;
+                    lo[e] += e2 + vl[e] * scale;
+                }
+            }
+            if (ok && row < a.p) {
+                const int ncol = n0 + half * 32;
+#pragma unroll
+                for (int e = 0; e < 32; ++e) {
+                    const int col = ncol + e;
+                    if (col < a.d) {
+                        float s2, e2;
+                        two_sum(hi[e], lo[e], s2, e2);
+                        a.Phi[(size_t)row * a.d + col] = s2;
+                        a.Plo[(size_t)row * a.d + col] = e2;
+                    }
                 }
             }
         }
@@ -536,8 +656,11 @@ cudaError_t launch_ptilde(const CUtensorMap &mapPd, const CUtensorMap &mapR, con
         attr_set = true;
     }
     ProjArgs a{out_hi, out_lo, pexp, rexp, status, p, d, g, d / g, p_pad, d};
-    dim3 grid(p_pad / 128, d_pad / 64, 1);
-    tc_proj_kernel<kHDig, true><<<grid, 320, C::kSmem, s>>>(mapPd, mapR, a);
+    // persistent: one CTA per SM over the (p_pad / 128) x (d / 64) tiles
+    (void)d_pad;
+    const int items = (p_pad / 128) * (d / 64);
+    const int ctas = items < num_sms() ? items : num_sms();
+    tc_proj_kernel<kHDig, true><<<dim3(ctas, 1, 1), 320, C::kSmem, s>>>(mapPd, mapR, a);
     return cudaGetLastError();
 }
 
