@@ -46,8 +46,8 @@ TRAFFIC = {
     "target": ("k_tc_target.cu", "18ee82cb694f", 38.299e6 + 0.152e6),
     "babai": ("k_babai.cu", "d2d96a20da85", 14.274e6 + 0.001536e6),
     "gram": ("k_tc_gram.cu", "c839a427ea94", 164.246e6 + 27.889664e6),
-    "proj": ("k_tc_proj.cu", "7fe129ae0adf", 1374.566e6 + 156.723968e6),
-    "ptilde": ("k_tc_proj.cu", "7fe129ae0adf", 138.449e6 + 90.958080e6),
+    "proj": ("k_tc_proj.cu", "b46541dbdbb2", 1370.069e6 + 156.471e6),
+    "ptilde": ("k_tc_proj.cu", "b46541dbdbb2", 134.248e6 + 150.687e6 + 222.887e6 + 103.208e6),
     "scale_solve": ("k_solve.cu", "f3195c119d2c", 35.257e6 + 0.0),
     # profiles/ncu_syrk_attn_in_4096_n32768.md, scaled from 32768 to 262144 tokens
     "syrk": ("k_syrk.cu", "3896afedc783", 8 * 537.171e6 + 40.712e6),
