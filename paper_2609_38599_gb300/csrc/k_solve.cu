@@ -243,6 +243,314 @@ __global__ void scale_solve_kernel(SolveArgs a) {
     }
 }
 
+
+// ---------------------------------------------------------------------------
+// Register-resident solve for G <= 32 (the g = 128 layers of 4096 inputs).
+//
+// Same steps, same decisions, no bulk float64: on GB300 float64 runs at
+// about 1/64 of the float32 rate, so the dot products of the gradient, the
+// refinement residuals and the objective are done in double-float (pairs of
+// float32 with error-free products and sums, about 48 significant bits).
+// Lane l owns row l of the Gram matrix (= column l: it is exactly
+// symmetric) as a double-float pair per entry, split from the float64 with
+// integer operations.  The float32 Cholesky keeps row l in registers and
+// broadcasts the column of each step with shuffles: the same operations in
+// the same order as warp_cholesky, so the factor (and the ridge decision)
+// is bit-identical.  The triangular solves multiply by the reciprocal of
+// the pivots; the float64-accurate refinement makes the stored scales
+// independent of that rounding.
+// ---------------------------------------------------------------------------
+
+struct DF {
+    float h, l;
+};
+
+__device__ __forceinline__ DF df_two_sum(float a, float b) {
+    const float s = __fadd_rn(a, b);
+    const float bb = __fsub_rn(s, a);
+    const float e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+    return {s, e};
+}
+
+// (h, l) += x * y: the exact product x y = p + pe, p added by two_sum
+__device__ __forceinline__ void df_add_prod(DF &a, float x, float y) {
+    const float p = __fmul_rn(x, y);
+    const float pe = __fmaf_rn(x, y, -p);
+    const DF s = df_two_sum(a.h, p);
+    a.h = s.h;
+    a.l = __fadd_rn(a.l, __fadd_rn(s.l, pe));
+}
+
+__device__ __forceinline__ DF df_add(DF a, DF b) {
+    const DF s = df_two_sum(a.h, b.h);
+    return {s.h, __fadd_rn(s.l, __fadd_rn(a.l, b.l))};
+}
+
+__device__ __forceinline__ DF df_neg(DF a) { return {-a.h, -a.l}; }
+
+__device__ __forceinline__ DF df_warp_sum(DF a) {
+    // two_sum is exact, so both lanes of a butterfly pair form the same value
+    for (int o = 16; o; o >>= 1) {
+        const DF b{__shfl_xor_sync(0xffffffffu, a.h, o), __shfl_xor_sync(0xffffffffu, a.l, o)};
+        a = df_add(a, b);
+    }
+    return a;
+}
+
+__device__ __forceinline__ double df_to_double(DF a) { return (double)a.h + (double)a.l; }
+
+// x = hi + lo with hi = x rounded to float32 (nearest, ties to even) and
+// lo = x - hi rounded to float32, by integer operations on the bits of x
+// for 2^-74 <= |x| < 2^126 (zero, tiny, huge and non-finite values take
+// the float64 conversions).
+__device__ __forceinline__ DF split_double(double x) {
+    const unsigned long long bits = (unsigned long long)__double_as_longlong(x);
+    const unsigned long long u = bits & 0x7FFFFFFFFFFFFFFFull;
+    const int ex = (int)(u >> 52);
+    if (ex < 949 || ex > 1148) {
+        const float h = __double2float_rn(x);
+        return {h, __double2float_rn(x - (double)h)};
+    }
+    // keep the top 24 significant bits, round to nearest even; a carry out
+    // of the mantissa moves into the exponent field, which is still exact
+    unsigned long long keep = u >> 29;
+    const unsigned long long rem = u & ((1ull << 29) - 1);
+    keep += (rem > (1ull << 28)) || (rem == (1ull << 28) && (keep & 1ull));
+    // float32 bits: re-bias the exponent from 1023 to 127
+    const uint32_t hb = (uint32_t)(keep - (896ull << 23));
+    // x - hi in units of x's last place (|r| <= 2^28), times 2^(ex - 1075)
+    const int r = (int)(long long)(u - (keep << 29));
+    const float unit = __uint_as_float((uint32_t)(ex - 1075 + 127) << 23);
+    float h = __uint_as_float(hb), l = __fmul_rn(__int2float_rn(r), unit);
+    if (bits >> 63) {
+        h = -h;
+        l = -l;
+    }
+    return {h, l};
+}
+
+// In-place lower Cholesky with lane a holding row a in A[]; the operations
+// and their order are those of warp_cholesky.
+__device__ __forceinline__ bool reg_cholesky(float (&A)[32], int G, float thr) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int k = 0; k < 32; ++k) {
+        if (k < G) {
+            const float piv = __shfl_sync(0xffffffffu, A[k], k);
+            if (!(piv > thr) || !isfinite(piv)) return false;   // warp-uniform
+            const float lkk = sqrtf(piv);
+            float lak = 0.f;
+            if (lane > k) lak = A[k] / lkk;
+            if (lane == k) A[k] = lkk;
+            if (lane > k) A[k] = lak;
+#pragma unroll
+            for (int b = k + 1; b < 32; ++b) {
+                const float lbk = __shfl_sync(0xffffffffu, lak, b);
+                if (lane >= b) A[b] = fmaf(-lak, lbk, A[b]);
+            }
+        }
+    }
+    return true;
+}
+
+// y <- (L L^T)^{-1} y with lane a holding y_a; L row-major in Ls (stride
+// 33), dinv = 1 / L_aa.
+__device__ __forceinline__ float reg_chol_solve(const float *Ls, int G, float dinv, float y) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int k = 0; k < 32; ++k) {
+        if (k < G) {
+            const float yk = __shfl_sync(0xffffffffu, __fmul_rn(y, dinv), k);
+            if (lane == k) y = yk;
+            if (lane > k) y = fmaf(-Ls[lane * 33 + k], yk, y);
+        }
+    }
+#pragma unroll
+    for (int k = 31; k >= 0; --k) {
+        if (k < G) {
+            const float xk = __shfl_sync(0xffffffffu, __fmul_rn(y, dinv), k);
+            if (lane == k) y = xk;
+            if (lane < k) y = fmaf(-Ls[k * 33 + lane], xk, y);
+        }
+    }
+    return y;
+}
+
+constexpr int kSmallWarps = 4;   // rows (warps) per block of the G <= 32 kernel
+
+__global__ void __launch_bounds__(32 * kSmallWarps) scale_solve_small_kernel(SolveArgs a) {
+    __shared__ float Lsh[kSmallWarps][32 * 33];
+    const int G = a.d / a.g;
+    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int j = blockIdx.x * kSmallWarps + w;
+    if (j >= a.p || (!a.eval_only && !a.active[j])) return;  // warp-uniform
+    const bool own = lane < G;
+    const double *gj = a.gram + (size_t)j * G * G;
+    const float so = own ? a.S[(size_t)j * G + lane] : 0.f;
+    const DF rh = split_double(own ? a.rhs[(size_t)j * G + lane] : 0.0);
+    // row `lane` of the Gram matrix, read column-wise (coalesced) by symmetry
+    DF gr[32];
+#pragma unroll
+    for (int c = 0; c < 32; ++c) gr[c] = split_double((own && c < G) ? gj[(size_t)c * G + lane] : 0.0);
+
+    // gradient g = rhs - Gram s_old and F(s_old) = wHw - s_old^T (rhs + g)
+    DF acc{0.f, 0.f};
+#pragma unroll
+    for (int c = 0; c < 32; ++c) {
+        if (c < G) {
+            const float sc = __shfl_sync(0xffffffffu, so, c);
+            df_add_prod(acc, gr[c].h, sc);
+            acc.l = __fmaf_rn(gr[c].l, sc, acc.l);
+        }
+    }
+    const DF gd = df_add(rh, df_neg(acc));
+    const bool bfin = isfinite(gd.h) && isfinite(gd.l);
+    DF fs{0.f, 0.f};
+    {
+        const DF t = df_add(rh, gd);
+        df_add_prod(fs, so, t.h);
+        fs.l = __fmaf_rn(so, t.l, fs.l);
+    }
+    const double F_old = a.wHw[j] - df_to_double(df_warp_sum(fs));
+    if (a.L_out && lane == 0) a.L_out[j] = F_old;
+    if (a.eval_only) return;
+    if (a.o.fixed_grid) {
+        bool stop = false;
+        if (a.o.early_stop && a.k >= 2) {
+            const double dec = a.L_prev[j] - F_old;
+            const double den = fmax(fabs(a.L_prev[j]), (double)a.o.eps);
+            stop = (dec / den <= (double)a.o.tau_rel) || (fabs(dec) <= (double)a.o.tau_abs);
+        }
+        if (lane == 0) {
+            a.L_prev[j] = F_old;
+            a.iters[j] = a.k;
+            if (stop) a.active[j] = 0;
+        }
+        return;
+    }
+
+    // float32 factor of the Gram matrix (entries rounded to nearest, as a
+    // float64 -> float32 conversion does), with the ridge retry
+    float A[32];
+    bool finite = true;
+    float diag = 0.f;
+#pragma unroll
+    for (int c = 0; c < 32; ++c) {
+        A[c] = gr[c].h;
+        finite &= (bool)isfinite(A[c]);
+        if (c == lane) diag = A[c];
+    }
+    finite = __all_sync(0xffffffffu, finite);
+    const float md = warp_max(own ? diag : 0.f);
+    bool ok = finite && reg_cholesky(A, G, a.o.rcond * fmaxf(md, a.o.eps));
+    int used_ridge = 0;
+    if (!ok) {
+        used_ridge = 1;
+#pragma unroll
+        for (int c = 0; c < 32; ++c) A[c] = (c == lane) ? gr[c].h + a.o.ridge : gr[c].h;
+        ok = reg_cholesky(A, G, 0.f);
+    }
+    ok = ok && __all_sync(0xffffffffu, bfin);
+    auto fail = [&]() {
+        if (lane == 0) {
+            a.ridge[j] += used_ridge;
+            a.rstat[j] = JARQ_ERR_NUMERICAL;
+            a.active[j] = 0;
+            atomicOr(a.status, ST_NUMERICAL);
+        }
+    };
+    if (!ok) {
+        fail();
+        return;
+    }
+    float *Ls = Lsh[w];
+    float ldiag = 1.f;
+#pragma unroll
+    for (int c = 0; c < 32; ++c) {
+        Ls[lane * 33 + c] = A[c];
+        if (c == lane) ldiag = A[c];
+    }
+    __syncwarp();
+    const float dinv = own ? 1.0f / ldiag : 0.f;
+
+    // (Gram + lambda I) inc = g - lambda s_old, refined twice with
+    // double-float residuals
+    const float lam = used_ridge ? a.o.ridge : 0.f;
+    DF b = gd;
+    if (used_ridge) {
+        df_add_prod(b, -lam, so);
+    }
+    DF inc{0.f, 0.f};
+    float y = own ? __fadd_rn(b.h, b.l) : 0.f;
+    for (int step = 0; step < 3; ++step) {
+        y = reg_chol_solve(Ls, G, dinv, y);
+        if (!own) y = 0.f;
+        inc = df_add(inc, DF{y, 0.f});
+        if (step == 2) break;
+        DF res = b;
+        if (used_ridge) {
+            df_add_prod(res, -lam, inc.h);
+            res.l = __fmaf_rn(-lam, inc.l, res.l);
+        }
+        DF q{0.f, 0.f};
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+            if (c < G) {
+                const float ih = __shfl_sync(0xffffffffu, inc.h, c);
+                const float il = __shfl_sync(0xffffffffu, inc.l, c);
+                df_add_prod(q, gr[c].h, ih);
+                q.l = __fmaf_rn(gr[c].h, il, q.l);
+                q.l = __fmaf_rn(gr[c].l, ih, q.l);
+            }
+        }
+        res = df_add(res, df_neg(q));
+        y = own ? __fadd_rn(res.h, res.l) : 0.f;
+    }
+    if (!__all_sync(0xffffffffu, isfinite(inc.h) && isfinite(inc.l))) {
+        fail();
+        return;
+    }
+    // s_new = float32(s_old + inc)
+    float sn = 0.f;
+    if (own) {
+        const DF t = df_two_sum(so, inc.h);
+        sn = __fadd_rn(t.h, __fadd_rn(t.l, inc.l));
+    }
+    // L^{(k)} = wHw - 2 s^T rhs + s^T Gram s at the stored float32 scales
+    DF gs{0.f, 0.f};
+#pragma unroll
+    for (int c = 0; c < 32; ++c) {
+        if (c < G) {
+            const float sc = __shfl_sync(0xffffffffu, sn, c);
+            df_add_prod(gs, gr[c].h, sc);
+            gs.l = __fmaf_rn(gr[c].l, sc, gs.l);
+        }
+    }
+    DF t1{0.f, 0.f}, t2{0.f, 0.f};
+    df_add_prod(t1, sn, rh.h);
+    t1.l = __fmaf_rn(sn, rh.l, t1.l);
+    df_add_prod(t2, sn, gs.h);
+    t2.l = __fmaf_rn(sn, gs.l, t2.l);
+    t1 = df_warp_sum(t1);
+    t2 = df_warp_sum(t2);
+    double L_new = a.wHw[j] - 2.0 * df_to_double(t1) + df_to_double(t2);
+    const bool keep_old = used_ridge && a.o.ridge_accept && !(L_new <= F_old);
+    if (keep_old) L_new = F_old;
+    bool stop = false;
+    if (a.o.early_stop && a.k >= 2) {
+        const double dec = a.L_prev[j] - L_new;
+        const double den = fmax(fabs(a.L_prev[j]), (double)a.o.eps);
+        stop = (dec / den <= (double)a.o.tau_rel) || (fabs(dec) <= (double)a.o.tau_abs);
+    }
+    if (!keep_old && own) a.S[(size_t)j * G + lane] = sn;
+    if (lane == 0) {
+        a.L_prev[j] = L_new;
+        a.iters[j] = a.k;
+        a.ridge[j] += used_ridge;
+        if (stop) a.active[j] = 0;
+    }
+}
+
 }  // namespace
 
 cudaError_t launch_scale_solve(const double *gram, const double *rhs, const double *wHw, float *S,
@@ -251,6 +559,12 @@ cudaError_t launch_scale_solve(const double *gram, const double *rhs, const doub
                                int g, int k, bool eval_only, const jarq_options &o,
                                cudaStream_t s) {
     const int G = d / g;
+    SolveArgs a{gram, rhs, wHw, S, L_prev, L_out, active, iters, ridge, rstat,
+                status, p, d, g, k, eval_only, o};
+    if (G <= 32) {
+        scale_solve_small_kernel<<<(p + kSmallWarps - 1) / kSmallWarps, 32 * kSmallWarps, 0, s>>>(a);
+        return cudaGetLastError();
+    }
     const size_t per_warp = solve_warp_bytes(G);
     int wpb = (int)((96 * 1024) / per_warp);
     if (wpb > 8) wpb = 8;
@@ -259,8 +573,6 @@ cudaError_t launch_scale_solve(const double *gram, const double *rhs, const doub
     cudaError_t e = cudaFuncSetAttribute(scale_solve_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    SolveArgs a{gram, rhs, wHw, S, L_prev, L_out, active, iters, ridge, rstat,
-                status, p, d, g, k, eval_only, o};
     scale_solve_kernel<<<(p + wpb - 1) / wpb, 32 * wpb, smem, s>>>(a);
     return cudaGetLastError();
 }

@@ -306,9 +306,21 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int t = 0; t < 4; ++t) acc[t] += pp[t * 128 + rl];
                     const int E = a.expo[gi * G + h];
-                    const double v = ldexp((double)acc[0] + ldexp((double)acc[1], -10) +
-                                               ldexp((double)acc[2], -20) + ldexp((double)acc[3], -30),
-                                           E - 9);
+                    double v;
+                    if constexpr (!WIDE) {
+                        // |acc_t| < 128 * 15 * 2^20 < 2^31: the digit sum is one
+                        // exact 64-bit integer, converted with a single rounding
+                        // (two float64 operations instead of eleven; float64 is a
+                        // narrow pipe on this GPU)
+                        const long long V = acc[0] * (1LL << 30) + acc[1] * (1LL << 20) +
+                                            acc[2] * (1LL << 10) + acc[3];
+                        v = __ll2double_rn(V) *
+                            __longlong_as_double((long long)(E - 39 + 1023) << 52);
+                    } else {
+                        v = ldexp((double)acc[0] + ldexp((double)acc[1], -10) +
+                                      ldexp((double)acc[2], -20) + ldexp((double)acc[3], -30),
+                                  E - 9);
+                    }
                     double *gr = a.gram + (size_t)row * G * G;
                     gr[(size_t)gi * G + h] = v;
                     gr[(size_t)h * G + gi] = v;
