@@ -300,17 +300,14 @@ __device__ __forceinline__ DF df_warp_sum(DF a) {
 __device__ __forceinline__ double df_to_double(DF a) { return (double)a.h + (double)a.l; }
 
 // x = hi + lo with hi = x rounded to float32 (nearest, ties to even) and
-// lo = x - hi rounded to float32, by integer operations on the bits of x
-// for 2^-74 <= |x| < 2^126 (zero, tiny, huge and non-finite values take
-// the float64 conversions).
-__device__ __forceinline__ DF split_double(double x) {
+// lo = x - hi rounded to float32, by integer operations on the bits of x.
+// Branch-free for zero and for 2^-74 <= |x| < 2^126; any other value
+// (tiny, huge, non-finite) sets `rare` and must be split by split_slow.
+__device__ __forceinline__ DF split_fast(double x, bool &rare) {
     const unsigned long long bits = (unsigned long long)__double_as_longlong(x);
     const unsigned long long u = bits & 0x7FFFFFFFFFFFFFFFull;
     const int ex = (int)(u >> 52);
-    if (ex < 949 || ex > 1148) {
-        const float h = __double2float_rn(x);
-        return {h, __double2float_rn(x - (double)h)};
-    }
+    rare = (u != 0) && (ex < 949 || ex > 1148);
     // keep the top 24 significant bits, round to nearest even; a carry out
     // of the mantissa moves into the exponent field, which is still exact
     unsigned long long keep = u >> 29;
@@ -320,8 +317,12 @@ __device__ __forceinline__ DF split_double(double x) {
     const uint32_t hb = (uint32_t)(keep - (896ull << 23));
     // x - hi in units of x's last place (|r| <= 2^28), times 2^(ex - 1075)
     const int r = (int)(long long)(u - (keep << 29));
-    const float unit = __uint_as_float((uint32_t)(ex - 1075 + 127) << 23);
+    const float unit = __uint_as_float((uint32_t)((ex - 948) & 0xFF) << 23);
     float h = __uint_as_float(hb), l = __fmul_rn(__int2float_rn(r), unit);
+    if (u == 0) {
+        h = 0.f;
+        l = 0.f;
+    }
     if (bits >> 63) {
         h = -h;
         l = -l;
@@ -329,8 +330,19 @@ __device__ __forceinline__ DF split_double(double x) {
     return {h, l};
 }
 
-// In-place lower Cholesky with lane a holding row a in A[]; the operations
-// and their order are those of warp_cholesky.
+__device__ __noinline__ DF split_slow(double x) {
+    const float h = __double2float_rn(x);
+    return {h, __double2float_rn(x - (double)h)};
+}
+
+__device__ __forceinline__ DF split_double(double x) {
+    bool rare;
+    const DF v = split_fast(x, rare);
+    return rare ? split_slow(x) : v;
+}
+
+// In-place lower Cholesky with lane a holding row a in A[]; on and below
+// the diagonal the operations and their order are those of warp_cholesky.
 __device__ __forceinline__ bool reg_cholesky(float (&A)[32], int G, float thr) {
     const int lane = threadIdx.x & 31;
 #pragma unroll
@@ -343,10 +355,13 @@ __device__ __forceinline__ bool reg_cholesky(float (&A)[32], int G, float thr) {
             if (lane > k) lak = A[k] / lkk;
             if (lane == k) A[k] = lkk;
             if (lane > k) A[k] = lak;
+            // entries b <= a take the update of warp_cholesky; the entries
+            // above the diagonal (b > a) are never read again, so they take
+            // it as well instead of a predicate per entry
 #pragma unroll
             for (int b = k + 1; b < 32; ++b) {
                 const float lbk = __shfl_sync(0xffffffffu, lak, b);
-                if (lane >= b) A[b] = fmaf(-lak, lbk, A[b]);
+                A[b] = fmaf(-lak, lbk, A[b]);
             }
         }
     }
@@ -354,31 +369,27 @@ __device__ __forceinline__ bool reg_cholesky(float (&A)[32], int G, float thr) {
 }
 
 // y <- (L L^T)^{-1} y with lane a holding y_a; L row-major in Ls (stride
-// 33), dinv = 1 / L_aa.
+// 33) with zeros above the diagonal, dinv = 1 / L_aa.
 __device__ __forceinline__ float reg_chol_solve(const float *Ls, int G, float dinv, float y) {
     const int lane = threadIdx.x & 31;
-#pragma unroll
-    for (int k = 0; k < 32; ++k) {
-        if (k < G) {
-            const float yk = __shfl_sync(0xffffffffu, __fmul_rn(y, dinv), k);
-            if (lane == k) y = yk;
-            if (lane > k) y = fmaf(-Ls[lane * 33 + k], yk, y);
-        }
+#pragma unroll 4
+    for (int k = 0; k < G; ++k) {
+        const float yk = __shfl_sync(0xffffffffu, __fmul_rn(y, dinv), k);
+        const float t = fmaf(-Ls[lane * 33 + k], yk, y);   // lanes a < k: L_ak = 0
+        y = lane == k ? yk : t;
     }
-#pragma unroll
-    for (int k = 31; k >= 0; --k) {
-        if (k < G) {
-            const float xk = __shfl_sync(0xffffffffu, __fmul_rn(y, dinv), k);
-            if (lane == k) y = xk;
-            if (lane < k) y = fmaf(-Ls[k * 33 + lane], xk, y);
-        }
+#pragma unroll 4
+    for (int k = G - 1; k >= 0; --k) {
+        const float xk = __shfl_sync(0xffffffffu, __fmul_rn(y, dinv), k);
+        const float t = fmaf(-Ls[k * 33 + lane], xk, y);   // lanes a > k: L_ka = 0
+        y = lane == k ? xk : t;
     }
     return y;
 }
 
 constexpr int kSmallWarps = 4;   // rows (warps) per block of the G <= 32 kernel
 
-__global__ void __launch_bounds__(32 * kSmallWarps) scale_solve_small_kernel(SolveArgs a) {
+__global__ void __launch_bounds__(32 * kSmallWarps, 4) scale_solve_small_kernel(SolveArgs a) {
     __shared__ float Lsh[kSmallWarps][32 * 33];
     const int G = a.d / a.g;
     const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -386,12 +397,27 @@ __global__ void __launch_bounds__(32 * kSmallWarps) scale_solve_small_kernel(Sol
     if (j >= a.p || (!a.eval_only && !a.active[j])) return;  // warp-uniform
     const bool own = lane < G;
     const double *gj = a.gram + (size_t)j * G * G;
-    const float so = own ? a.S[(size_t)j * G + lane] : 0.f;
-    const DF rh = split_double(own ? a.rhs[(size_t)j * G + lane] : 0.0);
-    // row `lane` of the Gram matrix, read column-wise (coalesced) by symmetry
-    DF gr[32];
+    // row `lane` of the Gram matrix, read column-wise (coalesced) by
+    // symmetry: every load is issued before the first is used
+    double gx[32];
 #pragma unroll
-    for (int c = 0; c < 32; ++c) gr[c] = split_double((own && c < G) ? gj[(size_t)c * G + lane] : 0.0);
+    for (int c = 0; c < 32; ++c) gx[c] = (own && c < G) ? gj[(size_t)c * G + lane] : 0.0;
+    const float so = own ? a.S[(size_t)j * G + lane] : 0.f;
+    const double rhs_d = own ? a.rhs[(size_t)j * G + lane] : 0.0;
+    DF gr[32];
+    uint32_t rare = 0;
+#pragma unroll
+    for (int c = 0; c < 32; ++c) {
+        bool rc;
+        gr[c] = split_fast(gx[c], rc);
+        rare |= (uint32_t)rc << c;
+    }
+    if (__any_sync(0xffffffffu, rare != 0)) {
+#pragma unroll
+        for (int c = 0; c < 32; ++c)
+            if ((rare >> c) & 1u) gr[c] = split_slow(gj[(size_t)c * G + lane]);
+    }
+    const DF rh = split_double(rhs_d);
 
     // gradient g = rhs - Gram s_old and F(s_old) = wHw - s_old^T (rhs + g)
     DF acc{0.f, 0.f};
@@ -467,7 +493,7 @@ __global__ void __launch_bounds__(32 * kSmallWarps) scale_solve_small_kernel(Sol
     float ldiag = 1.f;
 #pragma unroll
     for (int c = 0; c < 32; ++c) {
-        Ls[lane * 33 + c] = A[c];
+        Ls[lane * 33 + c] = c <= lane ? A[c] : 0.f;
         if (c == lane) ldiag = A[c];
     }
     __syncwarp();
