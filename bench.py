@@ -49,7 +49,7 @@ TRAFFIC = {
     "gram": ("k_tc_gram.cu", "461b29d32c89", 164.122e6 + 27.549e6),
     "proj": ("k_tc_proj.cu", "b46541dbdbb2", 1370.069e6 + 156.471e6),
     "ptilde": ("k_tc_proj.cu", "b46541dbdbb2", 134.248e6 + 150.687e6 + 222.887e6 + 103.208e6),
-    "scale_solve": ("k_solve.cu", "997566a9e983", 35.309e6 + 0.000256e6),
+    "scale_solve": ("k_solve.cu", "326c857f6b6b", 35.309e6 + 0.000256e6),
     # profiles/ncu_syrk_attn_in_4096_n32768.md, scaled from 32768 to 262144 tokens
     "syrk": ("k_syrk.cu", "3896afedc783", 8 * 537.171e6 + 40.712e6),
 }

@@ -4,9 +4,10 @@
 //  1. reads its G x G Gram matrix -- symmetric by construction, since the
 //     Gram kernel computes each block once and writes it to both triangles,
 //     so the symmetrisation of App. E "Solving for scales" is the identity
-//     on it -- and forms, in float64, the gradient g = rhs - Gram s_old of
-//     the current scales (rhs_i = c_i^T P_i from the target projection) and
-//     the objective F(s_old) = wHw - s_old^T (rhs + g);
+//     on it -- and forms, in float64 (double-float in the G <= 32 kernel
+//     below), the gradient g = rhs - Gram s_old of the current scales
+//     (rhs_i = c_i^T P_i from the target projection) and the objective
+//     F(s_old) = wHw - s_old^T (rhs + g);
 //  2. factors the Gram matrix by Cholesky in float32 (the paper solves this
 //     system in FP32).  A pivot at or below rcond * max(max diag, eps), a
 //     nonfinite entry or a failed factorisation adds ridge * I and retries
@@ -15,7 +16,7 @@
 //     increment of the scales: Gram s_new = rhs <=> Gram (s_new - s_old) = g,
 //     and with the ridge (Gram + lambda I) delta = g - lambda s_old (float32
 //     Cholesky, then two refinement steps whose residuals are formed in
-//     float64), and stores s_new rounded to float32;
+//     float64 or double-float), and stores s_new rounded to float32;
 //  4. evaluates L^{(k)} = F(s_new) = wHw - 2 s_new^T rhs + s_new^T Gram s_new
 //     at the stored float32 scales and applies the early stop of Eq.
 //     strict_stopping against L^{(k-1)}; with the ridge-acceptance option a
