@@ -44,11 +44,11 @@ DTYPE = "f32 (integer-digit fp16/bf16 tensor-core products with exact partial su
 # profiles/ncu_syrk_attn_in_4096_n32768.md), valid while the kernel's source
 # file is unchanged (first 12 hex digits of its SHA-1).
 TRAFFIC = {
-    "target": ("k_tc_target.cu", "18ee82cb694f", 38.299e6 + 0.152e6),
+    "target": ("k_tc_target.cu", "4ae89381851e", 38.299e6 + 0.152e6),
     "babai": ("k_babai.cu", "d2d96a20da85", 14.274e6 + 0.001536e6),
-    "gram": ("k_tc_gram.cu", "461b29d32c89", 164.122e6 + 27.549e6),
-    "proj": ("k_tc_proj.cu", "b46541dbdbb2", 1370.069e6 + 156.471e6),
-    "ptilde": ("k_tc_proj.cu", "b46541dbdbb2", 134.248e6 + 150.687e6 + 222.887e6 + 103.208e6),
+    "gram": ("k_tc_gram.cu", "38618e3a1081", 164.122e6 + 27.549e6),
+    "proj": ("k_tc_proj.cu", "6cf1b3d8cc4f", 1370.069e6 + 156.471e6),
+    "ptilde": ("k_tc_proj.cu", "6cf1b3d8cc4f", 134.248e6 + 150.687e6 + 222.887e6 + 103.208e6),
     "scale_solve": ("k_solve.cu", "326c857f6b6b", 35.309e6 + 0.000256e6),
     # profiles/ncu_syrk_attn_in_4096_n32768.md, scaled from 32768 to 262144 tokens
     "syrk": ("k_syrk.cu", "3896afedc783", 8 * 537.171e6 + 40.712e6),

@@ -7,6 +7,8 @@
 #include <cuda_fp16.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "../../include/jarq.h"
 
 namespace jarq {
@@ -258,7 +260,15 @@ cudaError_t launch_pdl_cluster(void (*kernel)(KArgs...), dim3 grid, dim3 block, 
 cudaError_t launch_init_rows(int *active, int *iters, int *accepted, int *ridge, int *rstat,
                              int p, cudaStream_t s);
 
+// Multiprocessor count of the current device (cached per device ordinal).
 int num_sms();
+
+// Enable `bytes` of dynamic shared memory for `func` on the current device.
+// The attribute is per device and a process may drive several devices, so
+// `done` is a bit mask over device ordinals; ordinals of 64 and above set
+// the attribute on every call.
+cudaError_t set_max_dynamic_smem(const void *func, int bytes,
+                                 std::atomic<unsigned long long> &done);
 
 // True for device (or managed) memory of the current context.
 bool on_device(const void *p);

@@ -476,16 +476,12 @@ cudaError_t launch_tc_gram(const CUtensorMap &mapC, const CUtensorMap &mapS, con
                            const int32_t *Z, const int *expo, const int *active, double *gram,
                            int p, int p_pad, int d, int d_pad, int g, int bits, int *status,
                            cudaStream_t s) {
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(tc_gram_kernel<false>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, gram_smem<false>());
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(tc_gram_kernel<true>,
-                                     cudaFuncAttributeMaxDynamicSharedMemorySize, gram_smem<true>());
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+    static std::atomic<unsigned long long> attr_narrow{0}, attr_wide{0};
+    cudaError_t e = set_max_dynamic_smem((const void *)tc_gram_kernel<false>, gram_smem<false>(),
+                                         attr_narrow);
+    if (e == cudaSuccess)
+        e = set_max_dynamic_smem((const void *)tc_gram_kernel<true>, gram_smem<true>(), attr_wide);
+    if (e != cudaSuccess) return e;
     const int G = d / g;
     GramArgs a{Q, Z, expo, active, gram, status, p, d, g, G, d_pad};
     dim3 grid(p_pad / 128, (G + 1) / 2, 1);

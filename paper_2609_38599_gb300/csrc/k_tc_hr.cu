@@ -267,13 +267,9 @@ template <int BN>
 cudaError_t launch_tc_hr_bn(const CUtensorMap &mapA, const CUtensorMap &mapB, const HrArgs &a,
                             dim3 grid, cudaStream_t s, bool programmatic = false) {
     using C = HrCfg<BN>;
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(tc_hr_kernel<BN>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+    static std::atomic<unsigned long long> attr_done{0};
+    const cudaError_t e = set_max_dynamic_smem((const void *)tc_hr_kernel<BN>, C::kSmem, attr_done);
+    if (e != cudaSuccess) return e;
     if (programmatic) return launch_pdl(tc_hr_kernel<BN>, grid, dim3(320), C::kSmem, s, mapA, mapB, a);
     tc_hr_kernel<BN><<<grid, 320, C::kSmem, s>>>(mapA, mapB, a);
     return cudaGetLastError();

@@ -648,13 +648,9 @@ cudaError_t launch_ptilde(const CUtensorMap &mapPd, const CUtensorMap &mapR, con
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     using C = ProjCfg<kHDig, true>;
-    static bool attr_set = false;
-    if (!attr_set) {
-        e = cudaFuncSetAttribute(tc_proj_kernel<kHDig, true>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+    static std::atomic<unsigned long long> attr_done{0};
+    e = set_max_dynamic_smem((const void *)tc_proj_kernel<kHDig, true>, C::kSmem, attr_done);
+    if (e != cudaSuccess) return e;
     ProjArgs a{out_hi, out_lo, pexp, rexp, status, p, d, g, d / g, p_pad, d};
     // persistent: one CTA per SM over the (p_pad / 128) x (d / 64) tiles
     (void)d_pad;
@@ -676,13 +672,10 @@ cudaError_t launch_tc_proj(const CUtensorMap &mapW, const CUtensorMap &mapH, flo
                            float *Plo, const int *wexp, const int *hexp, int p, int p_pad, int d,
                            int d_pad, int g, int *status, cudaStream_t s) {
     using C = ProjCfg<kWDig, false>;
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(tc_proj_kernel<kWDig, false>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+    static std::atomic<unsigned long long> attr_done{0};
+    const cudaError_t e =
+        set_max_dynamic_smem((const void *)tc_proj_kernel<kWDig, false>, C::kSmem, attr_done);
+    if (e != cudaSuccess) return e;
     ProjArgs a{Phi, Plo, wexp, hexp, status, p, d, g, d / g, p_pad, d_pad};
     dim3 grid(p_pad / 128, d_pad / 64, 1);
     tc_proj_kernel<kWDig, false><<<grid, 320, C::kSmem, s>>>(mapW, mapH, a);

@@ -298,13 +298,9 @@ cudaError_t launch_tc_target(const CUtensorMap &mapC, const CUtensorMap &mapT, f
                              float *out_lo, const float *S, const int *expoT, const int *active,
                              int p, int p_pad, int d_pad, int g, int G, int i, int nsplit,
                              int qmax, int *status, cudaStream_t s) {
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(tc_target_kernel,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+    static std::atomic<unsigned long long> attr_done{0};
+    const cudaError_t e = set_max_dynamic_smem((const void *)tc_target_kernel, kSmem, attr_done);
+    if (e != cudaSuccess) return e;
     const int per = (G + nsplit - 1) / nsplit;
     const int tiles = p_pad / 128;
     // The kernel supports clusters of 2 or 4 row tiles multicasting the digit
