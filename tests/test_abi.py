@@ -73,3 +73,16 @@ def test_argument_errors_return_before_cuda_work(jarq):
     assert lib.jarq_objective(None, None, None, None, None, 1, 3, None, None) == jarq.JARQ_ERR_ARG
     assert lib.jarq_hessian_din(None) == 0 and lib.jarq_hessian_group_size(None) == 0
     lib.jarq_hessian_destroy(None)
+
+
+def test_writeback_of_an_empty_layer_returns_ok_without_cuda_work(jarq):
+    """dout = 0: the write-back calls validate their sizes and return JARQ_OK
+    before touching any pointer (which may then be NULL)."""
+    lib = jarq.library()
+    assert lib.jarq_canonicalize(None, None, None, 0, 256, 64, 3, None) == 0
+    assert lib.jarq_dequantize(None, None, None, 0, 256, 64, 3, 1, None, None) == 0
+    assert lib.jarq_pack_codes(None, 0, 256, 3, None, None) == 0
+    # the sizes are still checked
+    assert lib.jarq_canonicalize(None, None, None, 0, 250, 64, 3, None) == jarq.JARQ_ERR_ARG
+    assert lib.jarq_dequantize(None, None, None, 0, 256, 64, 9, 1, None, None) == jarq.JARQ_ERR_ARG
+    assert lib.jarq_pack_codes(None, -1, 256, 3, None, None) == jarq.JARQ_ERR_ARG

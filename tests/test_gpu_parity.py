@@ -141,6 +141,41 @@ def test_k0_returns_host_state(jarq):
     np.testing.assert_allclose(st["L_final"], st["L_host"], rtol=0)
 
 
+def test_empty_layer_is_a_no_op(jarq):
+    """dout = 0 (no output rows): every layer entry point returns JARQ_OK and
+    touches nothing; the pointers may then be NULL."""
+    import ctypes
+    lay = tiny_layer()
+    hess = jarq.prepare(torch.as_tensor(lay.H, device="cuda"), lay.g)
+    lib = jarq.library()
+    h = hess.handle
+    o = jarq.default_options(max_iters=3)
+    OK = 0
+    assert lib.jarq_refine_layer(h, None, None, None, None, 0, lay.bits, ctypes.byref(o), None, None) == OK
+    assert lib.jarq_objective(h, None, None, None, None, 0, lay.bits, None, None) == OK
+    assert lib.jarq_objective_noalloc(h, None, None, None, None, 0, lay.bits, None, None) == OK
+    assert lib.jarq_residual_product(h, None, None, None, None, 0, lay.bits, None, None) == OK
+    assert lib.jarq_fit_scales(h, None, None, None, None, 0, lay.bits, 0, 3, None, None, None) == OK
+    assert lib.jarq_multicode_probe(h, None, None, None, None, 0, lay.bits, 0,
+                                    None, None, None, None, None, None) == OK
+    # the mu-target still needs its two Gram matrices (not read when dout = 0)
+    Hd = torch.as_tensor(lay.H, device="cuda")
+    assert lib.jarq_refine_layer_mu(h, None, None, None, None, 0, lay.bits, Hd.data_ptr(),
+                                    Hd.data_ptr(), 0.5, 0.0, ctypes.byref(o), None, None) == OK
+    assert lib.jarq_refine_layer_mu(h, None, None, None, None, 0, lay.bits, None, None, 0.5, 0.0,
+                                    ctypes.byref(o), None, None) == jarq.JARQ_ERR_ARG
+    # real buffers with dout = 0 stay untouched
+    S = torch.as_tensor(lay.S0[:1], device="cuda").clone()
+    Q = torch.as_tensor(lay.Q0[:1], device="cuda").clone()
+    W = torch.as_tensor(lay.W[:1], device="cuda")
+    Z = torch.as_tensor(lay.Z[:1], device="cuda")
+    assert lib.jarq_refine_layer(h, W.data_ptr(), S.data_ptr(), Q.data_ptr(), Z.data_ptr(), 0,
+                                 lay.bits, ctypes.byref(o), None, None) == OK
+    torch.cuda.synchronize()
+    assert np.array_equal(S.cpu().numpy(), lay.S0[:1]) and np.array_equal(Q.cpu().numpy(), lay.Q0[:1])
+    hess.close()
+
+
 def test_format_preserved(jarq):
     lay = small_layer(256, 64, 64, 4, seed=24)
     Z0 = lay.Z.copy()
