@@ -2,10 +2,12 @@
 
 One step = one ``jarq_refine_layer`` call refining the Llama-2-7B q_proj
 layer (4096 x 4096, g = 128, 3-bit, RTN host, K = 10 iterations, early stop
-off) from its host state: the whole hot path (per iteration the residual
-product H r, Gram matrices, joint scale solve and the 32-group Babai sweep).
-Inputs are seeded synthetic tensors resident in HBM; the working set per
-step (H, W, H r and the residual, 64 MB each) exceeds the 129 MB L2.
+off) from its host state: the whole hot path (once the target projection
+P = W H and its folded form; per iteration the Gram matrices, right-hand
+sides and joint scale solve, then the 32-group sweep of phase products and
+Babai proposals).  Inputs are seeded synthetic tensors resident in HBM; the
+working set per step (W, P and the folded P 64 MB each, the digit planes of
+H 336 MB) exceeds the 129 MB L2.
 
 ``value`` is weights refined per second over all ranks; ``e2e`` is the same
 metric through the C ABI with host buffers (host-to-device and back inside
