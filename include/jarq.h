@@ -184,11 +184,13 @@ jarq_status jarq_objective(jarq_hessian *h, const float *W, const float *S, cons
                            void *stream);
 
 /* The residual product H r_j of every row, r_j = w_j - D_{s_j}(q_j - z_j),
- * written as float32 to HR[dout][din] (host or device), computed by the
- * split-precision tensor-core kernel that gives the Gauss-Seidel sweep its
- * group slices (H r_j)_i (Sec. 3.3.2, Eq. conditional_residual).  It exists
- * so that tests can compare that contraction element by element with a
- * reference.  Same layouts and checks as jarq_refine_layer. */
+ * written as float32 to HR[dout][din] (host or device): the group slices
+ * (H r_j)_i of Sec. 3.3.2, Eq. conditional_residual, for every group at
+ * once.  It is computed by the split-precision tensor-core kernel behind
+ * jarq_objective (the refinement's sweep forms its Babai targets with the
+ * exact folded phase product instead), and it exists so that tests can
+ * compare that contraction element by element with a reference.  Same
+ * layouts and checks as jarq_refine_layer. */
 jarq_status jarq_residual_product(jarq_hessian *h, const float *W, const float *S,
                                   const uint8_t *Q, const int32_t *Z, int dout, int bits,
                                   float *HR, void *stream);

@@ -340,7 +340,7 @@ def multicode_probe(hess: Hessian, W, S, Q, Z, bits: int, group: int):
 
 def residual_product(hess: Hessian, W, S, Q, Z, bits: int, out=None):
     """``jarq_residual_product``: H r of every row (float32, dout x din), from
-    the tensor-core kernel of the sweep's residual products."""
+    the split-precision tensor-core kernel behind ``jarq_objective``."""
     dout, din = int(W.shape[0]), int(W.shape[1])
     if out is None:
         if _is_torch(W):
