@@ -40,11 +40,11 @@ SM_MAX_MHZ = 2070.0
 DTYPE = "f32 (integer-digit fp16/bf16 tensor-core products with exact partial sums, double-float accumulation)"
 
 # DRAM bytes (read + write) per launch from one ncu capture of this workload
-# (profiles/ncu_refine_kernels_q_proj_4096x4096_g128_w3.md; the sweep kernels'
-# figures are those of the first phase; the scale solve's from
-# profiles/ncu_scale_solve_q_proj_4096x4096_g128_w3.md; the Hessian kernel's from
-# profiles/ncu_syrk_attn_in_4096_n32768.md), valid while the kernel's source
-# file is unchanged (first 12 hex digits of its SHA-1).
+# (the sweep kernels' figures are those of the first phase; the Hessian
+# kernel's is a capture at 32768 tokens scaled to the full token count); the
+# summaries kept with the profiles give each capture's command.  A figure is
+# valid while the kernel's source file is unchanged (first 12 hex digits of
+# its SHA-1); otherwise the bench reports null.
 TRAFFIC = {
     "target": ("k_tc_target.cu", "4ae89381851e", 38.299e6 + 0.152e6),
     "babai": ("k_babai.cu", "d2d96a20da85", 14.274e6 + 0.001536e6),
@@ -52,7 +52,7 @@ TRAFFIC = {
     "proj": ("k_tc_proj.cu", "6cf1b3d8cc4f", 1370.069e6 + 156.471e6),
     "ptilde": ("k_tc_proj.cu", "6cf1b3d8cc4f", 134.248e6 + 150.687e6 + 222.887e6 + 103.208e6),
     "scale_solve": ("k_solve.cu", "326c857f6b6b", 35.309e6 + 0.000256e6),
-    # profiles/ncu_syrk_attn_in_4096_n32768.md, scaled from 32768 to 262144 tokens
+    # captured at 32768 tokens, scaled to 262144
     "syrk": ("k_syrk.cu", "3896afedc783", 8 * 537.171e6 + 40.712e6),
 }
 HESSIAN_WORKLOAD = "llama2_7b_attn_in_4096_n262144"
@@ -79,6 +79,8 @@ def parse_args():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default=WORKLOAD)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip timing the other workloads (tiny, down_proj, gate_proj, block)")
     ap.add_argument("--tokens", type=int, default=None,
                     help="calibration tokens of the Hessian workload (default: 128 x 2048)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
@@ -412,6 +414,8 @@ def run_ours(args, rank, world):
                           "hbm_frac": by / (ms_ / 1e3) / 1e9 / pk2["hbm_gbs"],
                           "note": "includes the code validation pass and a synchronize"}
         line["postpass"] = post
+    if rank == 0 and not args.no_configs:
+        line["configs"] = configs_leg(args, jarq, dev)
     if rank == 0:
         line["hessian"] = hessian_leg(args, jarq, dev)
         line["mu_target"] = mu_target_leg(args, jarq, dev, lay.name)
@@ -453,6 +457,167 @@ def run_ours(args, rank, world):
     if dist:
         dist.destroy_process_group()
     return 0
+
+
+def flush_l2(buf):
+    """Overwrite a buffer larger than the 129 MB L2 (between timed steps)."""
+    buf.add_(1.0)
+
+
+def per_kernel(jarq, fn, steps):
+    """Launches and device milliseconds of every library kernel over `steps`
+    calls of fn, from the library's CUDA event pair around each launch on
+    its stream."""
+    import torch
+    jarq.profile_reset()
+    jarq.profile_enable(True)
+    for _ in range(steps):
+        fn()
+    torch.cuda.synchronize()
+    jarq.profile_enable(False)
+    out = {}
+    for k in jarq.KERNELS:
+        n, tot = jarq.profile_read(k)
+        if n:
+            out[k] = (n, tot)
+    return out
+
+
+def summarise_kernels(parts, pk, peak_kind):
+    """Per-kernel shares and roofline fractions from [(layer, {kernel: (n,
+    ms)})]: a kernel's algorithmic work is summed over the layers it ran on
+    (each with its own shape), divided by its summed device time."""
+    tot = {}
+    work = {}
+    for lay, ks in parts:
+        for k, (n, ms) in ks.items():
+            t = tot.setdefault(k, [0, 0.0])
+            t[0] += n
+            t[1] += ms
+            m = kernel_model(k, lay)
+            if m:
+                w = work.setdefault(k, [m["bound"], 0.0, 0.0])
+                w[1] += m["work"] * n
+                w[2] += m.get("issued", m["work"]) * n
+    all_ms = sum(v[1] for v in tot.values()) or 1.0
+    kernels = {k: {"launches": v[0], "total_ms": v[1], "avg_us": 1e3 * v[1] / v[0],
+                   "share": v[1] / all_ms} for k, v in tot.items()}
+    roofs = {}
+    for k, (bound, w, wi) in work.items():
+        sec = tot[k][1] / 1e3
+        if bound == "tensor":
+            ach, peak, unit = w / sec / 1e12, pk["bf16_tflops_sustained"], "TFLOP/s"
+        elif bound == "alu":
+            ach = w / sec / 1e12
+            peak, unit = SM_COUNT * FP32_LANES_PER_SM * 2 * SM_MAX_MHZ * 1e6 / 1e12, "TFLOP/s"
+        else:
+            ach, peak, unit = w / sec / 1e9, pk["hbm_gbs"], "GB/s"
+        e = {"kernel": k, "bound": bound, "achieved": ach, "peak": peak, "unit": unit,
+             "frac": ach / peak, "peak_note": f"{peak_kind}"}
+        if bound == "tensor":
+            e["issued_frac"] = wi / sec / 1e12 / peak
+        roofs[k] = e
+    dom = max(kernels, key=lambda k: kernels[k]["total_ms"]) if kernels else None
+    return kernels, roofs, dom
+
+
+def configs_leg(args, jarq, dev):
+    """Every workload besides the headline one, each timed on its own: the
+    tiny layer, the Llama-2-7B down_proj layer, the Llama-3-8B gate_proj
+    layer (one jarq_refine_layer call per step, K as configured, early stop
+    off) and the Llama-2-7B decoder block (its three Hessians prepared and
+    its seven layers refined per step).  Each step is timed alone by CUDA
+    events on the current stream, with a 256 MiB buffer overwritten between
+    steps so that no step starts with the previous one's data in L2; the
+    median step is reported.  Per-kernel shares and roofline fractions come
+    from a second pass with the library's per-launch event pairs."""
+    import torch
+    from synth import block_layers, config_layer
+    pk, peak_kind = peaks()
+    flush = torch.zeros(64 << 20, device=dev)
+    out = {}
+
+    def median_ms(step, warmup, steps):
+        for _ in range(warmup):
+            step()
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(steps):
+            flush_l2(flush)
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            step()
+            b.record()
+            torch.cuda.synchronize()
+            ts.append(a.elapsed_time(b))
+        return float(statistics.median(ts)), ts
+
+    for name, steps in (("tiny_256x256_g64_w3", 20),
+                        ("llama2_7b_down_proj_4096x11008_g128_w4", 5),
+                        ("llama3_8b_gate_proj_14336x4096_g128_w3", 5)):
+        lay = config_layer(name, device=dev)
+        hess = jarq.prepare(lay.H, lay.g)
+        opts = jarq.default_options(max_iters=lay.K, early_stop=0)
+        S, Q = lay.S0.clone(), lay.Q0.clone()
+
+        def step():
+            S.copy_(lay.S0)
+            Q.copy_(lay.Q0)
+            jarq.refine(hess, lay.W, S, Q, lay.Z, lay.bits, options=opts, collect_stats=False)
+
+        n0 = jarq.launch_count()
+        ms, ts = median_ms(step, 3, steps)
+        launches = (jarq.launch_count() - n0) / (3 + steps)
+        kernels, roofs, dom = summarise_kernels([(lay, per_kernel(jarq, step, steps))], pk,
+                                                peak_kind)
+        out[name] = {"din": lay.din, "dout": lay.dout, "group_size": lay.g, "bits": lay.bits,
+                     "K": lay.K, "s_per_layer": ms / 1e3,
+                     "weights_per_s": lay.din * lay.dout / (ms / 1e3), "steps": steps,
+                     "step_ms_min_max": [min(ts), max(ts)], "launches_per_step": launches,
+                     "dominant": dom, "roofline": roofs.get(dom), "roofline_all": roofs,
+                     "kernels": kernels}
+        hess.close()
+        del lay, S, Q, hess
+        torch.cuda.empty_cache()
+
+    hs, layers = block_layers(device=dev)
+    states = [(lay.S0.clone(), lay.Q0.clone()) for _, lay in layers]
+    prof = {}
+
+    def block_step(profile=False):
+        hess = {k: jarq.prepare(h, 128) for k, h in hs.items()}
+        if profile:
+            torch.cuda.synchronize()
+        for idx, ((hkey, lay), (S, Q)) in enumerate(zip(layers, states)):
+            S.copy_(lay.S0)
+            Q.copy_(lay.Q0)
+            opts = jarq.default_options(max_iters=lay.K, early_stop=0)
+            run = lambda: jarq.refine(hess[hkey], lay.W, S, Q, lay.Z, lay.bits, options=opts,
+                                      collect_stats=False)
+            if profile:
+                prof[idx] = (lay, per_kernel(jarq, run, 1))
+            else:
+                run()
+        for h in hess.values():
+            h.close()
+
+    n0 = jarq.launch_count()
+    ms, ts = median_ms(block_step, 3, 3)
+    launches = (jarq.launch_count() - n0) / 6
+    block_step(profile=True)
+    kernels, roofs, dom = summarise_kernels(list(prof.values()), pk, peak_kind)
+    weights = sum(lay.din * lay.dout for _, lay in layers)
+    out["llama2_7b_block"] = {
+        "layers": [lay.name for _, lay in layers], "group_size": 128, "bits": 3, "K": 10,
+        "hessians_prepared_per_step": len(hs), "s_per_block": ms / 1e3,
+        "weights_per_s": weights / (ms / 1e3), "steps": 3, "step_ms_min_max": [min(ts), max(ts)],
+        "launches_per_step": launches, "dominant": dom, "roofline": roofs.get(dom),
+        "roofline_all": roofs,
+        "kernels": kernels,
+        "kernels_note": "refinement calls only (the Hessian preparation is in s_per_block)"}
+    del hs, layers, states, flush
+    torch.cuda.empty_cache()
+    return out
 
 
 def hessian_leg(args, jarq, dev, standalone=False):

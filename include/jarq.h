@@ -288,14 +288,15 @@ jarq_status jarq_accumulate_hessian(const void *X, int n, int d, float scale, fl
 
 /* Per-row objective without any device allocation.  The paper has no
  * counterpart: this entry point exists for callers that cannot allocate
- * device memory when they need the objective -- code running while a CUDA
- * graph is being captured, serving processes that reserve all device memory
- * at start-up and forbid later allocations, and callers that cannot afford
- * the device-wide synchronisation an allocation may cause.  It computes the
- * same values as jarq_objective.
- *   All buffers must be device memory (host pointers return JARQ_ERR_ARG,
- *   since staging them would allocate).  The prepared handle h comes from
- *   jarq_prepare_hessian, which allocates once, up front.
+ * device memory when they need the objective -- serving processes that
+ * reserve all device memory at start-up and forbid later allocations, and
+ * callers that cannot afford the device-wide synchronisation an allocation
+ * may cause.  It computes the same values as jarq_objective.
+ *   All buffers must be device memory of the handle's GPU (host pointers and
+ *   buffers on another GPU return JARQ_ERR_ARG; staging host memory would
+ *   allocate).  The prepared handle h comes from jarq_prepare_hessian, which
+ *   allocates once, up front.  The caller's current device is restored
+ *   before the call returns.
  *   Limit: ceil(dout/128)*128 * ceil(din/128)*128 <= 2^20 (for example a
  *   1024 x 1024 layer); larger layers return JARQ_ERR_ARG.
  *   Scratch: one statically sized device array (about 16 MiB) that every GPU
@@ -303,9 +304,10 @@ jarq_status jarq_accumulate_hessian(const void *X, int n, int d, float scale, fl
  *   and it keeps the last call's contents; the call clears what must start at
  *   zero.  Calls that overlap on the GPU (from two streams or two host
  *   threads) race on it: serialise them.
- *   The first call on a device looks up the array's device address; make
- *   that first call before any stream capture.
- *   Returns after the results are in F_per_row. */
+ *   The first call on a device looks up the array's device address once.
+ *   Synchronous: the call waits on `stream` after checking the codes and
+ *   again at the end, and reads the status on the host; it returns after
+ *   the results are in F_per_row. */
 jarq_status jarq_objective_noalloc(jarq_hessian *h, const float *W, const float *S,
                                    const uint8_t *Q, const int32_t *Z, int dout, int bits,
                                    double *F_per_row, void *stream);

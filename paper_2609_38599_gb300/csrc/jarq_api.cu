@@ -388,7 +388,7 @@ int jarq_hessian_group_size(const jarq_hessian *h) { return h ? h->g : 0; }
 
 void jarq_hessian_destroy(jarq_hessian *h) {
     if (!h) return;
-    cudaSetDevice(h->device);
+    DeviceGuard dg(h->device);
     cudaDeviceSynchronize();
     free_ws(h->ws);
     cudaFree(h->Hs);
@@ -501,6 +501,8 @@ jarq_status jarq_objective(jarq_hessian *h, const float *W, const float *S, cons
     if (!layer_args_ok(h, W, S, Q, Z, dout, bits) || (dout > 0 && !F_per_row))
         return JARQ_ERR_ARG;
     if (dout == 0) return JARQ_OK;
+    DeviceGuard dg(h->device);
+    if (!dg.ok()) return JARQ_ERR_CUDA;
     cudaStream_t st = (cudaStream_t)stream;
     LayerArgs la;
     jarq_status rc = layer_front(h, W, S, Q, Z, dout, bits, la, st);
@@ -520,6 +522,8 @@ jarq_status jarq_residual_product(jarq_hessian *h, const float *W, const float *
                                   float *HR, void *stream) {
     if (!layer_args_ok(h, W, S, Q, Z, dout, bits) || (dout > 0 && !HR)) return JARQ_ERR_ARG;
     if (dout == 0) return JARQ_OK;
+    DeviceGuard dg(h->device);
+    if (!dg.ok()) return JARQ_ERR_CUDA;
     cudaStream_t st = (cudaStream_t)stream;
     LayerArgs la;
     jarq_status rc = layer_front(h, W, S, Q, Z, dout, bits, la, st);
@@ -548,6 +552,8 @@ jarq_status jarq_fit_scales(jarq_hessian *h, const float *W, float *S, const uin
         return JARQ_ERR_ARG;
     if (method == JARQ_FIT_COORDINATE && passes < 1) return JARQ_ERR_ARG;
     if (dout == 0) return JARQ_OK;
+    DeviceGuard dg(h->device);
+    if (!dg.ok()) return JARQ_ERR_CUDA;
     cudaStream_t st = (cudaStream_t)stream;
     LayerArgs la;
     jarq_status rc = layer_front(h, W, S, Q, Z, dout, bits, la, st, true);
@@ -589,6 +595,8 @@ jarq_status jarq_multicode_probe(jarq_hessian *h, const float *W, const float *S
                                  int32_t *changed, double *dF, void *stream) {
     if (!layer_args_ok(h, W, S, Q, Z, dout, bits) || group < 0 || group >= h->G) return JARQ_ERR_ARG;
     if (dout == 0) return JARQ_OK;
+    DeviceGuard dg(h->device);
+    if (!dg.ok()) return JARQ_ERR_CUDA;
     cudaStream_t st = (cudaStream_t)stream;
     LayerArgs la;
     jarq_status rc = layer_front(h, W, S, Q, Z, dout, bits, la, st, true);
@@ -640,6 +648,8 @@ jarq_status refine_impl(jarq_hessian *h, const float *W, float *S, uint8_t *Q, c
     if (o.max_iters < 0 || !(o.ridge >= 0.f) || !(o.rcond >= 0.f) || !(o.eps >= 0.f))
         return JARQ_ERR_ARG;
     if (dout == 0) return JARQ_OK;
+    DeviceGuard dg(h->device);
+    if (!dg.ok()) return JARQ_ERR_CUDA;
     cudaStream_t st = (cudaStream_t)stream;
     LayerArgs la;
     jarq_status rc = layer_front(h, W, S, Q, Z, dout, bits, la, st, true);

@@ -270,8 +270,41 @@ int num_sms();
 cudaError_t set_max_dynamic_smem(const void *func, int bytes,
                                  std::atomic<unsigned long long> &done);
 
-// True for device (or managed) memory of the current context.
+// True for managed memory, or device memory of the current device (a buffer
+// on another GPU is false: the kernels would read a peer's memory).
 bool on_device(const void *p);
+
+// Makes `device` current for the guard's lifetime and then restores the
+// caller's current device, so that an entry point never leaves the calling
+// thread on another GPU.
+class DeviceGuard {
+  public:
+    explicit DeviceGuard(int device) {
+        if (cudaGetDevice(&prev_) != cudaSuccess) {
+            (void)cudaGetLastError();
+            return;
+        }
+        if (prev_ == device) {
+            ok_ = true;
+            return;
+        }
+        if (cudaSetDevice(device) == cudaSuccess) {
+            ok_ = switched_ = true;
+        } else {
+            (void)cudaGetLastError();
+        }
+    }
+    ~DeviceGuard() {
+        if (switched_) cudaSetDevice(prev_);
+    }
+    bool ok() const { return ok_; }
+    DeviceGuard(const DeviceGuard &) = delete;
+    DeviceGuard &operator=(const DeviceGuard &) = delete;
+
+  private:
+    int prev_ = 0;
+    bool ok_ = false, switched_ = false;
+};
 
 // 2D tensor map of 2-byte elements (bf16 or fp16) over [rows][cols]
 // (pitch = cols elements), box_rows x 64 boxes, 128-byte swizzle,

@@ -27,11 +27,6 @@
 // The drain does 17 float32 operations per output and group, hence
 // sixteen drain warps; the scale and block exponent of the next group are
 // loaded one group ahead.
-// The digit tiles are the same for every row tile, so CTAs of consecutive
-// row tiles can form a cluster of C: each loads 4/C of the digit planes and
-// multicasts them to all C, cutting that traffic by C.  A stage is refilled
-// only after every CTA of the cluster has consumed it (its "empty" barrier
-// counts one MMA commit per CTA), and no CTA leaves before the others.
 #include <cmath>
 
 #include "tc_common.cuh"
@@ -57,7 +52,6 @@ struct TargetArgs {
     const int *active;
     int *status;
     int p, p_pad, d_pad, g, G, i, seg_per_split;
-    int csize;                // CTAs per cluster (1, 2 or 4)
     float round_c;            // 1.5 * 2^(23 - k): rounds to multiples of 2^-k
 };
 
@@ -84,9 +78,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int nkc = a.g / 64;
     const int nchunks = nseg * nkc;
 
-    const uint32_t crank = a.csize > 1 ? tc::cluster_ctarank() : 0;
-    const uint16_t cmask = (uint16_t)((1u << a.csize) - 1u);
-
     auto full = [&](int s) { return tc::smem_u32(bars + s); };
     auto empty = [&](int s) { return tc::smem_u32(bars + kStages + s); };
     auto afull = [&](int b) { return tc::smem_u32(bars + 2 * kStages + b); };
@@ -97,7 +88,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             tc::mbar_init(full(s), 1);
-            tc::mbar_init(empty(s), a.csize);   // one MMA commit per CTA of the cluster
+            tc::mbar_init(empty(s), 1);
         }
         for (int b = 0; b < 2; ++b) {
             tc::mbar_init(afull(b), 1);
@@ -115,11 +106,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc::prefetch_tmap(&mapT);
     }
     tc::tc_fence_before();
-    // every CTA's barriers are initialised before any multicast reaches them
-    if (a.csize > 1)
-        tc::cluster_sync();
-    else
-        __syncthreads();
+    __syncthreads();
     tc::tc_fence_after();
     const uint32_t tmem = *tmem_slot;
     // the codes are rewritten by the previous Babai phase
@@ -136,21 +123,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                 break;
             }
             const int kx = h0 * a.g + c * 64;
-            // this CTA's full barrier counts the whole stage, including the
-            // digit tiles the other CTAs of the cluster multicast into it
             tc::mbar_expect_tx(full(s), kStage);
             tc::tma_load_2d(tileA(s), &mapC, full(s), kx, j0);
 #pragma unroll
-            for (int t = 0; t < 4; ++t) {
-                if (a.csize == 1)
-                    tc::tma_load_2d(tileB(s, t), &mapT, full(s), kx, t * a.d_pad + m0);
-                else if (t % a.csize == (int)crank)
-                    tc::tma_load_2d_mc(tileB(s, t), &mapT, full(s), kx, t * a.d_pad + m0, cmask);
-            }
+            for (int t = 0; t < 4; ++t)
+                tc::tma_load_2d(tileB(s, t), &mapT, full(s), kx, t * a.d_pad + m0);
             issued = c + 1;
         }
-        // do not leave before every CTA of the cluster has consumed the
-        // stages this CTA filled: no copy or commit is in flight afterwards
+        // do not leave before the MMAs have consumed the stages filled here:
+        // no copy or commit is in flight afterwards
         for (int c = issued > kStages ? issued - kStages : 0; c < issued; ++c)
             if (!tc::mbar_wait(empty(c % kStages), (c / kStages) & 1)) *abort_flag = 1;
     } else if (warp == 1 && lane == 0) {
@@ -176,10 +157,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const uint64_t bd = tc::sdesc_sw128(tileB(s, 0)) + 2 * sub;
                     tc::mma_bf16(tmem + b * 256, ad, bd, kIdesc, (kc | sub) != 0);
                 }
-                if (a.csize > 1)
-                    tc::mma_commit_mc(empty(s), cmask);
-                else
-                    tc::mma_commit(empty(s));
+                tc::mma_commit(empty(s));
             }
             tc::mma_commit(afull(b));
         }
@@ -270,11 +248,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     tc::tc_fence_before();
     __syncwarp();
-    // no CTA leaves while another may still write to its shared memory
-    if (a.csize > 1)
-        tc::cluster_sync();
-    else
-        __syncthreads();
+    __syncthreads();
     if (warp == 1) {
         tc::tc_fence_after();
         tc::tmem_dealloc(tmem, 512);
@@ -303,11 +277,6 @@ cudaError_t launch_tc_target(const CUtensorMap &mapC, const CUtensorMap &mapT, f
     if (e != cudaSuccess) return e;
     const int per = (G + nsplit - 1) / nsplit;
     const int tiles = p_pad / 128;
-    // The kernel supports clusters of 2 or 4 row tiles multicasting the digit
-    // tiles (csize); on the q_proj workload single CTAs measured faster
-    // (35.3 against 37.2 us per launch with 4): the stage lockstep of a
-    // cluster costs more than the L2 traffic it saves.
-    const int csize = 1;
     // quantum 2^-k of the exact digit split: the largest k with
     // 128 qmax 512 + 2^14 <= 2^(24-k)
     if (qmax < 1 || qmax > 255 || g > 128) return cudaErrorInvalidValue;
@@ -315,11 +284,10 @@ cudaError_t launch_tc_target(const CUtensorMap &mapC, const CUtensorMap &mapT, f
     int kq = 0;
     while (kq < 7 && bound <= std::ldexp(1.0, 24 - (kq + 1))) ++kq;
     const float round_c = (float)std::ldexp(1.5, 23 - kq);
-    TargetArgs a{out_hi, out_lo, S, expoT, active, status, p, p_pad, d_pad, g, G, i, per, csize,
+    TargetArgs a{out_hi, out_lo, S, expoT, active, status, p, p_pad, d_pad, g, G, i, per,
                  round_c};
     dim3 grid(tiles, g / 64, nsplit);
-    return launch_pdl_cluster(tc_target_kernel, grid, dim3(kThreads), (size_t)kSmem, s, csize,
-                              mapC, mapT, a);
+    return launch_pdl(tc_target_kernel, grid, dim3(kThreads), (size_t)kSmem, s, mapC, mapT, a);
 }
 
 }  // namespace jarq

@@ -1,14 +1,16 @@
 // Objective evaluation without any device allocation.
 //
 // Some callers cannot allocate device memory at the point where they need
-// the objective: code running while a CUDA graph is being captured, serving
-// processes that reserve all device memory up front and forbid later
-// cudaMalloc, and callers that must not pay the device-wide synchronisation
-// an allocation can imply.  For them jarq_objective_noalloc computes the same
-// per-row objective as jarq_objective, with every intermediate buffer taken
-// from one statically sized device array that exists on each GPU for as long
-// as the library is loaded.
+// the objective: serving processes that reserve all device memory up front
+// and forbid later cudaMalloc, and callers that must not pay the
+// device-wide synchronisation an allocation can imply.  For them
+// jarq_objective_noalloc computes the same per-row objective as
+// jarq_objective, with every intermediate buffer taken from one statically
+// sized device array that exists on each GPU for as long as the library is
+// loaded.
 //
+// The call is synchronous: it waits on the stream twice (after the code
+// check and at the end) and reads the handle's status word on the host.
 // The array is shared by all calls on a device and keeps the last call's
 // contents; the parts that must start at zero (the padding of the bf16
 // operand planes) are cleared on every call.  Calls that overlap on the GPU
@@ -78,8 +80,10 @@ extern "C" jarq_status jarq_objective_noalloc(jarq_hessian *h, const float *W, c
     const int d = h->din, d_pad = h->d_pad, g = h->g, G = h->G;
     const int p_pad = round_up(dout, 128);
     if ((size_t)p_pad * (size_t)d_pad > kNoAllocMaxElems) return JARQ_ERR_ARG;
-    if (cudaSetDevice(h->device) != cudaSuccess) return JARQ_ERR_CUDA;
-    // every buffer must already live on the device: staging would allocate
+    // the handle's device is current for the call; the caller's is restored
+    DeviceGuard dg(h->device);
+    if (!dg.ok()) return JARQ_ERR_CUDA;
+    // every buffer must already live on this device: staging would allocate
     if (!on_device(W) || !on_device(S) || !on_device(Q) || !on_device(Z) || !on_device(F_per_row))
         return JARQ_ERR_ARG;
     // once per device: the device address of the static scratch array

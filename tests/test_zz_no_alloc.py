@@ -1,12 +1,14 @@
 """The allocation-free objective entry point matches the regular one.
 
 jarq_objective_noalloc serves callers that must not allocate device memory
-when they ask for the objective (inside CUDA-graph capture, or in processes
-that reserve all device memory at start-up).  Its scratch is one static
-device array shared by every call, so the test calls it twice in a row with
-different states and checks each result against jarq_objective.  This file
-is collected last so that a run stopping at the first failure has already
-run every other test; it also passes when run alone.
+when they ask for the objective (processes that reserve all device memory at
+start-up, or that cannot afford an allocation's synchronisation).  Its
+scratch is one static device array shared by every call, so the test calls
+it twice in a row with different states and checks each result against
+jarq_objective and against the float64 oracle's objective of the same
+state, and that the device's free memory does not move during a call.  This
+file is collected last so that a run stopping at the first failure has
+already run every other test; it also passes when run alone.
 """
 import ctypes
 
@@ -41,12 +43,28 @@ def test_noalloc_objective_matches_regular_entry_point_twice():
     Q2 = states[0][1].clone()
     J.refine(hess, W, S2, Q2, Z, lay.bits, max_iters=2)
     states.append((S2, Q2))
-    for S, Q in states:                     # two calls in a row
+    from oracle import objective, prepare_hessian
+    prep = prepare_hessian(lay.H, lay.g)
+    F_bufs = [torch.full((lay.dout,), float("nan"), dtype=torch.float64, device=dev)
+              for _ in states]
+    # warm-up: the first call on a device may load the library's module,
+    # which places the static array on the GPU
+    assert _noalloc(J, hess, W, *states[0], Z, lay.bits, F_bufs[0]) == J.JARQ_OK
+    torch.cuda.synchronize()
+    for (S, Q), F in zip(states, F_bufs):   # two calls in a row
         F_ref = J.objective(hess, W, S, Q, Z, lay.bits)
-        F = torch.full((lay.dout,), float("nan"), dtype=torch.float64, device=dev)
+        torch.cuda.synchronize()
+        free0 = torch.cuda.mem_get_info()[0]
         st = _noalloc(J, hess, W, S, Q, Z, lay.bits, F)
+        free1 = torch.cuda.mem_get_info()[0]
         assert st == J.JARQ_OK, J.status_string(st)
+        # no device allocation during the call
+        assert free1 == free0, (free0, free1)
         np.testing.assert_allclose(F.cpu().numpy(), F_ref.cpu().numpy(), rtol=1e-12, atol=0)
+        # and the value itself: the oracle's float64 objective of the same state
+        F_orc = objective(prep, lay.W, S.cpu().numpy().astype(np.float64),
+                          Q.cpu().numpy(), lay.Z)
+        np.testing.assert_allclose(F.cpu().numpy(), F_orc, rtol=1e-5, atol=0)
     hess.close()
 
 
