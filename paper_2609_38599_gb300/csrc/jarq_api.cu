@@ -657,8 +657,6 @@ jarq_status refine_impl(jarq_hessian *h, const float *W, float *S, uint8_t *Q, c
     Workspace &w = h->ws;
     const int p = dout, d = h->din, g = h->g, G = h->G, qmax = (1 << bits) - 1;
     RUN("init_rows", 1, launch_init_rows(w.active, w.iters, w.accepted, w.ridge, w.rstat, p, st));
-    const ResidualView rv = rview(h);
-    const int nsplit = target_splits(w.p_pad, g, G);
     // target projection P = W H, w^T H w and the folded Pt, once per call
     RUN("slice_rows", 1, launch_slice_rows(la.W, w.wdig, w.wexp, p, d, h->d_pad, w.p_pad, g, st));
     RUN("proj", 1, launch_tc_proj(w.mapWd, h->mapD8, w.Phi, w.Plo, w.wexp, h->expo, p, w.p_pad, d,
@@ -681,14 +679,12 @@ jarq_status refine_impl(jarq_hessian *h, const float *W, float *S, uint8_t *Q, c
         RUN("scale_solve", 1, launch_scale_solve(w.gram, w.rhs, w.wHw, la.S, w.L_prev, L_out,
                                                  w.active, w.iters, w.ridge, w.rstat, h->dstatus,
                                                  p, d, g, k, false, o, st));
-        for (int i = 0; i < G; ++i) {
-            RUN("target", 1, launch_tc_target(w.mapC, h->mapHt, w.t_hi, w.t_lo, la.S, h->expoT,
-                                              w.active, p, w.p_pad, h->d_pad, g, G, i, nsplit,
-                                              qmax, h->dstatus, st));
-            RUN("babai", 1, launch_babai(w.t_hi, w.t_lo, w.Pt_hi, w.Pt_lo, nsplit, h->Lf, la.S, la.Q,
-                                         la.Z, rv, w.active, w.accepted, h->dstatus, p, g, i, qmax,
-                                         o.eps, st));
-        }
+        // the Gauss-Seidel sweep over the G groups: one launch, each row
+        // tile advancing through its phases on its own
+        RUN("sweep", 1, launch_sweep(w.mapC, h->mapHt, w.t_hi, w.t_lo, w.Pt_hi, w.Pt_lo, h->Lf,
+                                     la.S, h->expoT, la.Q, la.Z, w.cplane, w.active, w.accepted,
+                                     h->dstatus, p, w.p_pad, d, h->d_pad, g, G, qmax, o.eps,
+                                     st));
     }
     // objective of the returned state (and of the input state when K = 0)
     const bool want_final = stats && stats->L_final;

@@ -214,6 +214,13 @@ cudaError_t launch_ptilde(const CUtensorMap &mapPd, const CUtensorMap &mapR, con
                           float *out_hi, float *out_lo, int p, int p_pad, int d, int d_pad, int g,
                           int *status, cudaStream_t s);
 int target_splits(int p_pad, int g, int G);
+int sweep_k_parts(int g);
+cudaError_t launch_sweep(const CUtensorMap &mapC, const CUtensorMap &mapT, float *t_hi,
+                         float *t_lo, const float *pt_hi, const float *pt_lo, const float *Lf,
+                         const float *S, const int *expoT, uint8_t *Q, const int32_t *Z,
+                         __half *cplane, const int *active, int *accepted, int *status, int p,
+                         int p_pad, int d, int d_pad, int g, int G, int qmax, float eps,
+                         cudaStream_t s);
 cudaError_t launch_tc_target(const CUtensorMap &mapC, const CUtensorMap &mapT, float *out_hi,
                              float *out_lo, const float *S, const int *expoT, const int *active,
                              int p, int p_pad, int d_pad, int g, int G, int i, int nsplit, int qmax,
