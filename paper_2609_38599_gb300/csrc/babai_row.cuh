@@ -1,7 +1,6 @@
-// Bounded Babai proposal and acceptance for group i of one output row (Sec.
+// Bounded Babai proposal and acceptance for group i of output rows (Sec.
 // 3.3.2, Eqs. conditional_residual, group_bils, group_qr, babai_update; App.
-// E "Small scales"), executed by one warp.  Used by the per-phase Babai
-// kernel and by the fused sweep kernel.
+// E "Small scales"), executed by one warp.
 //
 // Lane l owns the NT = g/32 consecutive coordinates NT*l .. NT*l + NT - 1.
 // The group factor L_i = R_i^T (row-major g x g, float32) is in shared
@@ -78,123 +77,200 @@ __device__ __forceinline__ void load_vec_cg(const float *p, float (&v)[NT]) {
     }
 }
 
-// Proposal and acceptance for row j, group i.  Lg: L_i in shared memory;
-// rd: 1 / R_ll of this lane's coordinates.  Returns true when the row's codes
-// of group i changed.
-template <int NT>
-__device__ __forceinline__ bool babai_row(const BabaiRowArgs &a, int j, int i, const float *Lg,
-                                          const float (&rd)[NT], int lane) {
+// Proposal and acceptance of group i for R rows at once (js[r] < 0: no
+// row), their back substitutions interleaved so that one warp keeps R
+// independent dependency chains in flight.
+//
+// The scan is blocked by lanes: for lane block L (coordinates h = NT L + t)
+// the owning lane resolves its NT coordinates from the top one down, each
+// rounding followed by the column updates of its own lower coordinates with
+// the factor entries it holds in registers (Rl); then the NT changes are
+// broadcast and the lanes below L apply the NT column updates, in the same
+// descending order, from columns loaded before the broadcast.  Every u value
+// sees the same fused multiply-adds in the same order as the
+// coordinate-by-coordinate recursion (an update by a zero change leaves u
+// unchanged), so the codes are those of Eq. babai_update evaluated in that
+// order.
+//   Lg: L_i in shared memory; rd: 1 / R_ll and dg: R_ll of this lane's
+//   coordinates; Rl[t][tt] = R[l0+tt][l0+t] for tt < t (this lane's block
+//   of the factor).
+template <int NT, int R>
+__device__ __forceinline__ void babai_rows(const BabaiRowArgs &a, const int (&js)[R], int i,
+                                           const float *Lg, const float (&rd)[NT],
+                                           const float (&dg)[NT], const float (&Rl)[NT][NT],
+                                           int lane) {
     constexpr int g = 32 * NT;
     const int G = a.G, d = a.d;
     const int l0 = NT * lane;
     const int col0 = i * g;
-    if (!a.active[j]) return false;
-    const float s = a.S[(size_t)j * G + i];
-    if (!(fabsf(s) > a.eps)) return false;  // small-scale skip (also NaN)
-    const int z = a.Z[(size_t)j * G + i];
-    const size_t off = (size_t)j * d + col0;
-    // s y = Pt_i - sum_sp T_sp, in double-float
-    float y[NT], yl[NT];
-    load_vec<NT>(a.pt_hi + off + l0, y);
-    load_vec<NT>(a.pt_lo + off + l0, yl);
-    for (int sp = 0; sp < a.nsplit; ++sp) {
-        float th[NT], tl[NT];
-        const size_t o = ((size_t)sp * a.p_pad + j) * g + l0;
-        load_vec_cg<NT>(a.t_hi + o, th);
-        load_vec_cg<NT>(a.t_lo + o, tl);
+    bool live[R];
+    float s[R];
+    int z[R];
+    size_t off[R];
+    float y[R][NT], u[R][NT], qc[R][NT], qn[R][NT];
 #pragma unroll
-        for (int t = 0; t < NT; ++t) {
-            const float sm = y[t] - th[t];
-            const float bb = sm - y[t];
-            const float e = (y[t] - (sm - bb)) + (-th[t] - bb);
-            y[t] = sm;
-            yl[t] += e - tl[t];
+    for (int r = 0; r < R; ++r) {
+        const int j = js[r] >= 0 ? js[r] : 0;
+        live[r] = js[r] >= 0 && a.active[j];
+        s[r] = a.S[(size_t)j * G + i];
+        live[r] = live[r] && fabsf(s[r]) > a.eps;   // small-scale skip (also NaN)
+        z[r] = a.Z[(size_t)j * G + i];
+        off[r] = (size_t)j * d + col0;
+        // s y = Pt_i - sum_sp T_sp, in double-float
+        float yl[NT];
+        load_vec<NT>(a.pt_hi + off[r] + l0, y[r]);
+        load_vec<NT>(a.pt_lo + off[r] + l0, yl);
+        for (int sp = 0; sp < a.nsplit; ++sp) {
+            float th[NT], tl[NT];
+            const size_t o = ((size_t)sp * a.p_pad + j) * g + l0;
+            load_vec_cg<NT>(a.t_hi + o, th);
+            load_vec_cg<NT>(a.t_lo + o, tl);
+#pragma unroll
+            for (int t = 0; t < NT; ++t) {
+                const float sm = y[r][t] - th[t];
+                const float bb = sm - y[r][t];
+                const float e = (y[r][t] - (sm - bb)) + (-th[t] - bb);
+                y[r][t] = sm;
+                yl[t] += e - tl[t];
+            }
         }
-    }
-#pragma unroll
-    for (int t = 0; t < NT; ++t) y[t] += yl[t];
-    float qc[NT], qn[NT];   // current and proposed codes (small integers, exact)
-    {
         uint32_t packed = 0;
         if constexpr (NT == 4) {
-            packed = *reinterpret_cast<const uint32_t *>(a.Q + off + l0);
+            packed = *reinterpret_cast<const uint32_t *>(a.Q + off[r] + l0);
         } else {
-            packed = *reinterpret_cast<const uint16_t *>(a.Q + off + l0);
+            packed = *reinterpret_cast<const uint16_t *>(a.Q + off[r] + l0);
         }
 #pragma unroll
         for (int t = 0; t < NT; ++t) {
-            qc[t] = (float)((packed >> (8 * t)) & 0xFFu);
-            qn[t] = qc[t];
+            y[r][t] += yl[t];
+            qc[r][t] = (float)((packed >> (8 * t)) & 0xFFu);   // small integers, exact
+            qn[r][t] = qc[r][t];
         }
     }
-    // y = R^{-T} (H r)_i / s
-    float u[NT];
+    // y = R^{-T} (H r)_i / s; u = y
 #pragma unroll
-    for (int t = 0; t < NT; ++t) {
-        y[t] = y[t] / s;
-        u[t] = y[t];
-    }
+    for (int r = 0; r < R; ++r)
+#pragma unroll
+        for (int t = 0; t < NT; ++t) {
+            y[r][t] = y[r][t] / s[r];
+            u[r][t] = y[r][t];
+        }
     // back substitution (Eq. babai_update).  Rounding to the nearest even
     // integer adds and subtracts 1.5 * 2^23 (exact for |x| < 2^22; beyond
     // that the clamp to [0, qmax] gives the same code as rintf).
     const float qmaxf = (float)a.qmax;
     constexpr float kRound = 12582912.0f;      // 1.5 * 2^23
-    bool any = false;
-    // does any code change at u = y?
-    int nchg = 0;
+    bool scan[R], any[R];
+    bool scan_any = false;
 #pragma unroll
-    for (int t = 0; t < NT; ++t) {
-        const float x = fmaf(u[t], rd[t], qc[t]);
-        const float r = __fsub_rn(__fadd_rn(x, kRound), kRound);
-        nchg += fminf(fmaxf(r, 0.f), qmaxf) != qc[t];
+    for (int r = 0; r < R; ++r) {
+        // does any code change at u = y?  If not, none changes at all.
+        int nchg = 0;
+#pragma unroll
+        for (int t = 0; t < NT; ++t) {
+            const float x = fmaf(u[r][t], rd[t], qc[r][t]);
+            const float q = __fsub_rn(__fadd_rn(x, kRound), kRound);
+            nchg += fminf(fmaxf(q, 0.f), qmaxf) != qc[r][t];
+        }
+        scan[r] = __any_sync(0xffffffffu, live[r] && nchg != 0);
+        any[r] = false;
+        scan_any |= scan[r];
     }
-    if (__any_sync(0xffffffffu, nchg != 0)) {
-        // descending scan (Eq. babai_update), coordinate h = NT L + t
+    if (scan_any) {
+#pragma unroll 1
         for (int L = 31; L >= 0; --L) {
+            // columns h = NT L + t of R for this lane's coordinates, loaded
+            // before the changes are known (lanes below L only)
+            float col[NT][NT];
+            if (lane < L) {
 #pragma unroll
-            for (int t = NT - 1; t >= 0; --t) {
-                const int h = NT * L + t;
-                float dq = 0.f;
-                if (lane == L) {
-                    const float x = fmaf(u[t], rd[t], qc[t]);
-                    const float r = __fsub_rn(__fadd_rn(x, kRound), kRound);
-                    const float q = fminf(fmaxf(r, 0.f), qmaxf);
-                    dq = q - qc[t];
-                    qn[t] = q;
+                for (int t = 0; t < NT; ++t) load_vec<NT>(Lg + (NT * L + t) * g + l0, col[t]);
+            }
+            float dq[R][NT];
+#pragma unroll
+            for (int r = 0; r < R; ++r)
+#pragma unroll
+                for (int t = 0; t < NT; ++t) dq[r][t] = 0.f;
+            if (lane == L) {
+#pragma unroll
+                for (int r = 0; r < R; ++r) {
+                    if (!scan[r]) continue;
+#pragma unroll
+                    for (int t = NT - 1; t >= 0; --t) {
+                        const float x = fmaf(u[r][t], rd[t], qc[r][t]);
+                        const float q = fminf(fmaxf(__fsub_rn(__fadd_rn(x, kRound), kRound), 0.f),
+                                              qmaxf);
+                        dq[r][t] = q - qc[r][t];
+                        qn[r][t] = q;
+#pragma unroll
+                        for (int tt = 0; tt < t; ++tt)
+                            u[r][tt] = fmaf(-Rl[t][tt], dq[r][t], u[r][tt]);
+                    }
                 }
-                dq = __shfl_sync(0xffffffffu, dq, L);
-                if (dq != 0.f) {                      // warp-uniform
-                    any = true;
-                    float lr[NT];
-                    load_vec<NT>(Lg + h * g + l0, lr);   // R[l'][h] for l' = l0..
+            }
 #pragma unroll
-                    for (int tt = 0; tt < NT; ++tt)
-                        if (l0 + tt < h) u[tt] = fmaf(-lr[tt], dq, u[tt]);
+            for (int r = 0; r < R; ++r)
+#pragma unroll
+                for (int t = 0; t < NT; ++t) dq[r][t] = __shfl_sync(0xffffffffu, dq[r][t], L);
+#pragma unroll
+            for (int r = 0; r < R; ++r) {
+                bool nz = false;
+#pragma unroll
+                for (int t = 0; t < NT; ++t) nz |= dq[r][t] != 0.f;
+                if (nz) {                                   // warp-uniform
+                    any[r] = true;
+                    if (lane < L) {
+#pragma unroll
+                        for (int t = NT - 1; t >= 0; --t)
+#pragma unroll
+                            for (int tt = 0; tt < NT; ++tt)
+                                u[r][tt] = fmaf(-col[t][tt], dq[r][t], u[r][tt]);
+                    }
                 }
             }
         }
     }
-    if (!any) return false;
-    float acc = 0.f;
+    // dF = s^2 (||R Delta - y||^2 - ||y||^2) (Eq. group_bils); keep iff < 0
 #pragma unroll
-    for (int t = 0; t < NT; ++t) {
-        const float av = Lg[(l0 + t) * g + l0 + t] * (qn[t] - qc[t]) - u[t];
-        acc = fmaf(av - y[t], av + y[t], acc);
-    }
-    for (int o = 16; o; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    const float dF = s * s * acc;
-    if (!(isfinite(dF) && dF < 0.f)) return false;
+    for (int r = 0; r < R; ++r) {
+        if (!any[r]) continue;                              // warp-uniform
+        float acc = 0.f;
 #pragma unroll
-    for (int t = 0; t < NT; ++t) {
-        if (qn[t] != qc[t]) {
-            const int l = l0 + t;
-            const int qi = (int)qn[t];
-            a.Q[off + l] = (uint8_t)qi;
-            a.cplane[(size_t)j * a.d_pad + col0 + l] = __int2half_rn(qi - z);
+        for (int t = 0; t < NT; ++t) {
+            const float av = dg[t] * (qn[r][t] - qc[r][t]) - u[r][t];
+            acc = fmaf(av - y[r][t], av + y[r][t], acc);
         }
+        for (int o = 16; o; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+        const float dF = s[r] * s[r] * acc;
+        if (!(isfinite(dF) && dF < 0.f)) continue;
+        const int j = js[r];
+#pragma unroll
+        for (int t = 0; t < NT; ++t) {
+            if (qn[r][t] != qc[r][t]) {
+                const int l = l0 + t;
+                const int qi = (int)qn[r][t];
+                a.Q[off[r] + l] = (uint8_t)qi;
+                a.cplane[(size_t)j * a.d_pad + col0 + l] = __int2half_rn(qi - z[r]);
+            }
+        }
+        if (lane == 0) a.accepted[j] += 1;
     }
-    if (lane == 0) a.accepted[j] += 1;
-    return true;
+}
+
+// This lane's part of the group factor for babai_rows: 1 / R_ll, R_ll and
+// the lane's diagonal block.
+template <int NT>
+__device__ __forceinline__ void babai_lane_factor(const float *Lg, int lane, float (&rd)[NT],
+                                                  float (&dg)[NT], float (&Rl)[NT][NT]) {
+    constexpr int g = 32 * NT;
+    const int l0 = NT * lane;
+#pragma unroll
+    for (int t = 0; t < NT; ++t) {
+        dg[t] = Lg[(l0 + t) * g + l0 + t];
+        rd[t] = 1.0f / dg[t];
+#pragma unroll
+        for (int tt = 0; tt < NT; ++tt) Rl[t][tt] = tt < t ? Lg[(l0 + t) * g + l0 + tt] : 0.f;
+    }
 }
 
 }  // namespace jarq

@@ -202,11 +202,6 @@ cudaError_t launch_scale_solve(const double *gram, const double *rhs, const doub
                                int *iters, int *ridge, int *rstat, int *status, int p, int d,
                                int g, int k, bool eval_only, const jarq_options &o,
                                cudaStream_t s);
-cudaError_t launch_babai(const float *t_hi, const float *t_lo, const float *pt_hi,
-                         const float *pt_lo, int nsplit, const float *Lf, const float *S,
-                         uint8_t *Q, const int32_t *Z, ResidualView rv, const int *active,
-                         int *accepted, int *status, int p, int g, int i, int qmax, float eps,
-                         cudaStream_t s);
 cudaError_t launch_slice_rinv(const double *Rinv, __nv_bfloat16 *rdig, int *rexp, int d, int g,
                               cudaStream_t s);
 cudaError_t launch_ptilde(const CUtensorMap &mapPd, const CUtensorMap &mapR, const float *Phi,

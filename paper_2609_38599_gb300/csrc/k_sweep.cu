@@ -22,7 +22,7 @@
 //   warp 0       TMA producer (code tiles, digit tiles, the group factor)
 //   warp 1       TMEM allocation and the single-thread MMA issuer
 //   warps 2..17  drain (digit sums -> double-float partial), then Babai,
-//                two rows per warp
+//                two rows per warp with interleaved back substitutions
 // Three 48 KB pipeline stages and the 64 KB group factor fit the shared
 // memory of one SM; the 512 TMEM columns hold two 4-plane accumulators.
 //
@@ -293,15 +293,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!ok) {
                 *abort_flag = 1;
             } else {
-                const int l0 = NT * lane;
-                float rd[NT];
-#pragma unroll
-                for (int t = 0; t < NT; ++t) rd[t] = 1.0f / Lg[(l0 + t) * g + l0 + t];
-#pragma unroll 1
-                for (int rr = 0; rr < 2; ++rr) {
-                    const int j = j0 + 32 * rank + 2 * (warp - 2) + rr;
-                    if (j < a.p) babai_row<NT>(ra, j, i, Lg, rd, lane);
-                }
+                float rd[NT], dg[NT], Rl[NT][NT];
+                babai_lane_factor<NT>(Lg, lane, rd, dg, Rl);
+                const int j = j0 + 32 * rank + 2 * (warp - 2);
+                const int js[2] = {j < a.p ? j : -1, j + 1 < a.p ? j + 1 : -1};
+                babai_rows<NT, 2>(ra, js, i, Lg, rd, dg, Rl, lane);
             }
             // the accepted codes reach the next phase's tensor-map loads
             tc::fence_proxy_async_global();
