@@ -398,6 +398,7 @@ void jarq_hessian_destroy(jarq_hessian *h) {
     cudaFree(h->expo);
     cudaFree(h->Lf);
     cudaFree(h->L64);
+    cudaFree(h->Rpk);
     cudaFree(h->Rinv);
     cudaFree(h->rdig);
     cudaFree(h->rexp);
@@ -445,6 +446,7 @@ jarq_status jarq_prepare_hessian(const float *H, int din, int group_size, float 
         if ((e = make_tmap_f16(&h->mapD10, h->Hdig10, (uint64_t)4 * h->d_pad, h->d_pad, 64)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->Lf, (size_t)h->G * group_size * group_size)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->L64, (size_t)h->G * group_size * group_size)) != cudaSuccess) { rc = cuda_fail(e); break; }
+        if ((e = dalloc(&h->Rpk, (size_t)h->G * sweep_rpk_size(group_size))) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->Rinv, (size_t)h->G * group_size * group_size)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->rdig, (size_t)6 * din * group_size)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->rexp, (size_t)h->G)) != cudaSuccess) { rc = cuda_fail(e); break; }
@@ -465,6 +467,8 @@ jarq_status jarq_prepare_hessian(const float *H, int din, int group_size, float 
         { ProfScope ps("symmetrize", st); e = launch_symmetrize(Hsrc, h->Hs, h->Hplanes, din, h->d_pad, nu2, st); ps.done(); count_launches(1); }
         if (e != cudaSuccess) { rc = cuda_fail(e); break; }
         { ProfScope ps("group_factor", st); e = launch_group_factor(h->Hs, h->Lf, h->L64, h->Rinv, din, group_size, h->dstatus, st); ps.done(); count_launches(1); }
+        if (e != cudaSuccess) { rc = cuda_fail(e); break; }
+        { ProfScope ps("group_factor", st); e = launch_pack_rfactor(h->Lf, h->Rpk, h->G, group_size, st); ps.done(); count_launches(1); }
         if (e != cudaSuccess) { rc = cuda_fail(e); break; }
         { ProfScope ps("slices", st); e = launch_slice_rinv(h->Rinv, h->rdig, h->rexp, din, group_size, st); ps.done(); count_launches(1); }
         if (e != cudaSuccess) { rc = cuda_fail(e); break; }
@@ -681,7 +685,7 @@ jarq_status refine_impl(jarq_hessian *h, const float *W, float *S, uint8_t *Q, c
                                                  p, d, g, k, false, o, st));
         // the Gauss-Seidel sweep over the G groups: one launch, each row
         // tile advancing through its phases on its own
-        RUN("sweep", 1, launch_sweep(w.mapC, h->mapHt, w.t_hi, w.t_lo, w.Pt_hi, w.Pt_lo, h->Lf,
+        RUN("sweep", 1, launch_sweep(w.mapC, h->mapHt, w.t_hi, w.t_lo, w.Pt_hi, w.Pt_lo, h->Rpk,
                                      la.S, h->expoT, la.Q, la.Z, w.cplane, w.active, w.accepted,
                                      h->dstatus, p, w.p_pad, d, h->d_pad, g, G, qmax, o.eps,
                                      st));

@@ -1,6 +1,6 @@
 // One Gauss-Seidel sweep over all G groups in one launch (Sec. 3.3.2; App. E
 // "Order of updates"): for every row tile, the phase products T_i and the
-// Babai proposals of groups i = 0 .. G-1 in order.
+// bounded Babai proposals of groups i = 0 .. G-1 in order.
 //
 // Rows are independent (the objective separates over output rows, Sec. 3.3),
 // so phase i+1 of a 128-row tile needs only phase i of the same tile: the
@@ -9,30 +9,40 @@
 // the phase product
 //     T_i = sum_h s_h Ht_ih c_h          (Eq. conditional_residual, folded)
 // -- g/64 column parts of group i times 4/(g/64) parts of the K range --
-// exactly as the per-phase product kernel does (integer digit planes of the
-// folded rows Ht in fp16, exact tensor-core digit sums, double-float
-// combine), and writes its double-float partial to global memory.  A
-// cluster barrier makes the partials visible; then each CTA runs the Babai
-// proposal and acceptance (babai_row.cuh) for its 32 rows of the tile, with
-// the group factor L_i staged in shared memory by one bulk copy, writes the
-// accepted codes to Q and to the fp16 code plane, and a second cluster
-// barrier makes those codes visible to the next phase's tensor-map loads.
+// from integer digit planes of the folded rows Ht (fp16, exact tensor-core
+// digit sums, double-float combine) and writes its double-float partial to
+// global memory.  Each CTA then forms the Babai targets
+//     y = (Pt_i - T_i) / s_i = R_i^{-T} (H r)_i / s_i
+// of its 32 rows of the tile from the partials of all four, and one Babai
+// warp runs the proposal and acceptance of those 32 rows, one row per lane,
+// while the product of the next phase proceeds.
 //
-// One CTA (576 threads):
-//   warp 0       TMA producer (code tiles, digit tiles, the group factor)
+// Overlap.  Group i's codes change only in phase i, so the product of phase
+// i+1 needs phase i's result only for the K chunks of group i.  The CTA
+// whose K range holds group i takes that group last in phase i+1, and its
+// producer waits for the codes of all four Babai warps only before loading
+// it; the other K chunks, and the other CTAs, go on meanwhile.
+//
+// One CTA (608 threads):
+//   warp 0       TMA producer (code tiles, digit tiles)
 //   warp 1       TMEM allocation and the single-thread MMA issuer
-//   warps 2..17  drain (digit sums -> double-float partial), then Babai,
-//                two rows per warp with interleaved back substitutions
-// Three 48 KB pipeline stages and the 64 KB group factor fit the shared
-// memory of one SM; the 512 TMEM columns hold two 4-plane accumulators.
+//   warps 2..17  drain: digit sums -> double-float partial; then the Babai
+//                targets of two rows each, written to shared memory
+//   warp 18      Babai: 32 rows, one per lane, back substitution by blocks
+//                of 16 coordinates (its own factor R_i, bulk-copied)
+// Cluster signals: two counters in every CTA's shared memory that each of
+// the four CTAs increments once per phase (remote reductions with release
+// semantics at cluster scope; readers poll with acquire): `pcnt` -- the
+// partials of the phase are in global memory; `ccnt` -- the codes of the
+// phase are in Q and the code plane.  Phase i is complete at 4 (i + 1).
+// Counters, unlike barrier phases, may be waited for out of order: the
+// producer waits only in the phases where it holds the pending group.
 //
-// Every wait on an mbarrier is bounded; on a timeout the CTA stops issuing
-// work, keeps arriving at the cluster barriers of the remaining phases (so
-// that no CTA of its cluster waits forever), drains its own copies and MMAs
-// and reports JARQ_ERR_TIMEOUT through the status word.
+// Every wait is bounded; on a timeout the CTA stops issuing work, keeps
+// arriving at the final cluster barrier (so no CTA of its cluster waits
+// forever), drains its own copies and MMAs and reports JARQ_ERR_TIMEOUT.
 #include <cmath>
 
-#include "babai_row.cuh"
 #include "tc_common.cuh"
 
 namespace jarq {
@@ -43,17 +53,36 @@ constexpr int kTileB = 64 * 64 * 2;    // one digit plane: 64 rows of Ht x 64 K
 constexpr int kStage = kTileA + 4 * kTileB;
 constexpr int kStages = 3;
 constexpr int kCluster = 4;            // CTAs per row tile
-constexpr int kLBytes = 128 * 128 * 4; // group factor, float32, g = 128 at most
-constexpr int kBarOff = kStages * kStage + kLBytes;
-constexpr int kSmem = 1024 + kBarOff + 256;
+constexpr int kRows = 128 / kCluster;  // Babai rows per CTA (one per lane)
 constexpr uint32_t kIdesc = tc::idesc_f16_f32(128, 256);
 constexpr int kDrainWarps = 16;
-constexpr int kThreads = 32 * (2 + kDrainWarps);
+constexpr int kBabaiWarp = 2 + kDrainWarps;
+constexpr int kThreads = 32 * (kBabaiWarp + 1);
+
+// Packed rows of R_i (upper triangular, g x g): row l holds columns
+// 16 floor(l/16) .. g-1, so every row starts on a 64-byte boundary and a
+// block of 16 columns is four aligned float4.
+__host__ __device__ constexpr int rpk_row_off(int l, int g) {
+    return 16 * ((l >> 4) * g - 8 * (l >> 4) * ((l >> 4) - 1)) + (l & 15) * (g - 16 * (l >> 4));
+}
+__host__ __device__ constexpr int rpk_size(int g) { return rpk_row_off(g, g); }
+
+// shared memory (g = 128 sizes; g = 64 uses less of each)
+constexpr int kOffRpk = kStages * kStage;
+constexpr int kOffU = kOffRpk + rpk_size(128) * 4;
+constexpr int kOffY = kOffU + 128 * kRows * 4;
+constexpr int kOffC = kOffY + 128 * kRows * 4;
+constexpr int kOffRd = kOffC + 32 * kRows * 4;
+constexpr int kOffDg = kOffRd + 128 * 4;
+constexpr int kOffRow = kOffDg + 128 * 4;         // s, z, live of the 32 rows
+constexpr int kOffBar = kOffRow + 3 * kRows * 4;
+constexpr int kSmem = 1024 + kOffBar + 256;
+static_assert(kSmem <= 232448, "shared memory of one CTA");
 
 struct SweepArgs {
-    float *t_hi, *t_lo;           // [nks][p_pad][g] partials of T_i
+    float *t_hi, *t_lo;           // [2][nks][p_pad][g] partials of T_i (two phases)
     const float *pt_hi, *pt_lo;   // [p][d] folded target projection
-    const float *Lf;              // [G][g][g] L_i = R_i^T
+    const float *Rpk;             // [G][rpk_size(g)] packed factors R_i
     const float *S;               // [p][G]
     const int *expoT;             // [G][G] block exponents of Ht
     uint8_t *Q;                   // [p][d]
@@ -72,6 +101,25 @@ __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
     e = (a - (s - bb)) + (b - bb);
 }
 
+// Group of K unit u of phase i for the CTA whose K range is [h0, h0 + nseg):
+// when that range holds group i-1 (whose codes phase i-1 is still deciding),
+// the units start after it and end with it.
+__device__ __forceinline__ int unit_group(int u, int i, int h0, int nseg) {
+    const int gp = i - 1;
+    const int rot = (gp >= h0 && gp < h0 + nseg) ? gp - h0 + 1 : 0;
+    int k = rot + u;
+    if (k >= nseg) k -= nseg;
+    return h0 + k;
+}
+
+// Smem index of coordinate l of Babai row r in the u and y arrays: [l][r],
+// the row index XOR-ed with l/4 so that both the drain's writes (a row per
+// warp, l across lanes) and the Babai warp's reads (l fixed, a row per lane)
+// are free of bank conflicts.
+__device__ __forceinline__ int uy_idx(int l, int r) { return l * kRows + (r ^ ((l >> 2) & 31)); }
+// Word of the code array holding codes 4k .. 4k+3 of row r.
+__device__ __forceinline__ int c_idx(int k, int r) { return k * kRows + (r ^ (k & 31)); }
+
 template <int NT>
 __global__ void __launch_bounds__(kThreads, 1)
     sweep_kernel(const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapT,
@@ -79,11 +127,21 @@ __global__ void __launch_bounds__(kThreads, 1)
     constexpr int g = 32 * NT;
     constexpr int ncol = g / 64;            // column parts of a group
     constexpr int nkc = g / 64;             // 64-wide K chunks per group
+    constexpr int kRpk = rpk_size(g);
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    float *Lg = (float *)(smem + kStages * kStage);
-    uint64_t *bars = (uint64_t *)(smem + kBarOff);
-    uint32_t *tmem_slot = (uint32_t *)(bars + 2 * kStages + 6);
+    float *Rs = (float *)(smem + kOffRpk);
+    float *Ub = (float *)(smem + kOffU);
+    float *Yb = (float *)(smem + kOffY);
+    uint32_t *Cb = (uint32_t *)(smem + kOffC);
+    float *Rd = (float *)(smem + kOffRd);
+    float *Dg = (float *)(smem + kOffDg);
+    float *rowS = (float *)(smem + kOffRow);
+    int *rowZ = (int *)(rowS + kRows);
+    int *rowLive = rowZ + kRows;
+    uint64_t *bars = (uint64_t *)(smem + kOffBar);
+    uint32_t *tmem_slot = (uint32_t *)(bars + 2 * kStages + 9);
+    uint32_t *counters = tmem_slot + 4;   // pcnt, ccnt
     volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
     int *consumed = (int *)(tmem_slot + 2);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -98,8 +156,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto empty = [&](int s) { return tc::smem_u32(bars + kStages + s); };
     auto afull = [&](int b) { return tc::smem_u32(bars + 2 * kStages + b); };
     auto aempty = [&](int b) { return tc::smem_u32(bars + 2 * kStages + 2 + b); };
-    const uint32_t lbar = tc::smem_u32(bars + 2 * kStages + 4);
-    const uint32_t done = tc::smem_u32(bars + 2 * kStages + 5);
+    const uint32_t pcnt = tc::smem_u32(counters);       // partials, 4 per phase
+    const uint32_t ccnt = tc::smem_u32(counters + 1);   // codes, 4 per phase
+    const uint32_t ybar = tc::smem_u32(bars + 2 * kStages + 6);   // Babai targets, 16 warps
+    const uint32_t lbar = tc::smem_u32(bars + 2 * kStages + 7);   // factor copy
+    const uint32_t done = tc::smem_u32(bars + 2 * kStages + 8);
     auto tileA = [&](int s) { return tc::smem_u32(smem + s * kStage); };
     auto tileB = [&](int s, int t) { return tc::smem_u32(smem + s * kStage + kTileA + t * kTileB); };
 
@@ -112,6 +173,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc::mbar_init(afull(b), 1);
             tc::mbar_init(aempty(b), kDrainWarps);
         }
+        counters[0] = 0;
+        counters[1] = 0;
+        tc::mbar_init(ybar, kDrainWarps);
         tc::mbar_init(lbar, 1);
         tc::mbar_init(done, 1);
         *abort_flag = 0;
@@ -127,42 +191,40 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc::prefetch_tmap(&mapT);
     }
     tc::tc_fence_before();
-    __syncthreads();
+    __syncwarp();
+    // every CTA's barriers are initialised before any CTA arrives on them
+    tc::cluster_sync();
     tc::tc_fence_after();
     const uint32_t tmem = *tmem_slot;
     // scales, active rows and codes come from the preceding kernels
     tc::pdl_wait();
     tc::pdl_launch_dependents();
 
-    const BabaiRowArgs ra{a.t_hi, a.t_lo, a.pt_hi, a.pt_lo, a.nks, a.S, a.Q, a.Z, a.cplane,
-                          a.active, a.accepted, a.p_pad, a.d, a.d_pad, g, a.G, a.qmax, a.eps};
     int cp = 0;               // producer: chunks issued
-    int nl = 0;               // producer: group-factor copies issued
-    int cm = 0, um = 0;       // MMA issuer: chunks consumed, accumulator units
-    int ud = 0;               // drain: accumulator units drained
+    int cm = 0;               // MMA issuer: chunks consumed
+    int nl = 0;               // Babai warp: factor copies issued
 
-    for (int i = 0; i < a.G; ++i) {
-        if (warp == 0 && lane == 0) {
-            // ---------------- producer
-            if (!*abort_flag) {
-                // the group factor of this phase; the buffer is free, the
-                // previous phase's Babai ended before the last cluster barrier
-                tc::fence_proxy_async_smem();
-                tc::mbar_expect_tx(lbar, (uint32_t)(g * g * sizeof(float)));
-                tc::bulk_load(tc::smem_u32(Lg), a.Lf + (size_t)i * g * g, g * g * sizeof(float),
-                              lbar);
-                ++nl;
-                // codes written by the previous phase, before the tensor-map loads
-                tc::fence_proxy_async_global();
-            }
+    if (warp == 0 && lane == 0) {
+        // ------------------------------------------------ producer
+        for (int i = 0; i < a.G && !*abort_flag; ++i) {
             const int m0 = i * g + cpart * 64;    // first row of Ht (output column)
-            for (int c = 0; c < nchunks && !*abort_flag; ++c) {
+            const bool holds = i >= 1 && i - 1 >= h0 && i - 1 < h0 + nseg;
+            for (int c = 0; c < nchunks; ++c) {
+                const int u = c / nkc, kc = c % nkc;
+                if (holds && u == nseg - 1 && kc == 0) {
+                    // the last group is i-1: its codes from all four Babai warps
+                    if (!tc::wait_count_cluster(ccnt, kCluster * i)) {
+                        *abort_flag = 1;
+                        break;
+                    }
+                    tc::fence_proxy_async_global();
+                }
                 const int s = cp % kStages;
-                if (!tc::mbar_wait(empty(s), ((cp / kStages) & 1) ^ 1)) {
+                if (!tc::mbar_wait(empty(s), ((cp / kStages) & 1) ^ 1) || *abort_flag) {
                     *abort_flag = 1;
                     break;
                 }
-                const int kx = h0 * g + c * 64;
+                const int kx = unit_group(u, i, h0, nseg) * g + kc * 64;
                 tc::mbar_expect_tx(full(s), kStage);
                 tc::tma_load_2d(tileA(s), &mapC, full(s), kx, j0);
 #pragma unroll
@@ -170,11 +232,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tc::tma_load_2d(tileB(s, t), &mapT, full(s), kx, t * a.d_pad + m0);
                 ++cp;
             }
-        } else if (warp == 1 && lane == 0) {
-            // ---------------- MMA issuer: one accumulator unit per group h
-            for (int u = 0; u < nseg && !*abort_flag; ++u) {
+        }
+    } else if (warp == 1 && lane == 0) {
+        // ------------------------------------------------ MMA issuer
+        int um = 0;
+        for (int i = 0; i < a.G && !*abort_flag; ++i) {
+            for (int u = 0; u < nseg; ++u) {
                 const int b = um & 1;
-                if (!tc::mbar_wait(aempty(b), ((um >> 1) & 1) ^ 1)) {
+                if (!tc::mbar_wait(aempty(b), ((um >> 1) & 1) ^ 1) || *abort_flag) {
                     *abort_flag = 1;
                     break;
                 }
@@ -201,10 +266,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc::mma_commit(afull(b));
                 ++um;
             }
-        } else if (warp >= 2) {
-            // ---------------- drain: digits -> double-float x s_h 2^(E - 9) -> partial
-            const int q = warp & 3, cq = (warp - 2) >> 2;    // lane quarter, 16-column quarter
-            const int row = j0 + 32 * q + lane;
+        }
+    } else if (warp >= 2 && warp < kBabaiWarp) {
+        // ------------------------------------------------ drain + Babai targets
+        const int q = warp & 3, cq = (warp - 2) >> 2;    // lane quarter, 16-column quarter
+        const int row = j0 + 32 * q + lane;
+        const float *srow = a.S + (size_t)min(row, a.p - 1) * a.G;
+        const int dw = warp - 2;
+        int ud = 0;
+        for (int i = 0; i < a.G; ++i) {
             float hi[16], lo[16];
 #pragma unroll
             for (int e = 0; e < 16; ++e) {
@@ -212,17 +282,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                 lo[e] = 0.f;
             }
             bool ok = __all_sync(0xffffffffu, !*abort_flag);
-            const float *srow = a.S + (size_t)min(row, a.p - 1) * a.G;
             const int *erow = a.expoT + (size_t)i * a.G;
-            float s_next = nseg > 0 ? srow[h0] : 0.f;
-            int e_next = nseg > 0 ? erow[h0] : 0;
+            int hn = nseg > 0 ? unit_group(0, i, h0, nseg) : 0;
+            float s_next = nseg > 0 ? srow[hn] : 0.f;
+            int e_next = nseg > 0 ? erow[hn] : 0;
             for (int u = 0; u < nseg && ok; ++u) {
-                const int b = ud & 1, h = h0 + u;
+                const int b = ud & 1;
                 const float s_cur = row < a.p ? s_next : 0.f;
                 const int e_cur = e_next;
                 if (u + 1 < nseg) {
-                    s_next = srow[h + 1];
-                    e_next = erow[h + 1];
+                    hn = unit_group(u + 1, i, h0, nseg);
+                    s_next = srow[hn];
+                    e_next = erow[hn];
                 }
                 bool w = tc::mbar_wait(afull(b), (ud >> 1) & 1);
                 w = __shfl_sync(0xffffffffu, w && !*abort_flag, 0);
@@ -271,6 +342,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 ++ud;
             }
+            // partial of this CTA (slot i & 1: the targets of phase i-1 in
+            // every CTA were formed from the other slot before any CTA
+            // reaches this point of phase i+1)
+            float *th = a.t_hi + (size_t)(i & 1) * a.nks * a.p_pad * g;
+            float *tl = a.t_lo + (size_t)(i & 1) * a.nks * a.p_pad * g;
             if (ok && row < a.p) {
                 const size_t o = ((size_t)kpart * a.p_pad + row) * g + cpart * 64 + cq * 16;
 #pragma unroll
@@ -278,32 +354,237 @@ __global__ void __launch_bounds__(kThreads, 1)
                     float x[4], y[4];
 #pragma unroll
                     for (int k = 0; k < 4; ++k) two_sum(hi[e + k], lo[e + k], x[k], y[k]);
-                    *reinterpret_cast<float4 *>(a.t_hi + o + e) = make_float4(x[0], x[1], x[2], x[3]);
-                    *reinterpret_cast<float4 *>(a.t_lo + o + e) = make_float4(y[0], y[1], y[2], y[3]);
+                    *reinterpret_cast<float4 *>(th + o + e) = make_float4(x[0], x[1], x[2], x[3]);
+                    *reinterpret_cast<float4 *>(tl + o + e) = make_float4(y[0], y[1], y[2], y[3]);
                 }
             }
+            // each thread's partial is visible cluster-wide before the signal
+            tc::fence_acq_rel_cluster();
+            tc::named_bar_sync(1, 32 * kDrainWarps);
+            if (dw == 0 && lane == 0) {
+                tc::fence_acq_rel_cluster();
+                for (int r = 0; r < kCluster; ++r) tc::count_up_cluster(tc::map_cluster(pcnt, r));
+            }
+            // the Babai buffers are free once the codes of phase i-1 are out
+            bool okw = !*abort_flag;
+            if (okw && i >= 1) okw = tc::wait_count_cluster(ccnt, kCluster * i);
+            if (okw) okw = tc::wait_count_cluster(pcnt, kCluster * (i + 1));
+            okw = __all_sync(0xffffffffu, okw);
+            if (!okw) *abort_flag = 1;
+            // Babai targets of rows 2 dw, 2 dw + 1 of this CTA's 32:
+            // y = (Pt_i - sum of partials) / s in double-float
+            if (okw) {
+                const int l0 = NT * lane;
+#pragma unroll
+                for (int rr = 0; rr < 2; ++rr) {
+                    const int r = 2 * dw + rr;
+                    const int jr = j0 + kRows * rank + r;
+                    const int j = min(jr, a.p - 1);
+                    const float s = a.S[(size_t)j * a.G + i];
+                    const bool live = jr < a.p && a.active[j] != 0 && fabsf(s) > a.eps;
+                    const size_t off = (size_t)j * a.d + i * g + l0;
+                    float y[NT], yl[NT];
+                    if constexpr (NT == 4) {
+                        const float4 t0 = *reinterpret_cast<const float4 *>(a.pt_hi + off);
+                        const float4 t1 = *reinterpret_cast<const float4 *>(a.pt_lo + off);
+                        y[0] = t0.x; y[1] = t0.y; y[2] = t0.z; y[3] = t0.w;
+                        yl[0] = t1.x; yl[1] = t1.y; yl[2] = t1.z; yl[3] = t1.w;
+                    } else {
+                        const float2 t0 = *reinterpret_cast<const float2 *>(a.pt_hi + off);
+                        const float2 t1 = *reinterpret_cast<const float2 *>(a.pt_lo + off);
+                        y[0] = t0.x; y[1] = t0.y;
+                        yl[0] = t1.x; yl[1] = t1.y;
+                    }
+                    for (int sp = 0; sp < a.nks; ++sp) {
+                        const size_t o = ((size_t)sp * a.p_pad + j) * g + l0;
+                        float thv[NT], tlv[NT];
+                        if constexpr (NT == 4) {
+                            const float4 t0 = __ldcg(reinterpret_cast<const float4 *>(th + o));
+                            const float4 t1 = __ldcg(reinterpret_cast<const float4 *>(tl + o));
+                            thv[0] = t0.x; thv[1] = t0.y; thv[2] = t0.z; thv[3] = t0.w;
+                            tlv[0] = t1.x; tlv[1] = t1.y; tlv[2] = t1.z; tlv[3] = t1.w;
+                        } else {
+                            const float2 t0 = __ldcg(reinterpret_cast<const float2 *>(th + o));
+                            const float2 t1 = __ldcg(reinterpret_cast<const float2 *>(tl + o));
+                            thv[0] = t0.x; thv[1] = t0.y;
+                            tlv[0] = t1.x; tlv[1] = t1.y;
+                        }
+#pragma unroll
+                        for (int t = 0; t < NT; ++t) {
+                            const float sm = y[t] - thv[t];
+                            const float bb = sm - y[t];
+                            const float e = (y[t] - (sm - bb)) + (-thv[t] - bb);
+                            y[t] = sm;
+                            yl[t] += e - tlv[t];
+                        }
+                    }
+#pragma unroll
+                    for (int t = 0; t < NT; ++t) {
+                        const float v = live ? (y[t] + yl[t]) / s : 0.f;
+                        Yb[uy_idx(l0 + t, r)] = v;
+                        Ub[uy_idx(l0 + t, r)] = v;
+                    }
+                    // codes: one word per 4 coordinates
+                    uint32_t packed;
+                    if constexpr (NT == 4) {
+                        packed = *reinterpret_cast<const uint32_t *>(a.Q + off);
+                        Cb[c_idx(lane, r)] = packed;
+                    } else {
+                        packed = *reinterpret_cast<const uint16_t *>(a.Q + off);
+                        const uint32_t other = __shfl_down_sync(0xffffffffu, packed, 1);
+                        if ((lane & 1) == 0) Cb[c_idx(lane >> 1, r)] = packed | (other << 16);
+                    }
+                    if (lane == 0) {
+                        rowS[r] = s;
+                        rowZ[r] = a.Z[(size_t)j * a.G + i];
+                        rowLive[r] = live ? 1 : 0;
+                    }
+                }
+            }
+            __threadfence_block();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(ybar);
         }
-        __syncwarp();
-        // the partials of every CTA of the tile are in global memory
-        tc::cluster_sync();
-        if (warp >= 2) {
-            // ---------------- Babai for this CTA's 32 rows of the tile
-            bool ok = !*abort_flag && tc::mbar_wait(lbar, i & 1);
+    } else if (warp == kBabaiWarp) {
+        // ------------------------------------------------ Babai, one row per lane
+        const int r = lane;
+        const int jr = j0 + kRows * rank + r;
+        if (lane == 0) {
+            tc::mbar_expect_tx(lbar, (uint32_t)(kRpk * sizeof(float)));
+            tc::bulk_load(tc::smem_u32(Rs), a.Rpk, kRpk * sizeof(float), lbar);
+            ++nl;
+        }
+        const float qmaxf = (float)a.qmax;
+        constexpr float kRound = 12582912.0f;      // 1.5 * 2^23: rounds to nearest even
+        for (int i = 0; i < a.G; ++i) {
+            bool ok = !*abort_flag && tc::mbar_wait(ybar, i & 1) && tc::mbar_wait(lbar, i & 1);
             ok = __all_sync(0xffffffffu, ok);
             if (!ok) {
                 *abort_flag = 1;
-            } else {
-                float rd[NT], dg[NT], Rl[NT][NT];
-                babai_lane_factor<NT>(Lg, lane, rd, dg, Rl);
-                const int j = j0 + 32 * rank + 2 * (warp - 2);
-                const int js[2] = {j < a.p ? j : -1, j + 1 < a.p ? j + 1 : -1};
-                babai_rows<NT, 2>(ra, js, i, Lg, rd, dg, Rl, lane);
+                break;
             }
-            // the accepted codes reach the next phase's tensor-map loads
+            // 1 / R_ll and R_ll of the group
+#pragma unroll
+            for (int t = 0; t < NT; ++t) {
+                const int l = NT * lane + t;
+                const float dgv = Rs[rpk_row_off(l, g) + (l & 15)];
+                Dg[l] = dgv;
+                Rd[l] = 1.0f / dgv;
+            }
+            __syncwarp();
+            const bool live = rowLive[r] != 0;
+            const float s = rowS[r];
+            // back substitution (Eq. babai_update) relative to the current
+            // codes: z + x_l = q_l + u_l / R_ll with u = y - R Delta, blocks of
+            // 16 coordinates from the top; the change of the group objective
+            // (Eq. group_bils) dF = s^2 sum_l (a_l - y_l)(a_l + y_l),
+            // a_l = R_ll Delta_l - u_l, is summed as coordinates become final
+            bool any = false;
+            float acc = 0.f;
+            for (int b0 = g - 16; b0 >= 0; b0 -= 16) {
+                float u[16], dq[16];
+                uint32_t cw[4];   // current codes of the block, four per word
+#pragma unroll
+                for (int t = 0; t < 16; ++t) u[t] = Ub[uy_idx(b0 + t, r)];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) cw[k] = Cb[c_idx((b0 >> 2) + k, r)];
+                bool bany = false;
+#pragma unroll
+                for (int t = 15; t >= 0; --t) {
+                    const int l = b0 + t;
+                    const float qc = (float)((cw[t >> 2] >> (8 * (t & 3))) & 0xFFu);
+                    const float x = fmaf(u[t], Rd[l], qc);
+                    const float qv =
+                        fminf(fmaxf(__fsub_rn(__fadd_rn(x, kRound), kRound), 0.f), qmaxf);
+                    dq[t] = live ? qv - qc : 0.f;
+                    bany |= dq[t] != 0.f;
+#pragma unroll
+                    for (int tt = 0; tt < t; ++tt)
+                        u[tt] = fmaf(-Rs[rpk_row_off(b0 + tt, g) + t], dq[t], u[tt]);
+                    // coordinate l is final
+                    const float av = Dg[l] * dq[t] - u[t];
+                    const float yv = Yb[uy_idx(l, r)];
+                    acc = fmaf(av - yv, av + yv, acc);
+                }
+                any |= bany;
+                // proposed codes of the block (current code + integer change)
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    uint32_t w = 0;
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const int c = (int)((cw[k] >> (8 * e)) & 0xFFu) + (int)dq[4 * k + e];
+                        w |= (uint32_t)c << (8 * e);
+                    }
+                    Cb[c_idx((b0 >> 2) + k, r)] = w;
+                }
+                // column updates of the coordinates below the block, in
+                // descending column order
+                if (__any_sync(0xffffffffu, bany)) {
+#pragma unroll 2
+                    for (int l = 0; l < b0; ++l) {
+                        const float4 *rr = reinterpret_cast<const float4 *>(
+                            Rs + rpk_row_off(l, g) + (b0 - 16 * (l >> 4)));
+                        float rv[16];
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            const float4 v4 = rr[k];
+                            rv[4 * k] = v4.x; rv[4 * k + 1] = v4.y;
+                            rv[4 * k + 2] = v4.z; rv[4 * k + 3] = v4.w;
+                        }
+                        float ul = Ub[uy_idx(l, r)];
+#pragma unroll
+                        for (int t = 15; t >= 0; --t) ul = fmaf(-rv[t], dq[t], ul);
+                        Ub[uy_idx(l, r)] = ul;
+                    }
+                }
+            }
+            const float dF = s * s * acc;
+            const bool accept = live && any && isfinite(dF) && dF < 0.f;
+            if (accept) {
+                const int j = jr;
+                const int z = rowZ[r];
+                const size_t off = (size_t)j * a.d + i * g;
+                __half *crow = a.cplane + (size_t)j * a.d_pad + i * g;
+#pragma unroll 2
+                for (int k4 = 0; k4 < g / 16; ++k4) {
+                    uint32_t w[4];
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) w[k] = Cb[c_idx(4 * k4 + k, r)];
+                    *reinterpret_cast<uint4 *>(a.Q + off + 16 * k4) = make_uint4(w[0], w[1], w[2], w[3]);
+                    uint32_t hw[8];
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) {
+                        const uint32_t c0 = (w[k >> 1] >> (16 * (k & 1))) & 0xFFu;
+                        const uint32_t c1 = (w[k >> 1] >> (16 * (k & 1) + 8)) & 0xFFu;
+                        const __half h0v = __int2half_rn((int)c0 - z);
+                        const __half h1v = __int2half_rn((int)c1 - z);
+                        hw[k] = (uint32_t)__half_as_ushort(h0v) | ((uint32_t)__half_as_ushort(h1v) << 16);
+                    }
+                    uint4 *cdst = reinterpret_cast<uint4 *>(crow + 16 * k4);
+                    cdst[0] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+                    cdst[1] = make_uint4(hw[4], hw[5], hw[6], hw[7]);
+                }
+                a.accepted[j] += 1;
+            }
+            // the accepted codes reach the other CTAs' tensor-map loads
             tc::fence_proxy_async_global();
+            tc::fence_acq_rel_cluster();
+            __syncwarp();
+            if (lane == 0) {
+                if (i + 1 < a.G) {
+                    // the next group's factor (this phase is done with the buffer)
+                    tc::fence_proxy_async_smem();
+                    tc::mbar_expect_tx(lbar, (uint32_t)(kRpk * sizeof(float)));
+                    tc::bulk_load(tc::smem_u32(Rs), a.Rpk + (size_t)(i + 1) * kRpk,
+                                  kRpk * sizeof(float), lbar);
+                    ++nl;
+                }
+                tc::fence_acq_rel_cluster();
+                for (int rk = 0; rk < kCluster; ++rk) tc::count_up_cluster(tc::map_cluster(ccnt, rk));
+            }
+            __syncwarp();
         }
-        __syncwarp();
-        tc::cluster_sync();
     }
 
     // ---------------- teardown: nothing of this CTA may be in flight
@@ -317,10 +598,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         // copies issued but never consumed (after a timeout)
         for (int c = *consumed; c < cp; ++c)
             if (!tc::mbar_wait(full(c % kStages), (c / kStages) & 1)) *abort_flag = 1;
-        if (nl > 0 && !tc::mbar_wait(lbar, (nl - 1) & 1)) *abort_flag = 1;
+    }
+    if (warp == kBabaiWarp && lane == 0 && nl > 0) {
+        if (!tc::mbar_wait(lbar, (nl - 1) & 1)) *abort_flag = 1;
     }
     tc::tc_fence_before();
-    __syncthreads();
+    __syncwarp();
+    // no CTA leaves while another may still arrive on its barriers
+    tc::cluster_sync();
     if (warp == 1) {
         tc::tc_fence_after();
         tc::tmem_dealloc(tmem, 512);
@@ -330,12 +615,30 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 }  // namespace
 
-// Parts of the K range of the sweep's phase products: the four CTAs of a
-// row tile are (g/64 column parts) x (K parts).
 int sweep_k_parts(int g) { return kCluster / (g / 64); }
 
+int sweep_rpk_size(int g) { return rpk_size(g); }
+
+// R_i in the packed row layout of the sweep kernel, from L_i = R_i^T
+// (row-major); entries left of the diagonal are zero.
+__global__ void pack_rfactor_kernel(const float *__restrict__ Lf, float *__restrict__ Rpk, int g) {
+    const int i = blockIdx.x;
+    const float *L = Lf + (size_t)i * g * g;
+    float *out = Rpk + (size_t)i * rpk_size(g);
+    for (int l = threadIdx.y; l < g; l += blockDim.y) {
+        const int c0 = 16 * (l >> 4);
+        for (int h = c0 + threadIdx.x; h < g; h += blockDim.x)
+            out[rpk_row_off(l, g) + (h - c0)] = h >= l ? L[(size_t)h * g + l] : 0.f;
+    }
+}
+
+cudaError_t launch_pack_rfactor(const float *Lf, float *Rpk, int G, int g, cudaStream_t s) {
+    pack_rfactor_kernel<<<G, dim3(32, 8), 0, s>>>(Lf, Rpk, g);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_sweep(const CUtensorMap &mapC, const CUtensorMap &mapT, float *t_hi,
-                         float *t_lo, const float *pt_hi, const float *pt_lo, const float *Lf,
+                         float *t_lo, const float *pt_hi, const float *pt_lo, const float *Rpk,
                          const float *S, const int *expoT, uint8_t *Q, const int32_t *Z,
                          __half *cplane, const int *active, int *accepted, int *status, int p,
                          int p_pad, int d, int d_pad, int g, int G, int qmax, float eps,
@@ -349,7 +652,7 @@ cudaError_t launch_sweep(const CUtensorMap &mapC, const CUtensorMap &mapT, float
     int kq = 0;
     while (kq < 7 && bound <= std::ldexp(1.0, 24 - (kq + 1))) ++kq;
     const float round_c = (float)std::ldexp(1.5, 23 - kq);
-    SweepArgs a{t_hi, t_lo, pt_hi, pt_lo, Lf, S, expoT, Q, Z, cplane, active, accepted, status,
+    SweepArgs a{t_hi, t_lo, pt_hi, pt_lo, Rpk, S, expoT, Q, Z, cplane, active, accepted, status,
                 p, p_pad, d, d_pad, G, qmax, nks, seg, eps, round_c};
     const dim3 grid((p_pad / 128) * kCluster);
     if (g == 128) {

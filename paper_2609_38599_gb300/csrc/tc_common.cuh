@@ -78,6 +78,38 @@ __device__ __forceinline__ void cluster_sync() {
                  "barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
+// Address of the same shared-memory location in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t map_cluster(uint32_t addr, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+    return r;
+}
+// Add 1 to a counter in the shared memory of any CTA of the cluster (address
+// from map_cluster), releasing this thread's prior writes at cluster scope.
+__device__ __forceinline__ void count_up_cluster(uint32_t cluster_addr) {
+    asm volatile("red.release.cluster.shared::cluster.add.u32 [%0], 1;" ::"r"(cluster_addr)
+                 : "memory");
+}
+// Wait (bounded) until a local counter that CTAs of the cluster increment
+// reaches `target`, acquiring their writes at cluster scope.  Counters only
+// grow, so a waiter may skip any number of increments.
+__device__ __forceinline__ bool wait_count_cluster(uint32_t addr, uint32_t target) {
+#pragma unroll 1
+    for (uint32_t i = 0; i < kWaitIters; ++i) {
+        uint32_t v;
+        asm volatile("ld.acquire.cluster.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
+        if (v >= target) return true;
+    }
+    return false;
+}
+__device__ __forceinline__ void fence_acq_rel_cluster() {
+    asm volatile("fence.acq_rel.cluster;" ::: "memory");
+}
+// Barrier over the `nthreads` threads (a multiple of 32) that name barrier `id`.
+__device__ __forceinline__ void named_bar_sync(uint32_t id, uint32_t nthreads) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
 // Proxy fences: order this thread's generic-proxy accesses of global (or
 // shared) memory before its later async-proxy (TMA) accesses and vice versa.
 __device__ __forceinline__ void fence_proxy_async_global() {
