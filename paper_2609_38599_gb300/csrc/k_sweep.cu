@@ -11,25 +11,31 @@
 // -- g/64 column parts of group i times 4/(g/64) parts of the K range --
 // from integer digit planes of the folded rows Ht (fp16, exact tensor-core
 // digit sums, double-float combine) and writes its double-float partial to
-// global memory.  Each CTA then forms the Babai targets
+// global memory.  Each CTA then runs the Babai proposals of its 32 rows of
+// the tile on the targets
 //     y = (Pt_i - T_i) / s_i = R_i^{-T} (H r)_i / s_i
-// of its 32 rows of the tile from the partials of all four, and one Babai
-// warp runs the proposal and acceptance of those 32 rows, one row per lane,
-// while the product of the next phase proceeds.
+// formed from the partials of all four CTAs.
+//
+// Babai (Eq. babai_update) is systolic over the 16 drain warps: lane r holds
+// row r of the CTA's 32, warp w holds coordinates [w CB, (w+1) CB) of the
+// group (CB = g/16).  Warp 15 resolves its coordinates first and hands the
+// code changes down through shared memory; warp w applies the column
+// updates of every higher block in descending column order as they arrive,
+// then resolves its own block from the top.  Each u_l thus sees the same
+// fused multiply-adds in the same order as the coordinate-by-coordinate
+// recursion.  The change of the group objective (Eq. group_bils) is summed
+// per warp and reduced over the warps per row; a proposal is kept iff it is
+// finite and below zero (an unchanged row gives exactly zero).
 //
 // Overlap.  Group i's codes change only in phase i, so the product of phase
 // i+1 needs phase i's result only for the K chunks of group i.  The CTA
 // whose K range holds group i takes that group last in phase i+1, and its
-// producer waits for the codes of all four Babai warps only before loading
-// it; the other K chunks, and the other CTAs, go on meanwhile.
+// producer waits for the codes of all four CTAs only before loading it.
 //
-// One CTA (608 threads):
+// One CTA (576 threads):
 //   warp 0       TMA producer (code tiles, digit tiles)
 //   warp 1       TMEM allocation and the single-thread MMA issuer
-//   warps 2..17  drain: digit sums -> double-float partial; then the Babai
-//                targets of two rows each, written to shared memory
-//   warp 18      Babai: 32 rows, one per lane, back substitution by blocks
-//                of 16 coordinates (its own factor R_i, bulk-copied)
+//   warps 2..17  drain (digit sums -> double-float partial), then Babai
 // Cluster signals: two counters in every CTA's shared memory that each of
 // the four CTAs increments once per phase (remote reductions with release
 // semantics at cluster scope; readers poll with acquire): `pcnt` -- the
@@ -56,12 +62,10 @@ constexpr int kCluster = 4;            // CTAs per row tile
 constexpr int kRows = 128 / kCluster;  // Babai rows per CTA (one per lane)
 constexpr uint32_t kIdesc = tc::idesc_f16_f32(128, 256);
 constexpr int kDrainWarps = 16;
-constexpr int kBabaiWarp = 2 + kDrainWarps;
-constexpr int kThreads = 32 * (kBabaiWarp + 1);
+constexpr int kThreads = 32 * (2 + kDrainWarps);
 
 // Packed rows of R_i (upper triangular, g x g): row l holds columns
-// 16 floor(l/16) .. g-1, so every row starts on a 64-byte boundary and a
-// block of 16 columns is four aligned float4.
+// 16 floor(l/16) .. g-1, so every row starts on a 64-byte boundary.
 __host__ __device__ constexpr int rpk_row_off(int l, int g) {
     return 16 * ((l >> 4) * g - 8 * (l >> 4) * ((l >> 4) - 1)) + (l & 15) * (g - 16 * (l >> 4));
 }
@@ -69,14 +73,13 @@ __host__ __device__ constexpr int rpk_size(int g) { return rpk_row_off(g, g); }
 
 // shared memory (g = 128 sizes; g = 64 uses less of each)
 constexpr int kOffRpk = kStages * kStage;
-constexpr int kOffU = kOffRpk + rpk_size(128) * 4;
-constexpr int kOffY = kOffU + 128 * kRows * 4;
-constexpr int kOffC = kOffY + 128 * kRows * 4;
-constexpr int kOffRd = kOffC + 32 * kRows * 4;
-constexpr int kOffDg = kOffRd + 128 * 4;
-constexpr int kOffRow = kOffDg + 128 * 4;         // s, z, live of the 32 rows
-constexpr int kOffBar = kOffRow + 3 * kRows * 4;
-constexpr int kSmem = 1024 + kOffBar + 256;
+constexpr int kOffYs = kOffRpk + rpk_size(128) * 4;   // targets / code changes [g][32]
+constexpr int kOffCs = kOffYs + 128 * kRows * 4;       // codes [g/4][32] words
+constexpr int kOffRow = kOffCs + 32 * kRows * 4;       // s, z, live of the 32 rows
+constexpr int kOffFp = kOffRow + 3 * kRows * 4;        // dF parts [16 warps][32]
+constexpr int kOffRd = kOffFp + kDrainWarps * kRows * 4;   // 1 / R_ll [g]
+constexpr int kOffBar = kOffRd + 128 * 4;
+constexpr int kSmem = 1024 + kOffBar + 512;
 static_assert(kSmem <= 232448, "shared memory of one CTA");
 
 struct SweepArgs {
@@ -112,13 +115,229 @@ __device__ __forceinline__ int unit_group(int u, int i, int h0, int nseg) {
     return h0 + k;
 }
 
-// Smem index of coordinate l of Babai row r in the u and y arrays: [l][r],
-// the row index XOR-ed with l/4 so that both the drain's writes (a row per
-// warp, l across lanes) and the Babai warp's reads (l fixed, a row per lane)
-// are free of bank conflicts.
-__device__ __forceinline__ int uy_idx(int l, int r) { return l * kRows + (r ^ ((l >> 2) & 31)); }
-// Word of the code array holding codes 4k .. 4k+3 of row r.
-__device__ __forceinline__ int c_idx(int k, int r) { return k * kRows + (r ^ (k & 31)); }
+// Shared-memory layout of the Babai exchange: per coordinate l a row of 32
+// slots (one per Babai row r), the row index XOR-ed with l/4 so that both the
+// target formation (a row per warp, l across lanes) and the systolic stage
+// (l fixed, a row per lane) are free of bank conflicts.  Ys holds the
+// targets y, then, once block w has consumed its own, that block's code
+// changes.  Cs holds the current codes, four per word.
+__device__ __forceinline__ int ys_idx(int l, int r) { return l * kRows + (r ^ ((l >> 2) & 31)); }
+__device__ __forceinline__ int cs_idx(int k, int r) { return k * kRows + (r ^ (k & 31)); }
+
+// Babai targets y = (Pt_i - sum of partials) / s of rows 2 dw, 2 dw + 1 of
+// the CTA's 32 (double-float until the subtraction is done), coalesced: a
+// row per warp, NT consecutive coordinates per lane.  Also the row's codes
+// and its scale, zero point and whether it takes a proposal.
+template <int NT>
+__device__ __forceinline__ void form_targets(const SweepArgs &a, float *Ys, uint32_t *Cs,
+                                             float *rowS, int *rowZ, int *rowLive, int i,
+                                             int dw, int lane, int jb, const float *th,
+                                             const float *tl, bool ok) {
+    constexpr int g = 32 * NT;
+    constexpr int nks = kCluster / (g / 64);   // K parts of the phase product
+    const int l0 = NT * lane;
+#pragma unroll
+    for (int rr = 0; rr < 2; ++rr) {
+        const int r = 2 * dw + rr;
+        const int jr = jb + r;
+        const int j = min(jr, a.p - 1);
+        const float s = a.S[(size_t)j * a.G + i];
+        const bool live = ok && jr < a.p && a.active[j] != 0 && fabsf(s) > a.eps;
+        const size_t off = (size_t)j * a.d + i * g + l0;
+        float y[NT], yl[NT];
+        if constexpr (NT == 4) {
+            const float4 t0 = *reinterpret_cast<const float4 *>(a.pt_hi + off);
+            const float4 t1 = *reinterpret_cast<const float4 *>(a.pt_lo + off);
+            y[0] = t0.x; y[1] = t0.y; y[2] = t0.z; y[3] = t0.w;
+            yl[0] = t1.x; yl[1] = t1.y; yl[2] = t1.z; yl[3] = t1.w;
+        } else {
+            const float2 t0 = *reinterpret_cast<const float2 *>(a.pt_hi + off);
+            const float2 t1 = *reinterpret_cast<const float2 *>(a.pt_lo + off);
+            y[0] = t0.x; y[1] = t0.y;
+            yl[0] = t1.x; yl[1] = t1.y;
+        }
+#pragma unroll
+        for (int sp = 0; sp < nks; ++sp) {
+            const size_t o = ((size_t)sp * a.p_pad + j) * g + l0;
+            float hv[NT], lv[NT];
+            if constexpr (NT == 4) {
+                const float4 h4 = __ldcg(reinterpret_cast<const float4 *>(th + o));
+                const float4 l4 = __ldcg(reinterpret_cast<const float4 *>(tl + o));
+                hv[0] = h4.x; hv[1] = h4.y; hv[2] = h4.z; hv[3] = h4.w;
+                lv[0] = l4.x; lv[1] = l4.y; lv[2] = l4.z; lv[3] = l4.w;
+            } else {
+                const float2 h2 = __ldcg(reinterpret_cast<const float2 *>(th + o));
+                const float2 l2 = __ldcg(reinterpret_cast<const float2 *>(tl + o));
+                hv[0] = h2.x; hv[1] = h2.y;
+                lv[0] = l2.x; lv[1] = l2.y;
+            }
+#pragma unroll
+            for (int e = 0; e < NT; ++e) {
+                const float sm = y[e] - hv[e];
+                const float bb = sm - y[e];
+                const float er = (y[e] - (sm - bb)) + (-hv[e] - bb);
+                y[e] = sm;
+                yl[e] += er - lv[e];
+            }
+        }
+#pragma unroll
+        for (int e = 0; e < NT; ++e) Ys[ys_idx(l0 + e, r)] = live ? (y[e] + yl[e]) / s : 0.f;
+        if constexpr (NT == 4) {
+            Cs[cs_idx(lane, r)] = *reinterpret_cast<const uint32_t *>(a.Q + off);
+        } else {
+            const uint32_t mine = *reinterpret_cast<const uint16_t *>(a.Q + off);
+            const uint32_t next = __shfl_down_sync(0xffffffffu, mine, 1);
+            if ((lane & 1) == 0) Cs[cs_idx(lane >> 1, r)] = mine | (next << 16);
+        }
+        if (lane == 0) {
+            rowS[r] = s;
+            rowZ[r] = a.Z[(size_t)j * a.G + i];
+            rowLive[r] = live ? 1 : 0;
+        }
+    }
+}
+
+// Systolic Babai for group i of the CTA's 32 rows (row r = lane) on the CB
+// coordinates of block w (warp), from the targets and codes in Ys and Cs.
+// Rs: packed R_i; Fp: per-warp dF parts [w][r]; blk: one flag per block, set
+// to i + 1 when the block's code changes of phase i are in Ys.  ok: every
+// earlier wait succeeded (else only the hand-off protocol is kept).
+template <int NT>
+__device__ __forceinline__ void babai_block(const SweepArgs &a, const float *Rs, float *Rds, float *Ys,
+                                            const uint32_t *Cs, const float *rowS,
+                                            const int *rowZ, const int *rowLive, float *Fp,
+                                            uint32_t *blk, int i, int w, int lane, int jb,
+                                            bool ok) {
+    constexpr int g = 32 * NT;
+    constexpr int CB = g / 16;              // coordinates per warp
+    const int c0 = w * CB;
+    const int r = lane;
+    const bool live = rowLive[r] != 0;
+    // this block's part of the factor: Rs[ro0 + tt rs + h] is R[c0 + tt][h]
+    // (the block's rows lie in one 16-row band of the packed layout); the
+    // diagonal and its reciprocals
+    const int ro0 = rpk_row_off(c0, g) - 16 * (c0 >> 4);
+    const int rs = g - 16 * (c0 >> 4);
+    // reciprocals of this block's diagonal, kept in shared memory (Rds) so
+    // that they occupy no registers while the block waits
+    if (lane < CB) Rds[c0 + lane] = 1.0f / Rs[ro0 + lane * rs + c0 + lane];
+    __syncwarp();
+    uint32_t cw[CB / 4];   // current codes, four per word
+#pragma unroll
+    for (int k = 0; k < CB / 4; ++k) cw[k] = Cs[cs_idx(c0 / 4 + k, r)];
+    auto qc = [&](int t) { return (float)((cw[t >> 2] >> (8 * (t & 3))) & 0xFFu); };
+    float u[CB], dq[CB];
+#pragma unroll
+    for (int t = 0; t < CB; ++t) u[t] = Ys[ys_idx(c0 + t, r)];
+    // tri[tt][t] = R[c0 + tt][c0 + t], t > tt: loaded just before the block
+    // above hands over (it is not needed earlier)
+    float tri[CB][CB];
+    auto load_tri = [&]() {
+#pragma unroll
+        for (int tt = 0; tt < CB - 1; ++tt) {
+#pragma unroll
+            for (int k = tt & ~3; k < CB; k += 4) {
+                const float4 v4 = *reinterpret_cast<const float4 *>(Rs + ro0 + tt * rs + c0 + k);
+                tri[tt][k] = v4.x; tri[tt][k + 1] = v4.y; tri[tt][k + 2] = v4.z; tri[tt][k + 3] = v4.w;
+            }
+        }
+    };
+    // column updates from every higher block, descending (per coordinate the
+    // columns in descending order)
+    for (int b = kDrainWarps - 1; b > w; --b) {
+        if (!tc::flag_wait(tc::smem_u32(blk + b), (uint32_t)(i + 1), b > w + 1)) ok = false;
+        float dv[CB];
+#pragma unroll
+        for (int t = 0; t < CB; ++t) dv[t] = Ys[ys_idx(b * CB + t, r)];
+#pragma unroll
+        for (int tt = 0; tt < CB; ++tt) {
+            float rv[CB];
+#pragma unroll
+            for (int k = 0; k < CB; k += 4) {
+                const float4 v4 = *reinterpret_cast<const float4 *>(Rs + ro0 + tt * rs + b * CB + k);
+                rv[k] = v4.x; rv[k + 1] = v4.y; rv[k + 2] = v4.z; rv[k + 3] = v4.w;
+            }
+#pragma unroll
+            for (int t = CB - 1; t >= 0; --t) u[tt] = fmaf(-rv[t], dv[t], u[tt]);
+        }
+    }
+    // own block, from the top (Eq. babai_update); the change of the group
+    // objective is summed as coordinates become final (Eq. group_bils).
+    load_tri();
+    const float qmaxf = (float)a.qmax;
+    constexpr float kRound = 12582912.0f;   // 1.5 * 2^23: rounds to nearest even
+    // everything off the dependency chain first: the current codes as
+    // floats and the reciprocals with a row that takes no proposal folded in
+    // (1 / R_ll = 0 keeps x = q, hence no change)
+    float rd[CB];
+#pragma unroll
+    for (int t = 0; t < CB; ++t) rd[t] = live ? Rds[c0 + t] : 0.f;
+#pragma unroll
+    for (int t = CB - 1; t >= 0; --t) {
+        const float qf = qc(t);
+        const float x = fmaf(u[t], rd[t], qf);
+        const float qv = fminf(fmaxf(__fsub_rn(__fadd_rn(x, kRound), kRound), 0.f), qmaxf);
+        dq[t] = qv - qf;
+        // the next coordinate's update first: it is on the chain
+        if (t > 0) u[t - 1] = fmaf(-tri[t - 1][t], dq[t], u[t - 1]);
+#pragma unroll
+        for (int tt = 0; tt + 1 < t; ++tt) u[tt] = fmaf(-tri[tt][t], dq[t], u[tt]);
+    }
+    // the block's part of the change of the group objective, with every u
+    // now final (targets read before the changes replace them)
+    float yv[CB];
+#pragma unroll
+    for (int t = 0; t < CB; ++t) yv[t] = Ys[ys_idx(c0 + t, r)];
+    // the block's changes replace its targets and go to the blocks below
+#pragma unroll
+    for (int t = 0; t < CB; ++t) Ys[ys_idx(c0 + t, r)] = dq[t];
+    __syncwarp();
+    if (lane == 0) tc::flag_store_release(tc::smem_u32(blk + w), (uint32_t)(i + 1));
+    float acc = 0.f;
+#pragma unroll
+    for (int t = CB - 1; t >= 0; --t) {
+        const float av = Rs[ro0 + t * rs + c0 + t] * dq[t] - u[t];
+        acc = fmaf(av - yv[t], av + yv[t], acc);
+    }
+    Fp[w * kRows + r] = acc;
+    // every block's dF part of this row
+    tc::named_bar_sync(1, 32 * kDrainWarps);
+    float F = 0.f;
+#pragma unroll
+    for (int b = kDrainWarps - 1; b >= 0; --b) F += Fp[b * kRows + r];
+    const float s = rowS[r];
+    const float dF = s * s * F;
+    const int jr = jb + r;
+    if (ok && live && isfinite(dF) && dF < 0.f) {
+        const int j = jr;
+        const int z = rowZ[r];
+        const size_t off = (size_t)j * a.d + i * g + c0;
+        uint32_t nw[CB / 4];
+#pragma unroll
+        for (int k = 0; k < CB / 4; ++k) {
+            uint32_t v = 0;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) v |= (uint32_t)((int)qc(4 * k + e) + (int)dq[4 * k + e]) << (8 * e);
+            nw[k] = v;
+        }
+        uint32_t hw[CB / 2];
+#pragma unroll
+        for (int k = 0; k < CB / 2; ++k) {
+            const int qa = (int)qc(2 * k) + (int)dq[2 * k], qb = (int)qc(2 * k + 1) + (int)dq[2 * k + 1];
+            hw[k] = (uint32_t)__half_as_ushort(__int2half_rn(qa - z)) |
+                    ((uint32_t)__half_as_ushort(__int2half_rn(qb - z)) << 16);
+        }
+        __half *crow = a.cplane + (size_t)j * a.d_pad + i * g + c0;
+        if constexpr (CB == 8) {
+            *reinterpret_cast<uint2 *>(a.Q + off) = make_uint2(nw[0], nw[1]);
+            *reinterpret_cast<uint4 *>(crow) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+        } else {
+            *reinterpret_cast<uint32_t *>(a.Q + off) = nw[0];
+            *reinterpret_cast<uint2 *>(crow) = make_uint2(hw[0], hw[1]);
+        }
+        if (w == 0) a.accepted[j] += 1;
+    }
+}
 
 template <int NT>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -131,16 +350,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     float *Rs = (float *)(smem + kOffRpk);
-    float *Ub = (float *)(smem + kOffU);
-    float *Yb = (float *)(smem + kOffY);
-    uint32_t *Cb = (uint32_t *)(smem + kOffC);
-    float *Rd = (float *)(smem + kOffRd);
-    float *Dg = (float *)(smem + kOffDg);
+    float *Ys = (float *)(smem + kOffYs);
+    uint32_t *Cs = (uint32_t *)(smem + kOffCs);
     float *rowS = (float *)(smem + kOffRow);
     int *rowZ = (int *)(rowS + kRows);
     int *rowLive = rowZ + kRows;
+    float *Fp = (float *)(smem + kOffFp);
+    float *Rds = (float *)(smem + kOffRd);
     uint64_t *bars = (uint64_t *)(smem + kOffBar);
-    uint32_t *tmem_slot = (uint32_t *)(bars + 2 * kStages + 9);
+    uint32_t *blk = (uint32_t *)(bars + 2 * kStages + 6);   // one flag per Babai block
+    uint32_t *tmem_slot = blk + kDrainWarps;
     uint32_t *counters = tmem_slot + 4;   // pcnt, ccnt
     volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
     int *consumed = (int *)(tmem_slot + 2);
@@ -158,9 +377,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto aempty = [&](int b) { return tc::smem_u32(bars + 2 * kStages + 2 + b); };
     const uint32_t pcnt = tc::smem_u32(counters);       // partials, 4 per phase
     const uint32_t ccnt = tc::smem_u32(counters + 1);   // codes, 4 per phase
-    const uint32_t ybar = tc::smem_u32(bars + 2 * kStages + 6);   // Babai targets, 16 warps
-    const uint32_t lbar = tc::smem_u32(bars + 2 * kStages + 7);   // factor copy
-    const uint32_t done = tc::smem_u32(bars + 2 * kStages + 8);
+    const uint32_t lbar = tc::smem_u32(bars + 2 * kStages + 4);   // factor copy
+    const uint32_t done = tc::smem_u32(bars + 2 * kStages + 5);
     auto tileA = [&](int s) { return tc::smem_u32(smem + s * kStage); };
     auto tileB = [&](int s, int t) { return tc::smem_u32(smem + s * kStage + kTileA + t * kTileB); };
 
@@ -175,7 +393,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         counters[0] = 0;
         counters[1] = 0;
-        tc::mbar_init(ybar, kDrainWarps);
+        for (int b = 0; b < kDrainWarps; ++b) blk[b] = 0;
         tc::mbar_init(lbar, 1);
         tc::mbar_init(done, 1);
         *abort_flag = 0;
@@ -202,13 +420,21 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     int cp = 0;               // producer: chunks issued
     int cm = 0;               // MMA issuer: chunks consumed
-    int nl = 0;               // Babai warp: factor copies issued
+    int nl = 0;               // drain leader: factor copies issued
 
     if (warp == 0 && lane == 0) {
         // ------------------------------------------------ producer
         for (int i = 0; i < a.G && !*abort_flag; ++i) {
             const int m0 = i * g + cpart * 64;    // first row of Ht (output column)
             const bool holds = i >= 1 && i - 1 >= h0 && i - 1 < h0 + nseg;
+            // the folded projection of this CTA's Babai rows for group i,
+            // read when the phase's targets are formed
+            for (int r = 0; r < kRows; ++r) {
+                const int j = j0 + kRows * rank + r;
+                if (j >= a.p) break;
+                tc::prefetch_l2(a.pt_hi + (size_t)j * a.d + i * g, g * sizeof(float));
+                tc::prefetch_l2(a.pt_lo + (size_t)j * a.d + i * g, g * sizeof(float));
+            }
             for (int c = 0; c < nchunks; ++c) {
                 const int u = c / nkc, kc = c % nkc;
                 if (holds && u == nseg - 1 && kc == 0) {
@@ -267,13 +493,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                 ++um;
             }
         }
-    } else if (warp >= 2 && warp < kBabaiWarp) {
+    } else if (warp >= 2) {
         // ------------------------------------------------ drain + Babai targets
         const int q = warp & 3, cq = (warp - 2) >> 2;    // lane quarter, 16-column quarter
         const int row = j0 + 32 * q + lane;
         const float *srow = a.S + (size_t)min(row, a.p - 1) * a.G;
         const int dw = warp - 2;
         int ud = 0;
+        if (dw == 0 && lane == 0) {
+            // the factor of group 0
+            tc::mbar_expect_tx(lbar, (uint32_t)(kRpk * sizeof(float)));
+            tc::bulk_load(tc::smem_u32(Rs), a.Rpk, kRpk * sizeof(float), lbar);
+            ++nl;
+        }
         for (int i = 0; i < a.G; ++i) {
             float hi[16], lo[16];
 #pragma unroll
@@ -365,226 +597,37 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc::fence_acq_rel_cluster();
                 for (int r = 0; r < kCluster; ++r) tc::count_up_cluster(tc::map_cluster(pcnt, r));
             }
-            // the Babai buffers are free once the codes of phase i-1 are out
+            // Babai of this CTA's 32 rows of the tile (one per lane) for
+            // the CB coordinates of this warp's block, once the partials of
+            // all four CTAs are out and the factor R_i is in shared memory
             bool okw = !*abort_flag;
-            if (okw && i >= 1) okw = tc::wait_count_cluster(ccnt, kCluster * i);
             if (okw) okw = tc::wait_count_cluster(pcnt, kCluster * (i + 1));
+            if (okw) okw = tc::mbar_wait(lbar, i & 1);
             okw = __all_sync(0xffffffffu, okw);
             if (!okw) *abort_flag = 1;
-            // Babai targets of rows 2 dw, 2 dw + 1 of this CTA's 32:
-            // y = (Pt_i - sum of partials) / s in double-float
-            if (okw) {
-                const int l0 = NT * lane;
-#pragma unroll
-                for (int rr = 0; rr < 2; ++rr) {
-                    const int r = 2 * dw + rr;
-                    const int jr = j0 + kRows * rank + r;
-                    const int j = min(jr, a.p - 1);
-                    const float s = a.S[(size_t)j * a.G + i];
-                    const bool live = jr < a.p && a.active[j] != 0 && fabsf(s) > a.eps;
-                    const size_t off = (size_t)j * a.d + i * g + l0;
-                    float y[NT], yl[NT];
-                    if constexpr (NT == 4) {
-                        const float4 t0 = *reinterpret_cast<const float4 *>(a.pt_hi + off);
-                        const float4 t1 = *reinterpret_cast<const float4 *>(a.pt_lo + off);
-                        y[0] = t0.x; y[1] = t0.y; y[2] = t0.z; y[3] = t0.w;
-                        yl[0] = t1.x; yl[1] = t1.y; yl[2] = t1.z; yl[3] = t1.w;
-                    } else {
-                        const float2 t0 = *reinterpret_cast<const float2 *>(a.pt_hi + off);
-                        const float2 t1 = *reinterpret_cast<const float2 *>(a.pt_lo + off);
-                        y[0] = t0.x; y[1] = t0.y;
-                        yl[0] = t1.x; yl[1] = t1.y;
-                    }
-                    for (int sp = 0; sp < a.nks; ++sp) {
-                        const size_t o = ((size_t)sp * a.p_pad + j) * g + l0;
-                        float thv[NT], tlv[NT];
-                        if constexpr (NT == 4) {
-                            const float4 t0 = __ldcg(reinterpret_cast<const float4 *>(th + o));
-                            const float4 t1 = __ldcg(reinterpret_cast<const float4 *>(tl + o));
-                            thv[0] = t0.x; thv[1] = t0.y; thv[2] = t0.z; thv[3] = t0.w;
-                            tlv[0] = t1.x; tlv[1] = t1.y; tlv[2] = t1.z; tlv[3] = t1.w;
-                        } else {
-                            const float2 t0 = __ldcg(reinterpret_cast<const float2 *>(th + o));
-                            const float2 t1 = __ldcg(reinterpret_cast<const float2 *>(tl + o));
-                            thv[0] = t0.x; thv[1] = t0.y;
-                            tlv[0] = t1.x; tlv[1] = t1.y;
-                        }
-#pragma unroll
-                        for (int t = 0; t < NT; ++t) {
-                            const float sm = y[t] - thv[t];
-                            const float bb = sm - y[t];
-                            const float e = (y[t] - (sm - bb)) + (-thv[t] - bb);
-                            y[t] = sm;
-                            yl[t] += e - tlv[t];
-                        }
-                    }
-#pragma unroll
-                    for (int t = 0; t < NT; ++t) {
-                        const float v = live ? (y[t] + yl[t]) / s : 0.f;
-                        Yb[uy_idx(l0 + t, r)] = v;
-                        Ub[uy_idx(l0 + t, r)] = v;
-                    }
-                    // codes: one word per 4 coordinates
-                    uint32_t packed;
-                    if constexpr (NT == 4) {
-                        packed = *reinterpret_cast<const uint32_t *>(a.Q + off);
-                        Cb[c_idx(lane, r)] = packed;
-                    } else {
-                        packed = *reinterpret_cast<const uint16_t *>(a.Q + off);
-                        const uint32_t other = __shfl_down_sync(0xffffffffu, packed, 1);
-                        if ((lane & 1) == 0) Cb[c_idx(lane >> 1, r)] = packed | (other << 16);
-                    }
-                    if (lane == 0) {
-                        rowS[r] = s;
-                        rowZ[r] = a.Z[(size_t)j * a.G + i];
-                        rowLive[r] = live ? 1 : 0;
-                    }
-                }
-            }
-            __threadfence_block();
-            __syncwarp();
-            if (lane == 0) tc::mbar_arrive(ybar);
-        }
-    } else if (warp == kBabaiWarp) {
-        // ------------------------------------------------ Babai, one row per lane
-        const int r = lane;
-        const int jr = j0 + kRows * rank + r;
-        if (lane == 0) {
-            tc::mbar_expect_tx(lbar, (uint32_t)(kRpk * sizeof(float)));
-            tc::bulk_load(tc::smem_u32(Rs), a.Rpk, kRpk * sizeof(float), lbar);
-            ++nl;
-        }
-        const float qmaxf = (float)a.qmax;
-        constexpr float kRound = 12582912.0f;      // 1.5 * 2^23: rounds to nearest even
-        for (int i = 0; i < a.G; ++i) {
-            bool ok = !*abort_flag && tc::mbar_wait(ybar, i & 1) && tc::mbar_wait(lbar, i & 1);
-            ok = __all_sync(0xffffffffu, ok);
-            if (!ok) {
-                *abort_flag = 1;
-                break;
-            }
-            // 1 / R_ll and R_ll of the group
-#pragma unroll
-            for (int t = 0; t < NT; ++t) {
-                const int l = NT * lane + t;
-                const float dgv = Rs[rpk_row_off(l, g) + (l & 15)];
-                Dg[l] = dgv;
-                Rd[l] = 1.0f / dgv;
-            }
-            __syncwarp();
-            const bool live = rowLive[r] != 0;
-            const float s = rowS[r];
-            // back substitution (Eq. babai_update) relative to the current
-            // codes: z + x_l = q_l + u_l / R_ll with u = y - R Delta, blocks of
-            // 16 coordinates from the top; the change of the group objective
-            // (Eq. group_bils) dF = s^2 sum_l (a_l - y_l)(a_l + y_l),
-            // a_l = R_ll Delta_l - u_l, is summed as coordinates become final
-            bool any = false;
-            float acc = 0.f;
-            for (int b0 = g - 16; b0 >= 0; b0 -= 16) {
-                float u[16], dq[16];
-                uint32_t cw[4];   // current codes of the block, four per word
-#pragma unroll
-                for (int t = 0; t < 16; ++t) u[t] = Ub[uy_idx(b0 + t, r)];
-#pragma unroll
-                for (int k = 0; k < 4; ++k) cw[k] = Cb[c_idx((b0 >> 2) + k, r)];
-                bool bany = false;
-#pragma unroll
-                for (int t = 15; t >= 0; --t) {
-                    const int l = b0 + t;
-                    const float qc = (float)((cw[t >> 2] >> (8 * (t & 3))) & 0xFFu);
-                    const float x = fmaf(u[t], Rd[l], qc);
-                    const float qv =
-                        fminf(fmaxf(__fsub_rn(__fadd_rn(x, kRound), kRound), 0.f), qmaxf);
-                    dq[t] = live ? qv - qc : 0.f;
-                    bany |= dq[t] != 0.f;
-#pragma unroll
-                    for (int tt = 0; tt < t; ++tt)
-                        u[tt] = fmaf(-Rs[rpk_row_off(b0 + tt, g) + t], dq[t], u[tt]);
-                    // coordinate l is final
-                    const float av = Dg[l] * dq[t] - u[t];
-                    const float yv = Yb[uy_idx(l, r)];
-                    acc = fmaf(av - yv, av + yv, acc);
-                }
-                any |= bany;
-                // proposed codes of the block (current code + integer change)
-#pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    uint32_t w = 0;
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const int c = (int)((cw[k] >> (8 * e)) & 0xFFu) + (int)dq[4 * k + e];
-                        w |= (uint32_t)c << (8 * e);
-                    }
-                    Cb[c_idx((b0 >> 2) + k, r)] = w;
-                }
-                // column updates of the coordinates below the block, in
-                // descending column order
-                if (__any_sync(0xffffffffu, bany)) {
-#pragma unroll 2
-                    for (int l = 0; l < b0; ++l) {
-                        const float4 *rr = reinterpret_cast<const float4 *>(
-                            Rs + rpk_row_off(l, g) + (b0 - 16 * (l >> 4)));
-                        float rv[16];
-#pragma unroll
-                        for (int k = 0; k < 4; ++k) {
-                            const float4 v4 = rr[k];
-                            rv[4 * k] = v4.x; rv[4 * k + 1] = v4.y;
-                            rv[4 * k + 2] = v4.z; rv[4 * k + 3] = v4.w;
-                        }
-                        float ul = Ub[uy_idx(l, r)];
-#pragma unroll
-                        for (int t = 15; t >= 0; --t) ul = fmaf(-rv[t], dq[t], ul);
-                        Ub[uy_idx(l, r)] = ul;
-                    }
-                }
-            }
-            const float dF = s * s * acc;
-            const bool accept = live && any && isfinite(dF) && dF < 0.f;
-            if (accept) {
-                const int j = jr;
-                const int z = rowZ[r];
-                const size_t off = (size_t)j * a.d + i * g;
-                __half *crow = a.cplane + (size_t)j * a.d_pad + i * g;
-#pragma unroll 2
-                for (int k4 = 0; k4 < g / 16; ++k4) {
-                    uint32_t w[4];
-#pragma unroll
-                    for (int k = 0; k < 4; ++k) w[k] = Cb[c_idx(4 * k4 + k, r)];
-                    *reinterpret_cast<uint4 *>(a.Q + off + 16 * k4) = make_uint4(w[0], w[1], w[2], w[3]);
-                    uint32_t hw[8];
-#pragma unroll
-                    for (int k = 0; k < 8; ++k) {
-                        const uint32_t c0 = (w[k >> 1] >> (16 * (k & 1))) & 0xFFu;
-                        const uint32_t c1 = (w[k >> 1] >> (16 * (k & 1) + 8)) & 0xFFu;
-                        const __half h0v = __int2half_rn((int)c0 - z);
-                        const __half h1v = __int2half_rn((int)c1 - z);
-                        hw[k] = (uint32_t)__half_as_ushort(h0v) | ((uint32_t)__half_as_ushort(h1v) << 16);
-                    }
-                    uint4 *cdst = reinterpret_cast<uint4 *>(crow + 16 * k4);
-                    cdst[0] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-                    cdst[1] = make_uint4(hw[4], hw[5], hw[6], hw[7]);
-                }
-                a.accepted[j] += 1;
-            }
+            form_targets<NT>(a, Ys, Cs, rowS, rowZ, rowLive, i, dw, lane, j0 + kRows * rank, th,
+                             tl, okw);
+            tc::named_bar_sync(1, 32 * kDrainWarps);
+            babai_block<NT>(a, Rs, Rds, Ys, Cs, rowS, rowZ, rowLive, Fp, blk, i, dw, lane,
+                            j0 + kRows * rank, okw);
             // the accepted codes reach the other CTAs' tensor-map loads
             tc::fence_proxy_async_global();
             tc::fence_acq_rel_cluster();
-            __syncwarp();
-            if (lane == 0) {
-                if (i + 1 < a.G) {
-                    // the next group's factor (this phase is done with the buffer)
+            tc::named_bar_sync(1, 32 * kDrainWarps);
+            if (dw == 0 && lane == 0) {
+                tc::fence_acq_rel_cluster();
+                for (int rk = 0; rk < kCluster; ++rk) tc::count_up_cluster(tc::map_cluster(ccnt, rk));
+                // the next group's factor (every warp is done with this one)
+                if (i + 1 < a.G && okw) {
                     tc::fence_proxy_async_smem();
                     tc::mbar_expect_tx(lbar, (uint32_t)(kRpk * sizeof(float)));
                     tc::bulk_load(tc::smem_u32(Rs), a.Rpk + (size_t)(i + 1) * kRpk,
                                   kRpk * sizeof(float), lbar);
                     ++nl;
                 }
-                tc::fence_acq_rel_cluster();
-                for (int rk = 0; rk < kCluster; ++rk) tc::count_up_cluster(tc::map_cluster(ccnt, rk));
             }
-            __syncwarp();
         }
+        if (dw == 0 && lane == 0 && nl > 0 && !tc::mbar_wait(lbar, (nl - 1) & 1)) *abort_flag = 1;
     }
 
     // ---------------- teardown: nothing of this CTA may be in flight
@@ -598,9 +641,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         // copies issued but never consumed (after a timeout)
         for (int c = *consumed; c < cp; ++c)
             if (!tc::mbar_wait(full(c % kStages), (c / kStages) & 1)) *abort_flag = 1;
-    }
-    if (warp == kBabaiWarp && lane == 0 && nl > 0) {
-        if (!tc::mbar_wait(lbar, (nl - 1) & 1)) *abort_flag = 1;
     }
     tc::tc_fence_before();
     __syncwarp();

@@ -54,6 +54,10 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
 __device__ __forceinline__ void prefetch_tmap(const CUtensorMap *m) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(m) : "memory");
 }
+// Bring `bytes` (multiple of 16, 16-byte aligned) of global memory into L2.
+__device__ __forceinline__ void prefetch_l2(const void *p, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
 // 2D tiled load of the box at (x = inner element index, y = row) into shared
 // memory, completing `bytes` on `bar`.
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *m, uint32_t bar,
@@ -99,6 +103,23 @@ __device__ __forceinline__ bool wait_count_cluster(uint32_t addr, uint32_t targe
         uint32_t v;
         asm volatile("ld.acquire.cluster.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
         if (v >= target) return true;
+    }
+    return false;
+}
+// Flags in this CTA's shared memory: a release store and a bounded polling
+// wait (acquire) until the flag reaches `target`.
+__device__ __forceinline__ void flag_store_release(uint32_t addr, uint32_t v) {
+    asm volatile("st.release.cta.shared::cta.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+// `relaxed`: sleep between polls, leaving the issue slots to warps doing
+// work (for waits that are not on a critical path).
+__device__ __forceinline__ bool flag_wait(uint32_t addr, uint32_t target, bool relaxed) {
+#pragma unroll 1
+    for (uint32_t i = 0; i < kWaitIters; ++i) {
+        uint32_t v;
+        asm volatile("ld.acquire.cta.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
+        if (v >= target) return true;
+        if (relaxed) __nanosleep(64);
     }
     return false;
 }
