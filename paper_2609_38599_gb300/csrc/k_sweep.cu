@@ -16,33 +16,41 @@
 //     y = (Pt_i - T_i) / s_i = R_i^{-T} (H r)_i / s_i
 // formed from the partials of all four CTAs.
 //
-// Babai (Eq. babai_update) is systolic over the 16 drain warps: lane r holds
-// row r of the CTA's 32, warp w holds coordinates [w CB, (w+1) CB) of the
-// group (CB = g/16).  Warp 15 resolves its coordinates first and hands the
-// code changes down through shared memory; warp w applies the column
-// updates of every higher block in descending column order as they arrive,
-// then resolves its own block from the top.  Each u_l thus sees the same
-// fused multiply-adds in the same order as the coordinate-by-coordinate
-// recursion.  The change of the group objective (Eq. group_bils) is summed
-// per warp and reduced over the warps per row; a proposal is kept iff it is
-// finite and below zero (an unchanged row gives exactly zero).
-//
 // Overlap.  Group i's codes change only in phase i, so the product of phase
 // i+1 needs phase i's result only for the K chunks of group i.  The CTA
 // whose K range holds group i takes that group last in phase i+1, and its
 // producer waits for the codes of all four CTAs only before loading it.
+// The Babai proposals of phase i therefore run on their own warps while the
+// product of phase i+1 streams through the tensor cores: the product is
+// bound by the tile loads of each SM, and the drain warps that combine its
+// digit sums are idle most of the time, so a phase costs about one product.
 //
-// One CTA (576 threads):
-//   warp 0       TMA producer (code tiles, digit tiles)
-//   warp 1       TMEM allocation and the single-thread MMA issuer
-//   warps 2..17  drain (digit sums -> double-float partial), then Babai
-// Cluster signals: two counters in every CTA's shared memory that each of
-// the four CTAs increments once per phase (remote reductions with release
-// semantics at cluster scope; readers poll with acquire): `pcnt` -- the
-// partials of the phase are in global memory; `ccnt` -- the codes of the
-// phase are in Q and the code plane.  Phase i is complete at 4 (i + 1).
-// Counters, unlike barrier phases, may be waited for out of order: the
-// producer waits only in the phases where it holds the pending group.
+// Babai (Eq. babai_update) is systolic over 8 warps: lane r holds row r of
+// the CTA's 32, warp w holds coordinates [w CB, (w+1) CB) of the group
+// (CB = g/8, resolved as sub-blocks of 8).  Warp 7 resolves its
+// coordinates first and hands the code changes down through shared memory;
+// warp w applies the column updates of every higher block in descending
+// column order as they arrive, then resolves its own block from the top.
+// Each u_l thus sees the same fused multiply-adds in the same order as the
+// coordinate-by-coordinate recursion.  The change of the group objective
+// (Eq. group_bils) is summed per warp and reduced over the warps per row; a
+// proposal is kept iff it is finite and below zero (an unchanged row gives
+// exactly zero).
+//
+// One CTA (832 threads):
+//   warp 0        TMA producer (code tiles, digit tiles)
+//   warp 1        TMEM allocation and the single-thread MMA issuer
+//   warps 2..17   drain: digit sums -> double-float partial of T_i
+//   warps 18..25  Babai: targets, proposals, acceptance, codes
+// Cluster signals: two sets of counters in every CTA's shared memory, one
+// counter per source CTA, which that CTA increments once per phase (remote
+// reductions with release semantics at cluster scope; readers poll with
+// acquire): `pcnt` -- the partials of the phase are in global memory;
+// `ccnt` -- the codes of the phase are in Q and the code plane.  Phase i is
+// complete when all four counters of a set reach i + 1.  (A single summed
+// counter would not do: the CTAs may be a phase apart.)  Counters, unlike
+// barrier phases, may be waited for out of order: the producer waits only
+// in the phases where it holds the pending group.
 //
 // Every wait is bounded; on a timeout the CTA stops issuing work, keeps
 // arriving at the final cluster barrier (so no CTA of its cluster waits
@@ -57,12 +65,16 @@ namespace {
 constexpr int kTileA = 128 * 64 * 2;   // codes: 128 rows x 64 K, fp16
 constexpr int kTileB = 64 * 64 * 2;    // one digit plane: 64 rows of Ht x 64 K
 constexpr int kStage = kTileA + 4 * kTileB;
-constexpr int kStages = 3;
+constexpr int kStages = 2;
 constexpr int kCluster = 4;            // CTAs per row tile
 constexpr int kRows = 128 / kCluster;  // Babai rows per CTA (one per lane)
 constexpr uint32_t kIdesc = tc::idesc_f16_f32(128, 256);
 constexpr int kDrainWarps = 16;
-constexpr int kThreads = 32 * (2 + kDrainWarps);
+constexpr int kBabaiWarps = 8;
+constexpr int kDrain0 = 2;                         // first drain warp
+constexpr int kBabai0 = kDrain0 + kDrainWarps;     // first Babai warp
+constexpr int kThreads = 32 * (kBabai0 + kBabaiWarps);
+constexpr int kBarDrain = 1, kBarBabai = 2;        // named barriers
 
 // Packed rows of R_i (upper triangular, g x g): row l holds columns
 // 16 floor(l/16) .. g-1, so every row starts on a 64-byte boundary.
@@ -72,13 +84,15 @@ __host__ __device__ constexpr int rpk_row_off(int l, int g) {
 __host__ __device__ constexpr int rpk_size(int g) { return rpk_row_off(g, g); }
 
 // shared memory (g = 128 sizes; g = 64 uses less of each)
-constexpr int kOffRpk = kStages * kStage;
-constexpr int kOffYs = kOffRpk + rpk_size(128) * 4;   // targets / code changes [g][32]
-constexpr int kOffCs = kOffYs + 128 * kRows * 4;       // codes [g/4][32] words
-constexpr int kOffRow = kOffCs + 32 * kRows * 4;       // s, z, live of the 32 rows
-constexpr int kOffFp = kOffRow + 3 * kRows * 4;        // dF parts [16 warps][32]
-constexpr int kOffRd = kOffFp + kDrainWarps * kRows * 4;   // 1 / R_ll [g]
-constexpr int kOffBar = kOffRd + 128 * 4;
+constexpr int kOffLo = kStages * kStage;                   // drain low parts [16][512]
+constexpr int kOffRpk = kOffLo + 16 * 32 * kDrainWarps * 4;
+constexpr int kOffYs = kOffRpk + rpk_size(128) * 4;        // targets / code changes [g][32]
+constexpr int kOffCs = kOffYs + 128 * kRows * 4;           // codes [g/4][32] words
+constexpr int kOffRow = kOffCs + 32 * kRows * 4;           // s, z, live of the 32 rows
+constexpr int kOffFp = kOffRow + 3 * kRows * 4;            // dF parts [8 warps][32]
+constexpr int kOffRd = kOffFp + kBabaiWarps * kRows * 4;   // 1 / R_ll [g]
+constexpr int kOffUs = kOffRd + 128 * 4;                   // u stash [8 warps][8][32]
+constexpr int kOffBar = kOffUs + kBabaiWarps * 8 * kRows * 4;
 constexpr int kSmem = 1024 + kOffBar + 512;
 static_assert(kSmem <= 232448, "shared memory of one CTA");
 
@@ -124,21 +138,22 @@ __device__ __forceinline__ int unit_group(int u, int i, int h0, int nseg) {
 __device__ __forceinline__ int ys_idx(int l, int r) { return l * kRows + (r ^ ((l >> 2) & 31)); }
 __device__ __forceinline__ int cs_idx(int k, int r) { return k * kRows + (r ^ (k & 31)); }
 
-// Babai targets y = (Pt_i - sum of partials) / s of rows 2 dw, 2 dw + 1 of
+// Babai targets y = (Pt_i - sum of partials) / s of rows 4 bw .. 4 bw + 3 of
 // the CTA's 32 (double-float until the subtraction is done), coalesced: a
-// row per warp, NT consecutive coordinates per lane.  Also the row's codes
+// row at a time, NT consecutive coordinates per lane.  Also each row's codes
 // and its scale, zero point and whether it takes a proposal.
 template <int NT>
 __device__ __forceinline__ void form_targets(const SweepArgs &a, float *Ys, uint32_t *Cs,
                                              float *rowS, int *rowZ, int *rowLive, int i,
-                                             int dw, int lane, int jb, const float *th,
+                                             int bw, int lane, int jb, const float *th,
                                              const float *tl, bool ok) {
     constexpr int g = 32 * NT;
     constexpr int nks = kCluster / (g / 64);   // K parts of the phase product
+    constexpr int per = kRows / kBabaiWarps;   // rows per Babai warp
     const int l0 = NT * lane;
 #pragma unroll
-    for (int rr = 0; rr < 2; ++rr) {
-        const int r = 2 * dw + rr;
+    for (int rr = 0; rr < per; ++rr) {
+        const int r = per * bw + rr;
         const int jr = jb + r;
         const int j = min(jr, a.p - 1);
         const float s = a.S[(size_t)j * a.G + i];
@@ -198,53 +213,35 @@ __device__ __forceinline__ void form_targets(const SweepArgs &a, float *Ys, uint
 }
 
 // Systolic Babai for group i of the CTA's 32 rows (row r = lane) on the CB
-// coordinates of block w (warp), from the targets and codes in Ys and Cs.
-// Rs: packed R_i; Fp: per-warp dF parts [w][r]; blk: one flag per block, set
-// to i + 1 when the block's code changes of phase i are in Ys.  ok: every
-// earlier wait succeeded (else only the hand-off protocol is kept).
+// coordinates of block w (Babai warp), from the targets and codes in Ys and
+// Cs.  Rs: packed R_i; Rds: 1 / R_ll; Fp: per-warp dF parts [w][r]; blk: one
+// flag per block, set to i + 1 when the block's code changes of phase i are
+// in Ys.  ok: every earlier wait succeeded (else only the hand-off protocol
+// is kept).
 template <int NT>
-__device__ __forceinline__ void babai_block(const SweepArgs &a, const float *Rs, float *Rds, float *Ys,
-                                            const uint32_t *Cs, const float *rowS,
+__device__ __forceinline__ void babai_block(const SweepArgs &a, const float *Rs, float *Rds,
+                                            float *Us, float *Ys, const uint32_t *Cs, const float *rowS,
                                             const int *rowZ, const int *rowLive, float *Fp,
                                             uint32_t *blk, int i, int w, int lane, int jb,
                                             bool ok) {
     constexpr int g = 32 * NT;
-    constexpr int CB = g / 16;              // coordinates per warp
+    constexpr int CB = g / kBabaiWarps;     // coordinates per warp (16 or 8)
+    constexpr int NSB = CB / 8;             // sub-blocks of 8 coordinates
     const int c0 = w * CB;
     const int r = lane;
     const bool live = rowLive[r] != 0;
-    // this block's part of the factor: Rs[ro0 + tt rs + h] is R[c0 + tt][h]
-    // (the block's rows lie in one 16-row band of the packed layout); the
-    // diagonal and its reciprocals
+    // Rs[ro0 + tt rs + h] is R[c0 + tt][h]: the block's rows lie in one
+    // 16-row band of the packed layout
     const int ro0 = rpk_row_off(c0, g) - 16 * (c0 >> 4);
     const int rs = g - 16 * (c0 >> 4);
-    // reciprocals of this block's diagonal, kept in shared memory (Rds) so
-    // that they occupy no registers while the block waits
     if (lane < CB) Rds[c0 + lane] = 1.0f / Rs[ro0 + lane * rs + c0 + lane];
     __syncwarp();
-    uint32_t cw[CB / 4];   // current codes, four per word
-#pragma unroll
-    for (int k = 0; k < CB / 4; ++k) cw[k] = Cs[cs_idx(c0 / 4 + k, r)];
-    auto qc = [&](int t) { return (float)((cw[t >> 2] >> (8 * (t & 3))) & 0xFFu); };
-    float u[CB], dq[CB];
+    float u[CB];
 #pragma unroll
     for (int t = 0; t < CB; ++t) u[t] = Ys[ys_idx(c0 + t, r)];
-    // tri[tt][t] = R[c0 + tt][c0 + t], t > tt: loaded just before the block
-    // above hands over (it is not needed earlier)
-    float tri[CB][CB];
-    auto load_tri = [&]() {
-#pragma unroll
-        for (int tt = 0; tt < CB - 1; ++tt) {
-#pragma unroll
-            for (int k = tt & ~3; k < CB; k += 4) {
-                const float4 v4 = *reinterpret_cast<const float4 *>(Rs + ro0 + tt * rs + c0 + k);
-                tri[tt][k] = v4.x; tri[tt][k + 1] = v4.y; tri[tt][k + 2] = v4.z; tri[tt][k + 3] = v4.w;
-            }
-        }
-    };
     // column updates from every higher block, descending (per coordinate the
     // columns in descending order)
-    for (int b = kDrainWarps - 1; b > w; --b) {
+    for (int b = kBabaiWarps - 1; b > w; --b) {
         if (!tc::flag_wait(tc::smem_u32(blk + b), (uint32_t)(i + 1), b > w + 1)) ok = false;
         float dv[CB];
 #pragma unroll
@@ -261,50 +258,89 @@ __device__ __forceinline__ void babai_block(const SweepArgs &a, const float *Rs,
             for (int t = CB - 1; t >= 0; --t) u[tt] = fmaf(-rv[t], dv[t], u[tt]);
         }
     }
-    // own block, from the top (Eq. babai_update); the change of the group
-    // objective is summed as coordinates become final (Eq. group_bils).
-    load_tri();
+    // own block, sub-blocks of 8 from the top (Eq. babai_update); the
+    // change of the group objective is summed as coordinates become final
+    // (Eq. group_bils).  While a sub-block resolves, the u of the lower ones
+    // wait in shared memory (Us), which keeps the resolve in registers.
+    uint32_t cw[CB / 4];   // current codes, four per word
+#pragma unroll
+    for (int k = 0; k < CB / 4; ++k) cw[k] = Cs[cs_idx(c0 / 4 + k, r)];
+    auto qc = [&](int t) { return (float)((cw[t >> 2] >> (8 * (t & 3))) & 0xFFu); };
     const float qmaxf = (float)a.qmax;
     constexpr float kRound = 12582912.0f;   // 1.5 * 2^23: rounds to nearest even
-    // everything off the dependency chain first: the current codes as
-    // floats and the reciprocals with a row that takes no proposal folded in
-    // (1 / R_ll = 0 keeps x = q, hence no change)
-    float rd[CB];
+    float *us = Us + w * (CB - 8) * kRows;   // [CB - 8][32] of this warp
 #pragma unroll
-    for (int t = 0; t < CB; ++t) rd[t] = live ? Rds[c0 + t] : 0.f;
-#pragma unroll
-    for (int t = CB - 1; t >= 0; --t) {
-        const float qf = qc(t);
-        const float x = fmaf(u[t], rd[t], qf);
-        const float qv = fminf(fmaxf(__fsub_rn(__fadd_rn(x, kRound), kRound), 0.f), qmaxf);
-        dq[t] = qv - qf;
-        // the next coordinate's update first: it is on the chain
-        if (t > 0) u[t - 1] = fmaf(-tri[t - 1][t], dq[t], u[t - 1]);
-#pragma unroll
-        for (int tt = 0; tt + 1 < t; ++tt) u[tt] = fmaf(-tri[tt][t], dq[t], u[tt]);
-    }
-    // the block's part of the change of the group objective, with every u
-    // now final (targets read before the changes replace them)
-    float yv[CB];
-#pragma unroll
-    for (int t = 0; t < CB; ++t) yv[t] = Ys[ys_idx(c0 + t, r)];
-    // the block's changes replace its targets and go to the blocks below
-#pragma unroll
-    for (int t = 0; t < CB; ++t) Ys[ys_idx(c0 + t, r)] = dq[t];
-    __syncwarp();
-    if (lane == 0) tc::flag_store_release(tc::smem_u32(blk + w), (uint32_t)(i + 1));
+    for (int t = 0; t < CB - 8; ++t) us[t * kRows + r] = u[t];
     float acc = 0.f;
 #pragma unroll
-    for (int t = CB - 1; t >= 0; --t) {
-        const float av = Rs[ro0 + t * rs + c0 + t] * dq[t] - u[t];
-        acc = fmaf(av - yv[t], av + yv[t], acc);
+    for (int sb = NSB - 1; sb >= 0; --sb) {
+        const int s0 = 8 * sb;
+        float v[8];   // u of this sub-block
+#pragma unroll
+        for (int t = 0; t < 8; ++t) v[t] = (sb == NSB - 1) ? u[s0 + t] : us[(s0 + t) * kRows + r];
+        // tri[tt][t] = R[c0 + s0 + tt][c0 + s0 + t], t > tt
+        float tri[8][8];
+#pragma unroll
+        for (int tt = 0; tt < 7; ++tt) {
+#pragma unroll
+            for (int k = tt & ~3; k < 8; k += 4) {
+                const float4 v4 =
+                    *reinterpret_cast<const float4 *>(Rs + ro0 + (s0 + tt) * rs + c0 + s0 + k);
+                tri[tt][k] = v4.x; tri[tt][k + 1] = v4.y; tri[tt][k + 2] = v4.z; tri[tt][k + 3] = v4.w;
+            }
+        }
+        // a row that takes no proposal: 1 / R_ll = 0 keeps x = q, no change
+        float rd[8], dq[8];
+#pragma unroll
+        for (int t = 0; t < 8; ++t) rd[t] = live ? Rds[c0 + s0 + t] : 0.f;
+#pragma unroll
+        for (int t = 7; t >= 0; --t) {
+            const float qf = qc(s0 + t);
+            const float x = fmaf(v[t], rd[t], qf);
+            const float qv = fminf(fmaxf(__fsub_rn(__fadd_rn(x, kRound), kRound), 0.f), qmaxf);
+            dq[t] = qv - qf;
+            // the next coordinate's update first: it is on the chain
+            if (t > 0) v[t - 1] = fmaf(-tri[t - 1][t], dq[t], v[t - 1]);
+#pragma unroll
+            for (int tt = 0; tt + 1 < t; ++tt) v[tt] = fmaf(-tri[tt][t], dq[t], v[tt]);
+        }
+        // every u of the sub-block is final: its part of dF, then its changes
+        // replace its targets
+#pragma unroll
+        for (int t = 7; t >= 0; --t) {
+            const int l = c0 + s0 + t;
+            const float yv = Ys[ys_idx(l, r)];
+            const float av = Rs[ro0 + (s0 + t) * rs + l] * dq[t] - v[t];
+            acc = fmaf(av - yv, av + yv, acc);
+            Ys[ys_idx(l, r)] = dq[t];
+        }
+        // the lower sub-blocks of this block take this sub-block's columns
+#pragma unroll
+        for (int sl = 0; sl < sb; ++sl) {
+#pragma unroll
+            for (int tt = 0; tt < 8; ++tt) {
+                float rv[8];
+#pragma unroll
+                for (int k = 0; k < 8; k += 4) {
+                    const float4 v4 = *reinterpret_cast<const float4 *>(
+                        Rs + ro0 + (8 * sl + tt) * rs + c0 + s0 + k);
+                    rv[k] = v4.x; rv[k + 1] = v4.y; rv[k + 2] = v4.z; rv[k + 3] = v4.w;
+                }
+                float ul = us[(8 * sl + tt) * kRows + r];
+#pragma unroll
+                for (int t = 7; t >= 0; --t) ul = fmaf(-rv[t], dq[t], ul);
+                us[(8 * sl + tt) * kRows + r] = ul;
+            }
+        }
     }
+    __syncwarp();
+    if (lane == 0) tc::flag_store_release(tc::smem_u32(blk + w), (uint32_t)(i + 1));
     Fp[w * kRows + r] = acc;
     // every block's dF part of this row
-    tc::named_bar_sync(1, 32 * kDrainWarps);
+    tc::named_bar_sync(kBarBabai, 32 * kBabaiWarps);
     float F = 0.f;
 #pragma unroll
-    for (int b = kDrainWarps - 1; b >= 0; --b) F += Fp[b * kRows + r];
+    for (int b = kBabaiWarps - 1; b >= 0; --b) F += Fp[b * kRows + r];
     const float s = rowS[r];
     const float dF = s * s * F;
     const int jr = jb + r;
@@ -312,28 +348,26 @@ __device__ __forceinline__ void babai_block(const SweepArgs &a, const float *Rs,
         const int j = jr;
         const int z = rowZ[r];
         const size_t off = (size_t)j * a.d + i * g + c0;
-        uint32_t nw[CB / 4];
+        int qn[CB];
 #pragma unroll
-        for (int k = 0; k < CB / 4; ++k) {
-            uint32_t v = 0;
+        for (int t = 0; t < CB; ++t) qn[t] = (int)qc(t) + (int)Ys[ys_idx(c0 + t, r)];
+        uint32_t nw[CB / 4], hw[CB / 2];
 #pragma unroll
-            for (int e = 0; e < 4; ++e) v |= (uint32_t)((int)qc(4 * k + e) + (int)dq[4 * k + e]) << (8 * e);
-            nw[k] = v;
-        }
-        uint32_t hw[CB / 2];
+        for (int k = 0; k < CB / 4; ++k)
+            nw[k] = (uint32_t)qn[4 * k] | ((uint32_t)qn[4 * k + 1] << 8) |
+                    ((uint32_t)qn[4 * k + 2] << 16) | ((uint32_t)qn[4 * k + 3] << 24);
 #pragma unroll
-        for (int k = 0; k < CB / 2; ++k) {
-            const int qa = (int)qc(2 * k) + (int)dq[2 * k], qb = (int)qc(2 * k + 1) + (int)dq[2 * k + 1];
-            hw[k] = (uint32_t)__half_as_ushort(__int2half_rn(qa - z)) |
-                    ((uint32_t)__half_as_ushort(__int2half_rn(qb - z)) << 16);
-        }
+        for (int k = 0; k < CB / 2; ++k)
+            hw[k] = (uint32_t)__half_as_ushort(__int2half_rn(qn[2 * k] - z)) |
+                    ((uint32_t)__half_as_ushort(__int2half_rn(qn[2 * k + 1] - z)) << 16);
         __half *crow = a.cplane + (size_t)j * a.d_pad + i * g + c0;
-        if constexpr (CB == 8) {
+        if constexpr (CB == 16) {
+            *reinterpret_cast<uint4 *>(a.Q + off) = make_uint4(nw[0], nw[1], nw[2], nw[3]);
+            reinterpret_cast<uint4 *>(crow)[0] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+            reinterpret_cast<uint4 *>(crow)[1] = make_uint4(hw[4], hw[5], hw[6], hw[7]);
+        } else {
             *reinterpret_cast<uint2 *>(a.Q + off) = make_uint2(nw[0], nw[1]);
             *reinterpret_cast<uint4 *>(crow) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-        } else {
-            *reinterpret_cast<uint32_t *>(a.Q + off) = nw[0];
-            *reinterpret_cast<uint2 *>(crow) = make_uint2(hw[0], hw[1]);
         }
         if (w == 0) a.accepted[j] += 1;
     }
@@ -349,6 +383,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     constexpr int kRpk = rpk_size(g);
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    float *Lo = (float *)(smem + kOffLo);
     float *Rs = (float *)(smem + kOffRpk);
     float *Ys = (float *)(smem + kOffYs);
     uint32_t *Cs = (uint32_t *)(smem + kOffCs);
@@ -357,16 +392,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     int *rowLive = rowZ + kRows;
     float *Fp = (float *)(smem + kOffFp);
     float *Rds = (float *)(smem + kOffRd);
+    float *Us = (float *)(smem + kOffUs);
     uint64_t *bars = (uint64_t *)(smem + kOffBar);
     uint32_t *blk = (uint32_t *)(bars + 2 * kStages + 6);   // one flag per Babai block
-    uint32_t *tmem_slot = blk + kDrainWarps;
-    uint32_t *counters = tmem_slot + 4;   // pcnt, ccnt
+    uint32_t *tmem_slot = blk + kBabaiWarps;
     volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
     int *consumed = (int *)(tmem_slot + 2);
+    uint32_t *counters = tmem_slot + 4;   // pcnt[4], ccnt[4]
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int rank = (int)tc::cluster_ctarank();
     const int cpart = rank % ncol, kpart = rank / ncol;
     const int j0 = (blockIdx.x / kCluster) * 128;
+    const int jb = j0 + kRows * rank;     // first of this CTA's Babai rows
     const int h0 = kpart * a.seg;
     const int nseg = max(0, min(a.G, h0 + a.seg) - h0);
     const int nchunks = nseg * nkc;
@@ -375,10 +412,22 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto empty = [&](int s) { return tc::smem_u32(bars + kStages + s); };
     auto afull = [&](int b) { return tc::smem_u32(bars + 2 * kStages + b); };
     auto aempty = [&](int b) { return tc::smem_u32(bars + 2 * kStages + 2 + b); };
-    const uint32_t pcnt = tc::smem_u32(counters);       // partials, 4 per phase
-    const uint32_t ccnt = tc::smem_u32(counters + 1);   // codes, 4 per phase
     const uint32_t lbar = tc::smem_u32(bars + 2 * kStages + 4);   // factor copy
     const uint32_t done = tc::smem_u32(bars + 2 * kStages + 5);
+    const uint32_t pcnt = tc::smem_u32(counters);       // partials, one per source CTA
+    const uint32_t ccnt = tc::smem_u32(counters + 4);   // codes, one per source CTA
+    // phase i of every CTA of the cluster is out
+    auto wait_all = [&](uint32_t base, int i) {
+        bool ok = true;
+#pragma unroll 1
+        for (int k = 0; k < kCluster && ok; ++k) ok = tc::wait_count_cluster(base + 4 * k, i + 1);
+        return ok;
+    };
+    // this CTA's phase is out, in every CTA of the cluster
+    auto signal_all = [&](uint32_t base) {
+        tc::fence_acq_rel_cluster();
+        for (int r = 0; r < kCluster; ++r) tc::count_up_cluster(tc::map_cluster(base + 4 * rank, r));
+    };
     auto tileA = [&](int s) { return tc::smem_u32(smem + s * kStage); };
     auto tileB = [&](int s, int t) { return tc::smem_u32(smem + s * kStage + kTileA + t * kTileB); };
 
@@ -391,11 +440,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc::mbar_init(afull(b), 1);
             tc::mbar_init(aempty(b), kDrainWarps);
         }
-        counters[0] = 0;
-        counters[1] = 0;
-        for (int b = 0; b < kDrainWarps; ++b) blk[b] = 0;
         tc::mbar_init(lbar, 1);
         tc::mbar_init(done, 1);
+        for (int b = 0; b < kBabaiWarps; ++b) blk[b] = 0;
+        for (int k = 0; k < 2 * kCluster; ++k) counters[k] = 0;
         *abort_flag = 0;
         *consumed = 0;
         tc::fence_barrier_init();
@@ -410,7 +458,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     tc::tc_fence_before();
     __syncwarp();
-    // every CTA's barriers are initialised before any CTA arrives on them
+    // every CTA's counters are initialised before any CTA adds to them
     tc::cluster_sync();
     tc::tc_fence_after();
     const uint32_t tmem = *tmem_slot;
@@ -420,7 +468,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     int cp = 0;               // producer: chunks issued
     int cm = 0;               // MMA issuer: chunks consumed
-    int nl = 0;               // drain leader: factor copies issued
+    int nl = 0;               // Babai leader: factor copies issued
 
     if (warp == 0 && lane == 0) {
         // ------------------------------------------------ producer
@@ -429,17 +477,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             const bool holds = i >= 1 && i - 1 >= h0 && i - 1 < h0 + nseg;
             // the folded projection of this CTA's Babai rows for group i,
             // read when the phase's targets are formed
-            for (int r = 0; r < kRows; ++r) {
-                const int j = j0 + kRows * rank + r;
-                if (j >= a.p) break;
-                tc::prefetch_l2(a.pt_hi + (size_t)j * a.d + i * g, g * sizeof(float));
-                tc::prefetch_l2(a.pt_lo + (size_t)j * a.d + i * g, g * sizeof(float));
+            for (int r = 0; r < kRows && jb + r < a.p; ++r) {
+                tc::prefetch_l2(a.pt_hi + (size_t)(jb + r) * a.d + i * g, g * sizeof(float));
+                tc::prefetch_l2(a.pt_lo + (size_t)(jb + r) * a.d + i * g, g * sizeof(float));
             }
             for (int c = 0; c < nchunks; ++c) {
                 const int u = c / nkc, kc = c % nkc;
                 if (holds && u == nseg - 1 && kc == 0) {
-                    // the last group is i-1: its codes from all four Babai warps
-                    if (!tc::wait_count_cluster(ccnt, kCluster * i)) {
+                    // the last group is i-1: its codes from all four CTAs
+                    if (!wait_all(ccnt, i - 1)) {
                         *abort_flag = 1;
                         break;
                     }
@@ -493,25 +539,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                 ++um;
             }
         }
-    } else if (warp >= 2) {
-        // ------------------------------------------------ drain + Babai targets
-        const int q = warp & 3, cq = (warp - 2) >> 2;    // lane quarter, 16-column quarter
+    } else if (warp >= kDrain0 && warp < kBabai0) {
+        // ------------------------------------------------ drain
+        const int q = warp & 3, cq = (warp - kDrain0) >> 2;   // lane quarter, 16-column quarter
         const int row = j0 + 32 * q + lane;
         const float *srow = a.S + (size_t)min(row, a.p - 1) * a.G;
-        const int dw = warp - 2;
+        const int dw = warp - kDrain0;
+        // low parts of this thread's 16 double-float accumulators
+        float *lo = Lo + (threadIdx.x - 32 * kDrain0);
         int ud = 0;
-        if (dw == 0 && lane == 0) {
-            // the factor of group 0
-            tc::mbar_expect_tx(lbar, (uint32_t)(kRpk * sizeof(float)));
-            tc::bulk_load(tc::smem_u32(Rs), a.Rpk, kRpk * sizeof(float), lbar);
-            ++nl;
-        }
         for (int i = 0; i < a.G; ++i) {
-            float hi[16], lo[16];
+            float hi[16];
 #pragma unroll
             for (int e = 0; e < 16; ++e) {
                 hi[e] = 0.f;
-                lo[e] = 0.f;
+                lo[e * 32 * kDrainWarps] = 0.f;
             }
             bool ok = __all_sync(0xffffffffu, !*abort_flag);
             const int *erow = a.expoT + (size_t)i * a.G;
@@ -569,14 +611,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const float pe = fmaf(vh, scale, -ph);
                         two_sum(hi[cc + e], ph, s2, e2);
                         hi[cc + e] = s2;
-                        lo[cc + e] += e2 + fmaf(vl, scale, pe);
+                        lo[(cc + e) * 32 * kDrainWarps] += e2 + fmaf(vl, scale, pe);
                     }
                 }
                 ++ud;
             }
-            // partial of this CTA (slot i & 1: the targets of phase i-1 in
-            // every CTA were formed from the other slot before any CTA
-            // reaches this point of phase i+1)
+            // partial of this CTA in slot i & 1; the slot's previous contents
+            // (phase i-2) were read by every CTA's Babai warps before their
+            // codes of phase i-2 went out
+            if (ok && i >= 2 && !wait_all(ccnt, i - 2)) {
+                ok = false;
+                *abort_flag = 1;
+            }
             float *th = a.t_hi + (size_t)(i & 1) * a.nks * a.p_pad * g;
             float *tl = a.t_lo + (size_t)(i & 1) * a.nks * a.p_pad * g;
             if (ok && row < a.p) {
@@ -585,40 +631,47 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int e = 0; e < 16; e += 4) {
                     float x[4], y[4];
 #pragma unroll
-                    for (int k = 0; k < 4; ++k) two_sum(hi[e + k], lo[e + k], x[k], y[k]);
+                    for (int k = 0; k < 4; ++k)
+                        two_sum(hi[e + k], lo[(e + k) * 32 * kDrainWarps], x[k], y[k]);
                     *reinterpret_cast<float4 *>(th + o + e) = make_float4(x[0], x[1], x[2], x[3]);
                     *reinterpret_cast<float4 *>(tl + o + e) = make_float4(y[0], y[1], y[2], y[3]);
                 }
             }
             // each thread's partial is visible cluster-wide before the signal
             tc::fence_acq_rel_cluster();
-            tc::named_bar_sync(1, 32 * kDrainWarps);
-            if (dw == 0 && lane == 0) {
-                tc::fence_acq_rel_cluster();
-                for (int r = 0; r < kCluster; ++r) tc::count_up_cluster(tc::map_cluster(pcnt, r));
-            }
-            // Babai of this CTA's 32 rows of the tile (one per lane) for
-            // the CB coordinates of this warp's block, once the partials of
-            // all four CTAs are out and the factor R_i is in shared memory
-            bool okw = !*abort_flag;
-            if (okw) okw = tc::wait_count_cluster(pcnt, kCluster * (i + 1));
-            if (okw) okw = tc::mbar_wait(lbar, i & 1);
-            okw = __all_sync(0xffffffffu, okw);
-            if (!okw) *abort_flag = 1;
-            form_targets<NT>(a, Ys, Cs, rowS, rowZ, rowLive, i, dw, lane, j0 + kRows * rank, th,
-                             tl, okw);
-            tc::named_bar_sync(1, 32 * kDrainWarps);
-            babai_block<NT>(a, Rs, Rds, Ys, Cs, rowS, rowZ, rowLive, Fp, blk, i, dw, lane,
-                            j0 + kRows * rank, okw);
+            tc::named_bar_sync(kBarDrain, 32 * kDrainWarps);
+            if (dw == 0 && lane == 0) signal_all(pcnt);
+        }
+    } else if (warp >= kBabai0) {
+        // ------------------------------------------------ Babai
+        const int bw = warp - kBabai0;
+        if (bw == 0 && lane == 0) {
+            // the factor of group 0
+            tc::mbar_expect_tx(lbar, (uint32_t)(kRpk * sizeof(float)));
+            tc::bulk_load(tc::smem_u32(Rs), a.Rpk, kRpk * sizeof(float), lbar);
+            ++nl;
+        }
+        for (int i = 0; i < a.G; ++i) {
+            // the partials of all four CTAs and the factor R_i
+            bool ok = !*abort_flag;
+            if (ok) ok = wait_all(pcnt, i);
+            if (ok) ok = tc::mbar_wait(lbar, i & 1);
+            ok = __all_sync(0xffffffffu, ok);
+            if (!ok) *abort_flag = 1;
+            const float *th = a.t_hi + (size_t)(i & 1) * a.nks * a.p_pad * g;
+            const float *tl = a.t_lo + (size_t)(i & 1) * a.nks * a.p_pad * g;
+            form_targets<NT>(a, Ys, Cs, rowS, rowZ, rowLive, i, bw, lane, jb, th, tl, ok);
+            tc::named_bar_sync(kBarBabai, 32 * kBabaiWarps);
+            babai_block<NT>(a, Rs, Rds, Us, Ys, Cs, rowS, rowZ, rowLive, Fp, blk, i, bw, lane, jb,
+                            ok);
             // the accepted codes reach the other CTAs' tensor-map loads
             tc::fence_proxy_async_global();
             tc::fence_acq_rel_cluster();
-            tc::named_bar_sync(1, 32 * kDrainWarps);
-            if (dw == 0 && lane == 0) {
-                tc::fence_acq_rel_cluster();
-                for (int rk = 0; rk < kCluster; ++rk) tc::count_up_cluster(tc::map_cluster(ccnt, rk));
-                // the next group's factor (every warp is done with this one)
-                if (i + 1 < a.G && okw) {
+            tc::named_bar_sync(kBarBabai, 32 * kBabaiWarps);
+            if (bw == 0 && lane == 0) {
+                signal_all(ccnt);
+                // the next group's factor (every Babai warp is done with this one)
+                if (i + 1 < a.G && !*abort_flag) {
                     tc::fence_proxy_async_smem();
                     tc::mbar_expect_tx(lbar, (uint32_t)(kRpk * sizeof(float)));
                     tc::bulk_load(tc::smem_u32(Rs), a.Rpk + (size_t)(i + 1) * kRpk,
@@ -627,7 +680,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
         }
-        if (dw == 0 && lane == 0 && nl > 0 && !tc::mbar_wait(lbar, (nl - 1) & 1)) *abort_flag = 1;
+        if (bw == 0 && lane == 0 && nl > 0 && !tc::mbar_wait(lbar, (nl - 1) & 1)) *abort_flag = 1;
     }
 
     // ---------------- teardown: nothing of this CTA may be in flight
@@ -644,7 +697,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     tc::tc_fence_before();
     __syncwarp();
-    // no CTA leaves while another may still arrive on its barriers
+    // no CTA leaves while another may still add to its counters
     tc::cluster_sync();
     if (warp == 1) {
         tc::tc_fence_after();
