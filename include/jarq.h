@@ -331,7 +331,7 @@ const char *jarq_status_string(jarq_status s);
  * "hr_full", "grad", "gram", "scale_solve", "phase_hr", "babai",
  * "symmetrize", "group_factor", "slices", "slice_rows", "proj", "whw", "rhs",
  * "htilde", "ptilde", "target", "syrk", "mu_combine", "own_rhs", "scale_fit",
- * "probe", "sweep".  Not thread-safe. */
+ * "probe".  Not thread-safe. */
 void jarq_profile_enable(int on);
 void jarq_profile_reset(void);
 /* Accumulated launches and total device milliseconds of one kernel name since

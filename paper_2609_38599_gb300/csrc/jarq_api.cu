@@ -398,7 +398,6 @@ void jarq_hessian_destroy(jarq_hessian *h) {
     cudaFree(h->expo);
     cudaFree(h->Lf);
     cudaFree(h->L64);
-    cudaFree(h->Rpk);
     cudaFree(h->Rinv);
     cudaFree(h->rdig);
     cudaFree(h->rexp);
@@ -446,7 +445,6 @@ jarq_status jarq_prepare_hessian(const float *H, int din, int group_size, float 
         if ((e = make_tmap_f16(&h->mapD10, h->Hdig10, (uint64_t)4 * h->d_pad, h->d_pad, 64)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->Lf, (size_t)h->G * group_size * group_size)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->L64, (size_t)h->G * group_size * group_size)) != cudaSuccess) { rc = cuda_fail(e); break; }
-        if ((e = dalloc(&h->Rpk, (size_t)h->G * sweep_rpk_size(group_size))) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->Rinv, (size_t)h->G * group_size * group_size)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->rdig, (size_t)6 * din * group_size)) != cudaSuccess) { rc = cuda_fail(e); break; }
         if ((e = dalloc(&h->rexp, (size_t)h->G)) != cudaSuccess) { rc = cuda_fail(e); break; }
@@ -467,8 +465,6 @@ jarq_status jarq_prepare_hessian(const float *H, int din, int group_size, float 
         { ProfScope ps("symmetrize", st); e = launch_symmetrize(Hsrc, h->Hs, h->Hplanes, din, h->d_pad, nu2, st); ps.done(); count_launches(1); }
         if (e != cudaSuccess) { rc = cuda_fail(e); break; }
         { ProfScope ps("group_factor", st); e = launch_group_factor(h->Hs, h->Lf, h->L64, h->Rinv, din, group_size, h->dstatus, st); ps.done(); count_launches(1); }
-        if (e != cudaSuccess) { rc = cuda_fail(e); break; }
-        { ProfScope ps("group_factor", st); e = launch_pack_rfactor(h->Lf, h->Rpk, h->G, group_size, st); ps.done(); count_launches(1); }
         if (e != cudaSuccess) { rc = cuda_fail(e); break; }
         { ProfScope ps("slices", st); e = launch_slice_rinv(h->Rinv, h->rdig, h->rexp, din, group_size, st); ps.done(); count_launches(1); }
         if (e != cudaSuccess) { rc = cuda_fail(e); break; }
@@ -661,6 +657,8 @@ jarq_status refine_impl(jarq_hessian *h, const float *W, float *S, uint8_t *Q, c
     Workspace &w = h->ws;
     const int p = dout, d = h->din, g = h->g, G = h->G, qmax = (1 << bits) - 1;
     RUN("init_rows", 1, launch_init_rows(w.active, w.iters, w.accepted, w.ridge, w.rstat, p, st));
+    const ResidualView rv = rview(h);
+    const int nsplit = target_splits(w.p_pad, g, G);
     // target projection P = W H, w^T H w and the folded Pt, once per call
     RUN("slice_rows", 1, launch_slice_rows(la.W, w.wdig, w.wexp, p, d, h->d_pad, w.p_pad, g, st));
     RUN("proj", 1, launch_tc_proj(w.mapWd, h->mapD8, w.Phi, w.Plo, w.wexp, h->expo, p, w.p_pad, d,
@@ -683,12 +681,14 @@ jarq_status refine_impl(jarq_hessian *h, const float *W, float *S, uint8_t *Q, c
         RUN("scale_solve", 1, launch_scale_solve(w.gram, w.rhs, w.wHw, la.S, w.L_prev, L_out,
                                                  w.active, w.iters, w.ridge, w.rstat, h->dstatus,
                                                  p, d, g, k, false, o, st));
-        // the Gauss-Seidel sweep over the G groups: one launch, each row
-        // tile advancing through its phases on its own
-        RUN("sweep", 1, launch_sweep(w.mapC, h->mapHt, w.t_hi, w.t_lo, w.Pt_hi, w.Pt_lo, h->Rpk,
-                                     la.S, h->expoT, la.Q, la.Z, w.cplane, w.active, w.accepted,
-                                     h->dstatus, p, w.p_pad, d, h->d_pad, g, G, qmax, o.eps,
-                                     st));
+        for (int i = 0; i < G; ++i) {
+            RUN("target", 1, launch_tc_target(w.mapC, h->mapHt, w.t_hi, w.t_lo, la.S, h->expoT,
+                                              w.active, p, w.p_pad, h->d_pad, g, G, i, nsplit,
+                                              qmax, h->dstatus, st));
+            RUN("babai", 1, launch_babai(w.t_hi, w.t_lo, w.Pt_hi, w.Pt_lo, nsplit, h->Lf, la.S, la.Q,
+                                         la.Z, rv, w.active, w.accepted, h->dstatus, p, g, i, qmax,
+                                         o.eps, st));
+        }
     }
     // objective of the returned state (and of the input state when K = 0)
     const bool want_final = stats && stats->L_final;

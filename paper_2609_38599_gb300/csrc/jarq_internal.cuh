@@ -121,7 +121,6 @@ struct jarq_hessian {
     CUtensorMap mapD8, mapD10;    // tensor maps of Hdig8 / Hdig10, 64 x 64 boxes
     float *Lf = nullptr;          // [G][g][g] lower factor L_i = R_i^T, row-major
     double *L64 = nullptr;        // [G][g][g] the same in float64
-    float *Rpk = nullptr;         // [G][packed] R_i rows in the sweep kernel's layout
     double *Rinv = nullptr;       // [G][g][g] R_i^{-1} (upper), row-major, float64
     // R_i^{-1} in six base-2^8 digit planes, transposed per block (row i g + a,
     // column b: digit of R_i^{-1}[b][a]), one exponent per group
@@ -203,6 +202,11 @@ cudaError_t launch_scale_solve(const double *gram, const double *rhs, const doub
                                int *iters, int *ridge, int *rstat, int *status, int p, int d,
                                int g, int k, bool eval_only, const jarq_options &o,
                                cudaStream_t s);
+cudaError_t launch_babai(const float *t_hi, const float *t_lo, const float *pt_hi,
+                         const float *pt_lo, int nsplit, const float *Lf, const float *S,
+                         uint8_t *Q, const int32_t *Z, ResidualView rv, const int *active,
+                         int *accepted, int *status, int p, int g, int i, int qmax, float eps,
+                         cudaStream_t s);
 cudaError_t launch_slice_rinv(const double *Rinv, __nv_bfloat16 *rdig, int *rexp, int d, int g,
                               cudaStream_t s);
 cudaError_t launch_ptilde(const CUtensorMap &mapPd, const CUtensorMap &mapR, const float *Phi,
@@ -210,15 +214,6 @@ cudaError_t launch_ptilde(const CUtensorMap &mapPd, const CUtensorMap &mapR, con
                           float *out_hi, float *out_lo, int p, int p_pad, int d, int d_pad, int g,
                           int *status, cudaStream_t s);
 int target_splits(int p_pad, int g, int G);
-int sweep_k_parts(int g);
-int sweep_rpk_size(int g);
-cudaError_t launch_pack_rfactor(const float *Lf, float *Rpk, int G, int g, cudaStream_t s);
-cudaError_t launch_sweep(const CUtensorMap &mapC, const CUtensorMap &mapT, float *t_hi,
-                         float *t_lo, const float *pt_hi, const float *pt_lo, const float *Rpk,
-                         const float *S, const int *expoT, uint8_t *Q, const int32_t *Z,
-                         __half *cplane, const int *active, int *accepted, int *status, int p,
-                         int p_pad, int d, int d_pad, int g, int G, int qmax, float eps,
-                         cudaStream_t s);
 cudaError_t launch_tc_target(const CUtensorMap &mapC, const CUtensorMap &mapT, float *out_hi,
                              float *out_lo, const float *S, const int *expoT, const int *active,
                              int p, int p_pad, int d_pad, int g, int G, int i, int nsplit, int qmax,

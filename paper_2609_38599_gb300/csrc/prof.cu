@@ -12,7 +12,7 @@ const char *const kNames[] = {"validate", "residual", "init_rows", "hr_full", "g
                               "scale_solve", "phase_hr", "babai", "symmetrize", "group_factor",
                               "slices", "slice_rows", "proj", "whw", "rhs", "htilde", "ptilde",
                               "target", "syrk", "mu_combine", "own_rhs",
-                              "scale_fit", "probe", "sweep"};
+                              "scale_fit", "probe"};
 constexpr int kNumNames = sizeof(kNames) / sizeof(kNames[0]);
 
 struct Pending {

@@ -54,10 +54,6 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
 __device__ __forceinline__ void prefetch_tmap(const CUtensorMap *m) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(m) : "memory");
 }
-// Bring `bytes` (multiple of 16, 16-byte aligned) of global memory into L2.
-__device__ __forceinline__ void prefetch_l2(const void *p, uint32_t bytes) {
-    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
-}
 // 2D tiled load of the box at (x = inner element index, y = row) into shared
 // memory, completing `bytes` on `bar`.
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *m, uint32_t bar,
@@ -80,64 +76,6 @@ __device__ __forceinline__ uint32_t cluster_ctarank() {
 __device__ __forceinline__ void cluster_sync() {
     asm volatile("barrier.cluster.arrive.release.aligned;\n"
                  "barrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-
-// Address of the same shared-memory location in CTA `rank` of the cluster.
-__device__ __forceinline__ uint32_t map_cluster(uint32_t addr, uint32_t rank) {
-    uint32_t r;
-    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
-    return r;
-}
-// Add 1 to a counter in the shared memory of any CTA of the cluster (address
-// from map_cluster), releasing this thread's prior writes at cluster scope.
-__device__ __forceinline__ void count_up_cluster(uint32_t cluster_addr) {
-    asm volatile("red.release.cluster.shared::cluster.add.u32 [%0], 1;" ::"r"(cluster_addr)
-                 : "memory");
-}
-// Wait (bounded) until a local counter that CTAs of the cluster increment
-// reaches `target`, acquiring their writes at cluster scope.  Counters only
-// grow, so a waiter may skip any number of increments.
-__device__ __forceinline__ bool wait_count_cluster(uint32_t addr, uint32_t target) {
-#pragma unroll 1
-    for (uint32_t i = 0; i < kWaitIters; ++i) {
-        uint32_t v;
-        asm volatile("ld.acquire.cluster.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
-        if (v >= target) return true;
-    }
-    return false;
-}
-// Flags in this CTA's shared memory: a release store and a bounded polling
-// wait (acquire) until the flag reaches `target`.
-__device__ __forceinline__ void flag_store_release(uint32_t addr, uint32_t v) {
-    asm volatile("st.release.cta.shared::cta.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
-}
-// `relaxed`: sleep between polls, leaving the issue slots to warps doing
-// work (for waits that are not on a critical path).
-__device__ __forceinline__ bool flag_wait(uint32_t addr, uint32_t target, bool relaxed) {
-#pragma unroll 1
-    for (uint32_t i = 0; i < kWaitIters; ++i) {
-        uint32_t v;
-        asm volatile("ld.acquire.cta.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
-        if (v >= target) return true;
-        if (relaxed) __nanosleep(64);
-    }
-    return false;
-}
-__device__ __forceinline__ void fence_acq_rel_cluster() {
-    asm volatile("fence.acq_rel.cluster;" ::: "memory");
-}
-// Barrier over the `nthreads` threads (a multiple of 32) that name barrier `id`.
-__device__ __forceinline__ void named_bar_sync(uint32_t id, uint32_t nthreads) {
-    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
-}
-
-// Proxy fences: order this thread's generic-proxy accesses of global (or
-// shared) memory before its later async-proxy (TMA) accesses and vice versa.
-__device__ __forceinline__ void fence_proxy_async_global() {
-    asm volatile("fence.proxy.async.global;" ::: "memory");
-}
-__device__ __forceinline__ void fence_proxy_async_smem() {
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
 // Contiguous global -> shared copy of `bytes` (multiple of 16, both

@@ -119,7 +119,7 @@ def library():
 
 KERNELS = ("validate", "residual", "init_rows", "hr_full", "grad", "gram", "scale_solve",
            "phase_hr", "babai", "symmetrize", "group_factor", "slices", "slice_rows", "proj",
-           "whw", "rhs", "htilde", "ptilde", "target", "syrk", "mu_combine", "own_rhs", "scale_fit", "probe", "sweep")
+           "whw", "rhs", "htilde", "ptilde", "target", "syrk", "mu_combine", "own_rhs", "scale_fit", "probe")
 
 
 def profile_enable(on: bool = True):
