@@ -31,24 +31,32 @@
 namespace jarq {
 namespace {
 
-// In-place lower Cholesky of a G x G matrix (row stride G+1) by one warp.
-// Fails when a pivot is not above `thr` or is not finite.  Each lane owns
-// the rows a = lane (mod 32) of the trailing update; A[b][k] is read by all
-// lanes at once (a broadcast) and the rows a differ in bank (stride G + 1).
+// Offset of row a of a lower triangle stored row by row (packed).
+__device__ __forceinline__ int tri(int a) { return (a * (a + 1)) >> 1; }
+
+// In-place lower Cholesky of a G x G matrix stored as a packed lower
+// triangle, by one warp.  Fails when a pivot is not above `thr` or is not
+// finite.  Each lane owns the rows a = lane (mod 32) of the trailing update;
+// A[b][k] is read by all lanes at once (a broadcast).
 __device__ bool warp_cholesky(float *A, int G, float thr) {
-    const int lane = threadIdx.x & 31, ld = G + 1;
+    const int lane = threadIdx.x & 31;
     for (int k = 0; k < G; ++k) {
         __syncwarp();
-        const float piv = A[k * ld + k];
+        const float piv = A[tri(k) + k];
         if (!(piv > thr) || !isfinite(piv)) return false;
         const float lkk = sqrtf(piv);
         __syncwarp();
-        if (lane == 0) A[k * ld + k] = lkk;
-        for (int a = k + 1 + lane; a < G; a += 32) A[a * ld + k] /= lkk;
+        if (lane == 0) A[tri(k) + k] = lkk;
+        for (int a = k + 1 + lane; a < G; a += 32) A[tri(a) + k] /= lkk;
         __syncwarp();
         for (int a = k + 1 + lane; a < G; a += 32) {
-            const float lak = A[a * ld + k];
-            for (int b = k + 1; b <= a; ++b) A[a * ld + b] = fmaf(-lak, A[b * ld + k], A[a * ld + b]);
+            float *Aa = A + tri(a);
+            const float lak = Aa[k];
+            const float *Abk = A + tri(k + 1) + k;   // A[b][k], b = k + 1
+            for (int b = k + 1; b <= a; ++b) {
+                Aa[b] = fmaf(-lak, *Abk, Aa[b]);
+                Abk += b + 1;
+            }
         }
     }
     __syncwarp();
@@ -65,201 +73,12 @@ __device__ __forceinline__ float warp_max(float v) {
     return v;
 }
 
-struct SolveArgs {
-    const double *gram, *rhs, *wHw;
-    float *S;
-    double *L_prev;
-    double *L_out;       // optional: F(s_old) of every processed row
-    int *active, *iters, *ridge, *rstat, *status;
-    int p, d, g, k;
-    bool eval_only;
-    jarq_options o;
-};
-
-// Per-warp shared memory: float A[G][G+1], s_old[G], work[G]; double g[G], inc[G].
-__host__ __device__ inline size_t solve_warp_bytes(int G) {
-    size_t f = (size_t)G * (G + 1) + 2 * (size_t)G;
-    f = (f + 1) & ~(size_t)1;   // 8-byte alignment of the double part
-    return f * sizeof(float) + 2 * (size_t)G * sizeof(double);
-}
-
-// Forward and back substitution with the float32 factor in A: y <- (L L^T)^{-1} y.
-__device__ void warp_chol_solve(const float *A, int G, float *y) {
-    const int lane = threadIdx.x & 31, ld = G + 1;
-    for (int k = 0; k < G; ++k) {
-        __syncwarp();
-        const float yk = y[k] / A[k * ld + k];
-        __syncwarp();
-        if (lane == 0) y[k] = yk;
-        for (int t = k + 1 + lane; t < G; t += 32) y[t] = fmaf(-A[t * ld + k], yk, y[t]);
-    }
-    for (int k = G - 1; k >= 0; --k) {
-        __syncwarp();
-        const float sk = y[k] / A[k * ld + k];
-        __syncwarp();
-        if (lane == 0) y[k] = sk;
-        for (int t = lane; t < k; t += 32) y[t] = fmaf(-A[k * ld + t], sk, y[t]);
-    }
-    __syncwarp();
-}
-
-__global__ void scale_solve_kernel(SolveArgs a) {
-    extern __shared__ __align__(16) unsigned char smem_raw[];
-    const int G = a.d / a.g, ld = G + 1;
-    const int wpb = blockDim.x >> 5, w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int j = blockIdx.x * wpb + w;
-    if (j >= a.p || (!a.eval_only && !a.active[j])) return;  // warp-uniform
-    unsigned char *base = smem_raw + (size_t)w * solve_warp_bytes(G);
-    float *A = (float *)base;
-    float *so = A + G * ld;         // s_old
-    float *y = so + G;              // float work vector
-    size_t fcount = (size_t)G * ld + 2 * (size_t)G;
-    fcount = (fcount + 1) & ~(size_t)1;
-    double *b = (double *)(base + fcount * sizeof(float));   // gradient g
-    double *inc = b + G;                                      // increment of the scales
-    const double *gj = a.gram + (size_t)j * G * G;
-    const double *rj = a.rhs + (size_t)j * G;
-    // the Gram matrix is exactly symmetric: entry (r0, c0) is read as
-    // (c0, r0), so that lanes with consecutive r0 read consecutive addresses
-    auto gsym = [&](int r0, int c0) { return gj[c0 * G + r0]; };
-    for (int t = lane; t < G; t += 32) so[t] = a.S[(size_t)j * G + t];
-    __syncwarp();
-    // gradient g = rhs - Gram s_old and F(s_old) = wHw - s_old^T (rhs + g)
-    bool bfin = true;
-    double fs = 0.0;
-    for (int r0 = lane; r0 < G; r0 += 32) {
-        double gs = 0.0;
-        for (int c0 = 0; c0 < G; ++c0) gs = fma(gsym(r0, c0), (double)so[c0], gs);
-        const double gr = rj[r0] - gs;
-        b[r0] = gr;
-        fs += (double)so[r0] * (rj[r0] + gr);
-        bfin &= (bool)isfinite(gr);
-    }
-    const double F_old = a.wHw[j] - warp_sum(fs);
-    if (a.L_out && lane == 0) a.L_out[j] = F_old;
-    if (a.eval_only) return;
-    if (a.o.fixed_grid) {
-        // fixed grid: the scales stay; L^(k) is the objective of the current state
-        bool stop = false;
-        if (a.o.early_stop && a.k >= 2) {
-            const double dec = a.L_prev[j] - F_old;
-            const double den = fmax(fabs(a.L_prev[j]), (double)a.o.eps);
-            stop = (dec / den <= (double)a.o.tau_rel) || (fabs(dec) <= (double)a.o.tau_abs);
-        }
-        if (lane == 0) {
-            a.L_prev[j] = F_old;
-            a.iters[j] = a.k;
-            if (stop) a.active[j] = 0;
-        }
-        return;
-    }
-    auto load_sym = [&](float shift) -> bool {
-        bool finite = true;
-        for (int r0 = 0; r0 < G; ++r0)
-            for (int c0 = lane; c0 < G; c0 += 32) {
-                float v = (float)gj[r0 * G + c0];
-                if (r0 == c0) v += shift;
-                if (!isfinite(v)) finite = false;
-                A[r0 * ld + c0] = v;
-            }
-        __syncwarp();
-        return __all_sync(0xffffffffu, finite);
-    };
-    bool finite = load_sym(0.f);
-    float md = 0.f;
-    for (int t = lane; t < G; t += 32) md = fmaxf(md, A[t * ld + t]);
-    md = warp_max(md);
-    bool ok = finite && warp_cholesky(A, G, a.o.rcond * fmaxf(md, a.o.eps));
-    int used_ridge = 0;
-    if (!ok) {
-        used_ridge = 1;
-        load_sym(a.o.ridge);
-        ok = warp_cholesky(A, G, 0.f);
-    }
-    ok = ok && __all_sync(0xffffffffu, bfin);
-    auto fail = [&]() {
-        if (lane == 0) {
-            a.ridge[j] += used_ridge;
-            a.rstat[j] = JARQ_ERR_NUMERICAL;
-            a.active[j] = 0;
-            atomicOr(a.status, ST_NUMERICAL);
-        }
-    };
-    if (!ok) {
-        fail();
-        return;
-    }
-    // (Gram + lambda I) inc = g - lambda s_old, refined twice with float64 residuals
-    const double lam = used_ridge ? (double)a.o.ridge : 0.0;
-    for (int t = lane; t < G; t += 32) {
-        inc[t] = 0.0;
-        y[t] = (float)(b[t] - lam * (double)so[t]);
-    }
-    for (int step = 0; step < 3; ++step) {
-        warp_chol_solve(A, G, y);
-        for (int t = lane; t < G; t += 32) inc[t] += (double)y[t];
-        __syncwarp();
-        if (step == 2) break;
-        for (int r0 = lane; r0 < G; r0 += 32) {
-            double res = b[r0] - lam * ((double)so[r0] + inc[r0]);
-            for (int c0 = 0; c0 < G; ++c0) res = fma(-gsym(r0, c0), inc[c0], res);
-            y[r0] = (float)res;
-        }
-        __syncwarp();
-    }
-    bool sfin = true;
-    for (int t = lane; t < G; t += 32) sfin &= (bool)isfinite(inc[t]);
-    if (!__all_sync(0xffffffffu, sfin)) {
-        fail();
-        return;
-    }
-    for (int t = lane; t < G; t += 32) y[t] = (float)((double)so[t] + inc[t]);   // s_new
-    __syncwarp();
-    // L^{(k)} at the stored float32 scales, from the unridged symmetrised Gram
-    double t1 = 0.0, t2 = 0.0;
-    for (int r0 = lane; r0 < G; r0 += 32) {
-        double gs = 0.0;
-        for (int c0 = 0; c0 < G; ++c0) gs = fma(gsym(r0, c0), (double)y[c0], gs);
-        t1 += (double)y[r0] * rj[r0];
-        t2 += (double)y[r0] * gs;
-    }
-    double L_new = a.wHw[j] - 2.0 * warp_sum(t1) + warp_sum(t2);
-    // Remark ridge-acceptance (optional): a ridge-stabilised solve that would
-    // raise F_j is dropped and the previous scales stay
-    const bool keep_old = used_ridge && a.o.ridge_accept && !(L_new <= F_old);
-    if (keep_old) L_new = F_old;
-    bool stop = false;
-    if (a.o.early_stop && a.k >= 2) {
-        const double dec = a.L_prev[j] - L_new;
-        const double den = fmax(fabs(a.L_prev[j]), (double)a.o.eps);
-        stop = (dec / den <= (double)a.o.tau_rel) || (fabs(dec) <= (double)a.o.tau_abs);
-    }
-    if (!keep_old)
-        for (int t = lane; t < G; t += 32) a.S[(size_t)j * G + t] = y[t];
-    if (lane == 0) {
-        a.L_prev[j] = L_new;
-        a.iters[j] = a.k;
-        a.ridge[j] += used_ridge;
-        if (stop) a.active[j] = 0;
-    }
-}
-
-
 // ---------------------------------------------------------------------------
-// Register-resident solve for G <= 32 (the g = 128 layers of 4096 inputs).
-//
-// Same steps, same decisions, no bulk float64: on GB300 float64 runs at
-// about 1/64 of the float32 rate, so the dot products of the gradient, the
-// refinement residuals and the objective are done in double-float (pairs of
-// float32 with error-free products and sums, about 48 significant bits).
-// Lane l owns row l of the Gram matrix (= column l: it is exactly
-// symmetric) as a double-float pair per entry, split from the float64 with
-// integer operations.  The float32 Cholesky keeps row l in registers and
-// broadcasts the column of each step with shuffles: the same operations in
-// the same order as warp_cholesky, so the factor (and the ridge decision)
-// is bit-identical.  The triangular solves multiply by the reciprocal of
-// the pivots; the float64-accurate refinement makes the stored scales
-// independent of that rounding.
+// Double-float arithmetic (pairs of float32 with error-free products and
+// sums, about 48 significant bits): GB300 runs float64 at about 1/64 of the
+// float32 rate, so neither solve does float64 arithmetic in bulk.  The
+// Gram matrices arrive as float64 and are split into such pairs by integer
+// operations.
 // ---------------------------------------------------------------------------
 
 struct DF {
@@ -341,6 +160,261 @@ __device__ __forceinline__ DF split_double(double x) {
     const DF v = split_fast(x, rare);
     return rare ? split_slow(x) : v;
 }
+
+struct SolveArgs {
+    const double *gram, *rhs, *wHw;
+    float *S;
+    double *L_prev;
+    double *L_out;       // optional: F(s_old) of every processed row
+    int *active, *iters, *ridge, *rstat, *status;
+    int p, d, g, k;
+    bool eval_only;
+    jarq_options o;
+};
+
+// Per-warp shared memory: the packed lower factor A (G (G + 1) / 2
+// floats), s_old[G], y[G], and the double-float gradient (bh, bl) and
+// increment (ih, il), G each.
+__host__ __device__ inline size_t solve_warp_bytes(int G) {
+    return ((size_t)G * (G + 1) / 2 + 6 * (size_t)G) * sizeof(float);
+}
+
+// Forward and back substitution with the packed float32 factor in A:
+// y <- (L L^T)^{-1} y.
+__device__ void warp_chol_solve(const float *A, int G, float *y) {
+    const int lane = threadIdx.x & 31;
+    for (int k = 0; k < G; ++k) {
+        __syncwarp();
+        const float yk = y[k] / A[tri(k) + k];
+        __syncwarp();
+        if (lane == 0) y[k] = yk;
+        for (int t = k + 1 + lane; t < G; t += 32) y[t] = fmaf(-A[tri(t) + k], yk, y[t]);
+    }
+    for (int k = G - 1; k >= 0; --k) {
+        __syncwarp();
+        const float sk = y[k] / A[tri(k) + k];
+        __syncwarp();
+        if (lane == 0) y[k] = sk;
+        for (int t = lane; t < k; t += 32) y[t] = fmaf(-A[tri(k) + t], sk, y[t]);
+    }
+    __syncwarp();
+}
+
+// Row r0 of the (exactly symmetric) Gram matrix times x = xh + xl, in
+// double-float.  Entry (r0, c) is read as (c, r0), so that lanes with
+// consecutive r0 read consecutive addresses, eight loads at a time.
+template <bool kPair>
+__device__ __forceinline__ DF gram_dot(const double *gj, int G, int r0, const float *xh,
+                                       const float *xl) {
+    DF acc{0.f, 0.f};
+    auto term = [&](double v, int c) {
+        const DF e = split_double(v);
+        df_add_prod(acc, e.h, xh[c]);
+        acc.l = fmaf(e.l, xh[c], acc.l);
+        if (kPair) acc.l = fmaf(e.h, xl[c], acc.l);
+    };
+    int c = 0;
+    for (; c + 8 <= G; c += 8) {
+        double v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) v[u] = __ldg(gj + (size_t)(c + u) * G + r0);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) term(v[u], c + u);
+    }
+    for (; c < G; ++c) term(__ldg(gj + (size_t)c * G + r0), c);
+    return acc;
+}
+
+// Solve for G > 32 (e.g. 86 groups of the 11008-input layers): the Gram
+// matrix stays in global memory (L2) and is read row by row; the float32
+// factor lives in shared memory.  Every dot product with the Gram matrix --
+// the gradient, the two refinement residuals, the objective -- is summed in
+// double-float, each float64 entry split into a float pair first.
+__global__ void scale_solve_kernel(SolveArgs a) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const int G = a.d / a.g;
+    const int wpb = blockDim.x >> 5, w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int j = blockIdx.x * wpb + w;
+    if (j >= a.p || (!a.eval_only && !a.active[j])) return;  // warp-uniform
+    float *A = (float *)(smem_raw + (size_t)w * solve_warp_bytes(G));
+    float *so = A + tri(G);         // s_old
+    float *y = so + G;              // float work vector
+    float *bh = y + G, *bl = bh + G;    // gradient g (double-float)
+    float *ih = bl + G, *il = ih + G;   // increment of the scales (double-float)
+    const double *gj = a.gram + (size_t)j * G * G;
+    const double *rj = a.rhs + (size_t)j * G;
+    // the row's Gram matrix (8 G^2 bytes) is read by five or six passes:
+    // bring it into L2 once, all lines at a time
+    {
+        const char *gb = (const char *)gj;
+        const size_t bytes = (size_t)G * G * sizeof(double);
+        for (size_t off = (size_t)lane * 128; off < bytes; off += 32 * 128)
+            asm volatile("prefetch.global.L2 [%0];" ::"l"(gb + off));
+        if (lane == 0) asm volatile("prefetch.global.L2 [%0];" ::"l"(gb + bytes - 1));
+    }
+    for (int t = lane; t < G; t += 32) so[t] = a.S[(size_t)j * G + t];
+    __syncwarp();
+    // gradient g = rhs - Gram s_old and F(s_old) = wHw - s_old^T (rhs + g)
+    bool bfin = true;
+    DF fs{0.f, 0.f};
+    for (int r0 = lane; r0 < G; r0 += 32) {
+        const DF gs = gram_dot<false>(gj, G, r0, so, nullptr);
+        const DF rr = split_double(rj[r0]);
+        const DF gr = df_add(rr, df_neg(gs));
+        bh[r0] = gr.h;
+        bl[r0] = gr.l;
+        const DF rg = df_add(rr, gr);
+        df_add_prod(fs, so[r0], rg.h);
+        fs.l = fmaf(so[r0], rg.l, fs.l);
+        bfin &= (bool)isfinite(gr.h);
+    }
+    const double F_old = a.wHw[j] - df_to_double(df_warp_sum(fs));
+    if (a.L_out && lane == 0) a.L_out[j] = F_old;
+    if (a.eval_only) return;
+    if (a.o.fixed_grid) {
+        // fixed grid: the scales stay; L^(k) is the objective of the current state
+        bool stop = false;
+        if (a.o.early_stop && a.k >= 2) {
+            const double dec = a.L_prev[j] - F_old;
+            const double den = fmax(fabs(a.L_prev[j]), (double)a.o.eps);
+            stop = (dec / den <= (double)a.o.tau_rel) || (fabs(dec) <= (double)a.o.tau_abs);
+        }
+        if (lane == 0) {
+            a.L_prev[j] = F_old;
+            a.iters[j] = a.k;
+            if (stop) a.active[j] = 0;
+        }
+        return;
+    }
+    // float32 copy of the Gram matrix (the float of a split is the correctly
+    // rounded float32 of the entry), plus a ridge shift of the diagonal
+    auto load_sym = [&](float shift) -> bool {
+        bool finite = true;
+#pragma unroll 4
+        for (int r0 = 0; r0 < G; ++r0)
+            for (int c0 = lane; c0 <= r0; c0 += 32) {
+                float v = split_double(__ldg(gj + (size_t)r0 * G + c0)).h;
+                if (r0 == c0) v += shift;
+                if (!isfinite(v)) finite = false;
+                A[tri(r0) + c0] = v;
+            }
+        __syncwarp();
+        return __all_sync(0xffffffffu, finite);
+    };
+    bool finite = load_sym(0.f);
+    float md = 0.f;
+    for (int t = lane; t < G; t += 32) md = fmaxf(md, A[tri(t) + t]);
+    md = warp_max(md);
+    bool ok = finite && warp_cholesky(A, G, a.o.rcond * fmaxf(md, a.o.eps));
+    int used_ridge = 0;
+    if (!ok) {
+        used_ridge = 1;
+        load_sym(a.o.ridge);
+        ok = warp_cholesky(A, G, 0.f);
+    }
+    ok = ok && __all_sync(0xffffffffu, bfin);
+    auto fail = [&]() {
+        if (lane == 0) {
+            a.ridge[j] += used_ridge;
+            a.rstat[j] = JARQ_ERR_NUMERICAL;
+            a.active[j] = 0;
+            atomicOr(a.status, ST_NUMERICAL);
+        }
+    };
+    if (!ok) {
+        fail();
+        return;
+    }
+    // (Gram + lambda I) inc = g - lambda s_old, refined twice with
+    // double-float residuals
+    const float lam = used_ridge ? a.o.ridge : 0.f;
+    for (int t = lane; t < G; t += 32) {
+        ih[t] = 0.f;
+        il[t] = 0.f;
+        DF v{bh[t], bl[t]};
+        df_add_prod(v, -lam, so[t]);
+        y[t] = __fadd_rn(v.h, v.l);
+    }
+    for (int step = 0; step < 3; ++step) {
+        warp_chol_solve(A, G, y);
+        for (int t = lane; t < G; t += 32) {
+            const DF s2 = df_add({ih[t], il[t]}, {y[t], 0.f});
+            ih[t] = s2.h;
+            il[t] = s2.l;
+        }
+        __syncwarp();
+        if (step == 2) break;
+        for (int r0 = lane; r0 < G; r0 += 32) {
+            // res = g - lambda (s_old + inc) - Gram inc
+            DF res{bh[r0], bl[r0]};
+            df_add_prod(res, -lam, so[r0]);
+            df_add_prod(res, -lam, ih[r0]);
+            res.l = fmaf(-lam, il[r0], res.l);
+            res = df_add(res, df_neg(gram_dot<true>(gj, G, r0, ih, il)));
+            y[r0] = __fadd_rn(res.h, res.l);
+        }
+        __syncwarp();
+    }
+    bool sfin = true;
+    for (int t = lane; t < G; t += 32) sfin &= (bool)(isfinite(ih[t]) && isfinite(il[t]));
+    if (!__all_sync(0xffffffffu, sfin)) {
+        fail();
+        return;
+    }
+    // s_new = s_old + inc, rounded once to float32
+    for (int t = lane; t < G; t += 32) {
+        const DF s2 = df_add({so[t], 0.f}, {ih[t], il[t]});
+        y[t] = __fadd_rn(s2.h, s2.l);
+    }
+    __syncwarp();
+    // L^{(k)} at the stored float32 scales, from the unridged Gram matrix
+    DF t1{0.f, 0.f}, t2{0.f, 0.f};
+    for (int r0 = lane; r0 < G; r0 += 32) {
+        const DF gs = gram_dot<false>(gj, G, r0, y, nullptr);
+        const DF rr = split_double(rj[r0]);
+        df_add_prod(t1, y[r0], rr.h);
+        t1.l = fmaf(y[r0], rr.l, t1.l);
+        df_add_prod(t2, y[r0], gs.h);
+        t2.l = fmaf(y[r0], gs.l, t2.l);
+    }
+    double L_new = a.wHw[j] - 2.0 * df_to_double(df_warp_sum(t1)) + df_to_double(df_warp_sum(t2));
+    // Remark ridge-acceptance (optional): a ridge-stabilised solve that would
+    // raise F_j is dropped and the previous scales stay
+    const bool keep_old = used_ridge && a.o.ridge_accept && !(L_new <= F_old);
+    if (keep_old) L_new = F_old;
+    bool stop = false;
+    if (a.o.early_stop && a.k >= 2) {
+        const double dec = a.L_prev[j] - L_new;
+        const double den = fmax(fabs(a.L_prev[j]), (double)a.o.eps);
+        stop = (dec / den <= (double)a.o.tau_rel) || (fabs(dec) <= (double)a.o.tau_abs);
+    }
+    if (!keep_old)
+        for (int t = lane; t < G; t += 32) a.S[(size_t)j * G + t] = y[t];
+    if (lane == 0) {
+        a.L_prev[j] = L_new;
+        a.iters[j] = a.k;
+        a.ridge[j] += used_ridge;
+        if (stop) a.active[j] = 0;
+    }
+}
+
+
+// ---------------------------------------------------------------------------
+// Register-resident solve for G <= 32 (the g = 128 layers of 4096 inputs).
+//
+// Same steps, same decisions, no bulk float64: on GB300 float64 runs at
+// about 1/64 of the float32 rate, so the dot products of the gradient, the
+// refinement residuals and the objective are done in double-float (pairs of
+// float32 with error-free products and sums, about 48 significant bits).
+// Lane l owns row l of the Gram matrix (= column l: it is exactly
+// symmetric) as a double-float pair per entry, split from the float64 with
+// integer operations.  The float32 Cholesky keeps row l in registers and
+// broadcasts the column of each step with shuffles: the same operations in
+// the same order as warp_cholesky, so the factor (and the ridge decision)
+// is bit-identical.  The triangular solves multiply by the reciprocal of
+// the pivots; the float64-accurate refinement makes the stored scales
+// independent of that rounding.
+// ---------------------------------------------------------------------------
 
 // In-place lower Cholesky with lane a holding row a in A[]; on and below
 // the diagonal the operations and their order are those of warp_cholesky.
@@ -592,9 +666,11 @@ cudaError_t launch_scale_solve(const double *gram, const double *rhs, const doub
         scale_solve_small_kernel<<<(p + kSmallWarps - 1) / kSmallWarps, 32 * kSmallWarps, 0, s>>>(a);
         return cudaGetLastError();
     }
+    // at most four warps per block, and blocks small enough that several fit
+    // on an SM: the kernel is bound by the latency of each warp's chain
     const size_t per_warp = solve_warp_bytes(G);
-    int wpb = (int)((96 * 1024) / per_warp);
-    if (wpb > 8) wpb = 8;
+    int wpb = (int)((56 * 1024) / per_warp);
+    if (wpb > 4) wpb = 4;
     if (wpb < 1) wpb = 1;
     const size_t smem = per_warp * wpb;
     cudaError_t e = cudaFuncSetAttribute(scale_solve_kernel,

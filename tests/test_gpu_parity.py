@@ -77,6 +77,34 @@ def test_shapes_parity(jarq, din, dout, g, bits, K):
     assert Q.min() >= 0 and Q.max() <= (1 << bits) - 1
 
 
+def _many_group_layer(din, dout, g, bits, K, seed):
+    """A layer with the small-layer recipe whose Hessian is accumulated on
+    the GPU (torch generators), returned as NumPy arrays for the oracle."""
+    from synth.layers import hessian_torch, rtn_host_torch, weights_torch
+    H = hessian_torch(din, max(1, din // 16), 2, 20.0, 2 * din, 0.1, seed, "cuda")
+    W = weights_torch(dout, din, 0.02, 0.005, 8.0, "normal", seed + 1, "cuda")
+    S0, Q0, Z = rtn_host_torch(W, bits, g)
+    n = lambda x: x.cpu().numpy()
+    return Layer(f"many_{dout}x{din}_g{g}_w{bits}", n(W), n(H), n(S0), n(Q0), n(Z), bits, g, K)
+
+
+@pytest.mark.parametrize("din,dout,g,bits,K", [
+    (2304, 40, 64, 3, 2),     # 36 groups: the scale solve with G > 32
+    (4224, 24, 128, 4, 2),    # 33 groups of 128
+    (8192, 12, 64, 3, 1),     # 128 groups: the largest G the solve accepts
+])
+def test_many_groups_parity(jarq, din, dout, g, bits, K):
+    lay = _many_group_layer(din, dout, g, bits, K, seed=din + g)
+    prep, res = oracle_run(lay, K, False)
+    S, Q, st = gpu_refine(lay, K)
+    assert st["status"] == 0
+    m = compare_final(lay, prep, res, S, Q, st)
+    assert m["codes_same"] >= CODES_SAME, m
+    assert m["S_rel_max_same_rows"] <= REL_S and m["F_rel_max_same_rows"] <= REL_F, m
+    assert m["F_rel_all"] <= REL_F, m
+    assert m["gpu_no_worse_than_host"], m
+
+
 def test_lockstep_tiny_every_difference_is_a_near_tie(jarq):
     lay = tiny_layer()
 
