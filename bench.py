@@ -418,6 +418,7 @@ def run_ours(args, rank, world):
         line["configs"] = configs_leg(args, jarq, dev)
     if rank == 0:
         line["hessian"] = hessian_leg(args, jarq, dev)
+        line["early_stop"] = early_stop_leg(args, jarq, dev, lay, hess, ms)
         line["mu_target"] = mu_target_leg(args, jarq, dev, lay.name)
         line["ablations"] = ablation_leg(args, jarq, dev, lay, hess, ms)
     # end to end through the C ABI with pinned host buffers
@@ -767,6 +768,54 @@ def ablation_leg(args, jarq, dev, lay, hess, joint_ms):
     out["rows_improved_by_joint"] = float(np.mean(Fj < Ff))
     out["heldout"] = f"{c['tokens'] // 4} other tokens of the same distribution"
     return out
+
+
+def early_stop_leg(args, jarq, dev, lay, hess, fixed_ms):
+    """The main layer with the early stop of App. E (Eq. strict_stopping,
+    default thresholds) against the fixed K-iteration run of the main line:
+    seconds per layer, the rows' last solved iteration and, per iteration k,
+    the share of rows and of 128-row tiles still solved at k (a tile whose
+    rows have all stopped skips its phase products; stopped rows skip the
+    Babai step and the Gram)."""
+    import torch
+    opts = jarq.default_options(max_iters=lay.K, early_stop=1)
+    S = lay.S0.clone()
+    Q = lay.Q0.clone()
+
+    def step():
+        S.copy_(lay.S0)
+        Q.copy_(lay.Q0)
+        jarq.refine(hess, lay.W, S, Q, lay.Z, lay.bits, options=opts, collect_stats=False)
+
+    for _ in range(2):
+        step()
+    torch.cuda.synchronize()
+    steps = max(3, args.steps // 2)
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    n0 = jarq.launch_count()
+    a.record()
+    for _ in range(steps):
+        step()
+    b.record()
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / steps
+    launches = (jarq.launch_count() - n0) / steps
+    S.copy_(lay.S0)
+    Q.copy_(lay.Q0)
+    st = jarq.refine(hess, lay.W, S, Q, lay.Z, lay.bits, options=opts, collect_stats=True)
+    it = st.iters.cpu().numpy().astype(np.int64)
+    ntile = (len(it) + 127) // 128
+    tile_max = np.zeros(ntile * 128, np.int64)
+    tile_max[:len(it)] = it
+    tile_max = tile_max.reshape(ntile, 128).max(axis=1)
+    K = lay.K
+    return {"K": K, "tau_rel": opts.tau_rel, "tau_abs": opts.tau_abs, "steps": steps,
+            "s_per_layer": ms / 1e3, "weights_per_s": lay.din * lay.dout / (ms / 1e3),
+            "fixed_K_s_per_layer": fixed_ms / 1e3, "speedup_vs_fixed": fixed_ms / ms,
+            "launches_per_step": launches, "iters_mean": float(it.mean()),
+            "iters_hist": np.bincount(it, minlength=K + 1).tolist(),
+            "rows_solved_at_k": [float(np.mean(it >= k)) for k in range(1, K + 1)],
+            "tiles_solved_at_k": [float(np.mean(tile_max >= k)) for k in range(1, K + 1)]}
 
 
 def mu_target_leg(args, jarq, dev, name):

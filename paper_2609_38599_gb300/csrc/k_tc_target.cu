@@ -49,7 +49,7 @@ struct TargetArgs {
     float *out_hi, *out_lo;   // [nsplit][p_pad][g]
     const float *S;           // [p][G]
     const int *expoT;         // [G][G] block exponents of Ht
-    const int *active;
+    const int *active;        // optional: rows still refined
     int *status;
     int p, p_pad, d_pad, g, G, i, seg_per_split;
     float round_c;            // 1.5 * 2^(23 - k): rounds to multiples of 2^-k
@@ -74,9 +74,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int m0 = a.i * a.g + blockIdx.y * 64;          // first row of Ht (output column)
     const int h0 = blockIdx.z * a.seg_per_split;
     const int h1 = min(a.G, h0 + a.seg_per_split);
-    const int nseg = max(0, h1 - h0);
     const int nkc = a.g / 64;
-    const int nchunks = nseg * nkc;
 
     auto full = [&](int s) { return tc::smem_u32(bars + s); };
     auto empty = [&](int s) { return tc::smem_u32(bars + kStages + s); };
@@ -112,6 +110,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     // the codes are rewritten by the previous Babai phase
     tc::pdl_wait();
     tc::pdl_launch_dependents();
+    // a tile none of whose rows is still active (early stop, App. E) does
+    // no work: the Babai step reads the partials of active rows only
+    const bool live = __syncthreads_or(threadIdx.x < 128 && j0 + (int)threadIdx.x < a.p &&
+                                       (!a.active || a.active[j0 + threadIdx.x] != 0));
+    const int nseg = live ? max(0, h1 - h0) : 0;
+    const int nchunks = nseg * nkc;
 
     if (warp == 0 && lane == 0) {
         // ---------------- producer
