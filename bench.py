@@ -81,6 +81,9 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-configs", action="store_true",
                     help="skip timing the other workloads (tiny, down_proj, gate_proj, block)")
+    ap.add_argument("--main-only", action="store_true",
+                    help="time the main workload only: no post-passes, other workloads, "
+                         "extra legs, end-to-end pass or CPU baseline (profiling runs)")
     ap.add_argument("--tokens", type=int, default=None,
                     help="calibration tokens of the Hessian workload (default: 128 x 2048)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
@@ -387,7 +390,7 @@ def run_ours(args, rank, world):
     # write-back post-passes on the refined layer (not part of the step): the
     # returned weights cast to float16, the packed codes, canonicalisation
     post = {}
-    if rank == 0:
+    if rank == 0 and not args.main_only:
         pk2, _ = peaks()
 
         def timed(fn, reps=5):
@@ -414,15 +417,15 @@ def run_ours(args, rank, world):
                           "hbm_frac": by / (ms_ / 1e3) / 1e9 / pk2["hbm_gbs"],
                           "note": "includes the code validation pass and a synchronize"}
         line["postpass"] = post
-    if rank == 0 and not args.no_configs:
+    if rank == 0 and not args.no_configs and not args.main_only:
         line["configs"] = configs_leg(args, jarq, dev)
-    if rank == 0:
+    if rank == 0 and not args.main_only:
         line["hessian"] = hessian_leg(args, jarq, dev)
         line["early_stop"] = early_stop_leg(args, jarq, dev, lay, hess, ms)
         line["mu_target"] = mu_target_leg(args, jarq, dev, lay.name)
         line["ablations"] = ablation_leg(args, jarq, dev, lay, hess, ms)
     # end to end through the C ABI with pinned host buffers
-    if rank == 0 or True:
+    if not args.main_only:
         pin = lambda t: t.cpu().pin_memory().numpy()
         Wh, S0h, Q0h, Zh = pin(lay.W), pin(lay.S0), pin(lay.Q0), pin(lay.Z)
         Sh = torch.empty_like(lay.S0, device="cpu").pin_memory().numpy()
@@ -445,7 +448,7 @@ def run_ours(args, rank, world):
                        "h2d_bytes_per_step": int(Wh.nbytes + S0h.nbytes + Q0h.nbytes + Zh.nbytes),
                        "d2h_bytes_per_step": int(Sh.nbytes + Qh.nbytes),
                        "ms_per_step": e2e_s * 1e3}
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and not args.main_only:
         lay_np = layer_to_numpy(lay)
         rows, t = oracle_rows_per_second(lay_np, lay.K, args.cpu_seconds)
         line["cpu_baseline"] = {"value": rows * lay.din / t, "unit": UNIT,

@@ -12,9 +12,10 @@
 // is exact whatever the accumulator's rounding.  The epilogue forms the
 // integer dots G_t = sum_{m in grp i} c_j[m] D_t[j, m] and
 //     Gram_j[i,h] = 2^(E_ih - 9) (G_0 + G_1 2^-10 + G_2 2^-20 + G_3 2^-30)
-// in float64.  Only h <= i is computed; the block is mirrored.  A CTA owns
-// one 128-row tile and the group pair {i, G-1-i}, so every CTA processes
-// G + 1 blocks.
+// in float64.  Only h <= i is computed; the block is mirrored.  The pair of
+// groups {i, G-1-i} of a 128-row tile holds G + 1 blocks; a CTA owns one of
+// `nparts` contiguous ranges of them (the host picks nparts so that the
+// CTAs fill the SMs' last wave).
 //
 // Roles: warp 0 TMA producer; warp 1 TMEM allocation and MMA issuer;
 // warps 2..9 epilogue: warp w reads TMEM lanes 32 (w % 4) .. and 32 of the
@@ -59,6 +60,7 @@ struct GramArgs {
     double *gram;        // [p][G][G]
     int *status;
     int p, d, g, G, d_pad;
+    int nparts;          // block ranges per (row tile, group pair): blockIdx.z
 };
 
 __device__ __forceinline__ int exact_int(float x) {
@@ -100,7 +102,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int ngrp = (i_lo == i_hi) ? 1 : 2;
     auto group_of = [&](int n) { return n == 0 ? i_lo : i_hi; };
     const int units0 = (i_lo + 1) * nhalf;
-    const int nunits = units0 + (ngrp == 2 ? (i_hi + 1) * nhalf : 0);
+    const int nunits_pair = units0 + (ngrp == 2 ? (i_hi + 1) * nhalf : 0);
+    // this CTA's blocks: [nblk z / nparts, nblk (z + 1) / nparts) of the pair's
+    const int nblk = nunits_pair / nhalf;
+    const int ub = (nblk * (int)blockIdx.z / a.nparts) * nhalf;
+    const int nunits = (nblk * ((int)blockIdx.z + 1) / a.nparts) * nhalf - ub;
     auto unit = [&](int u, int &gi, int &h, int &half) {
         const int n = u < units0 ? 0 : 1;
         const int r = u < units0 ? u : u - units0;
@@ -152,7 +158,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 break;
             }
             int gi, h, half;
-            unit(c / nkc, gi, h, half);
+            unit(ub + c / nkc, gi, h, half);
             const int kx = h * g + (c % nkc) * 64;
             tc::mbar_expect_tx(full(s), kStage);
             tc::tma_load_2d(tileA(s), &mapC, full(s), kx, j0);
@@ -200,7 +206,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         long long acc[4] = {0, 0, 0, 0};
         for (int u = 0; u < nunits; ++u) {
             int gi, h, half;
-            unit(u, gi, h, half);
+            unit(ub + u, gi, h, half);
             if (gi != cur_g) {
                 // stage this warp's columns of group gi (row rl written by its own thread)
                 __syncwarp();
@@ -483,8 +489,23 @@ cudaError_t launch_tc_gram(const CUtensorMap &mapC, const CUtensorMap &mapS, con
         e = set_max_dynamic_smem((const void *)tc_gram_kernel<true>, gram_smem<true>(), attr_wide);
     if (e != cudaSuccess) return e;
     const int G = d / g;
-    GramArgs a{Q, Z, expo, active, gram, status, p, d, g, G, d_pad};
-    dim3 grid(p_pad / 128, (G + 1) / 2, 1);
+    // parts per (row tile, group pair), 1 to 4: the fewest waves of CTAs,
+    // each wave as long as one part of the pair's blocks plus a fixed cost
+    // of about 5 % of the whole pair
+    const int nsm = num_sms();
+    const long long ctas = (long long)(p_pad / 128) * ((G + 1) / 2);
+    int nparts = 1;
+    double best = 0.0;
+    for (int n = 1; n <= 4 && n <= G + 1; ++n) {
+        const long long waves = (ctas * n + nsm - 1) / nsm;
+        const double t = (double)waves * (1.0 / n + 0.05);
+        if (n == 1 || t < best - 1e-9) {
+            best = t;
+            nparts = n;
+        }
+    }
+    GramArgs a{Q, Z, expo, active, gram, status, p, d, g, G, d_pad, nparts};
+    dim3 grid(p_pad / 128, (G + 1) / 2, nparts);
     if (bits <= 4)
         tc_gram_kernel<false><<<grid, kThreads, gram_smem<false>(), s>>>(mapC, mapS, a);
     else
