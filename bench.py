@@ -39,18 +39,22 @@ FP32_LANES_PER_SM = 128
 SM_MAX_MHZ = 2070.0
 DTYPE = "f32 (integer-digit fp16/bf16 tensor-core products with exact partial sums, double-float accumulation)"
 
-# DRAM bytes (read + write) per launch from one ncu capture of this workload
-# (the sweep kernels' figures are those of the first phase; the Hessian
+# DRAM bytes (read + write) per launch from one ncu capture of the main
+# workload (q_proj; other workloads report null; the sweep kernels' figures
+# are those of the first phase; the Hessian
 # kernel's is a capture at 32768 tokens scaled to the full token count); the
 # summaries kept with the profiles give each capture's command.  A figure is
 # valid while the kernel's source file is unchanged (first 12 hex digits of
 # its SHA-1); otherwise the bench reports null.
 TRAFFIC = {
-    "target": ("k_tc_target.cu", "4ae89381851e", 38.299e6 + 0.152e6),
-    "babai": ("k_babai.cu", "d2d96a20da85", 14.274e6 + 0.001536e6),
-    "gram": ("k_tc_gram.cu", "38618e3a1081", 164.122e6 + 27.549e6),
-    "proj": ("k_tc_proj.cu", "6cf1b3d8cc4f", 1370.069e6 + 156.471e6),
+    "target": ("k_tc_target.cu", "fa2cb98ffc26", 38.313e6 + 0.0),
+    "babai": ("k_babai.cu", "d2d96a20da85", 14.274e6 + 0.003072e6),
+    "gram": ("k_tc_gram.cu", "abf8bda799a6", 146.620e6 + 24.483e6),
+    "proj": ("k_tc_proj.cu", "6cf1b3d8cc4f", 1370.489e6 + 154.061e6),
     "ptilde": ("k_tc_proj.cu", "6cf1b3d8cc4f", 134.248e6 + 150.687e6 + 222.887e6 + 103.208e6),
+    "rhs": ("k_tc_proj.cu", "6cf1b3d8cc4f", 151.550e6 + 0.255e6),
+    "whw": ("k_tc_proj.cu", "6cf1b3d8cc4f", 201.342e6 + 0.062e6),
+    "slice_rows": ("k_tc_proj.cu", "6cf1b3d8cc4f", 67.124e6 + 81.547e6),
     "scale_solve": ("k_solve.cu", "326c857f6b6b", 35.309e6 + 0.000256e6),
     # captured at 32768 tokens, scaled to 262144
     "syrk": ("k_syrk.cu", "3896afedc783", 8 * 537.171e6 + 40.712e6),
@@ -224,9 +228,13 @@ def run_reference(args, rank, world):
 
 
 def config_dict(lay, note=None):
+    MB = 1 << 20
+    pd, dd = lay.dout * lay.din, ((lay.din + 127) // 128 * 128) ** 2
     c = {"workload": lay.name, "din": lay.din, "dout": lay.dout, "group_size": lay.g,
          "bits": lay.bits, "K": lay.K, "early_stop": False, "host": "RTN",
-         "l2": "inputs larger than L2 (per step: W, P and the folded P 64 MB each, digit planes of H 336 MB)"}
+         "l2": f"inputs larger than L2 (per step: W {4 * pd // MB} MB, P and the folded P "
+               f"{8 * pd // MB} MB each as float pairs, digit planes of H and of the folded "
+               f"rows {28 * dd // MB} MB)"}
     if note:
         c["note"] = note
     return c
@@ -294,7 +302,9 @@ def roofline_entry(kernel, stats, lay, pk, peak_kind):
         peak, unit = pk["hbm_gbs"], "GB/s"
         note = f"HBM copy bandwidth ({peak_kind})"
     e = {"kernel": kernel, "bound": m["bound"], "achieved": achieved, "peak": peak, "unit": unit,
-         "frac": achieved / peak, "traffic": traffic_for(kernel), "avg_us": avg_s * 1e6,
+         "frac": achieved / peak,
+         "traffic": traffic_for(kernel) if lay.name == WORKLOAD else None,
+         "avg_us": avg_s * 1e6,
          "peak_note": note}
     if "issued" in m:
         e["issued_frac"] = m["issued"] / avg_s / 1e12 / peak

@@ -68,7 +68,7 @@ struct Workspace {
     int p_pad = 0;               // rows of the bf16 residual planes (multiple of 128)
     float *Hr = nullptr;         // [p][d]  H r for every row (objective entry point)
     float *r = nullptr;          // [p][d]  residual r = w - D_s (q - z)
-    double *gram = nullptr;      // [p][G][G]  Gram matrices of the current codes
+    float2 *gram = nullptr;      // [p][G][G]  Gram matrices of the current codes (float pairs)
     double *rhs = nullptr;       // [p][G]  rhs_i = c_i^T P_i (also the scratch of grad)
     float *t_hi = nullptr;       // [nsplit][p_pad][g]  split-K partials of the phase
     float *t_lo = nullptr;       //   product T_i (double-float)
@@ -151,7 +151,7 @@ cudaError_t launch_group_factor(const float *Hs, float *Lf, double *L64, double 
                                 int g, int *status, cudaStream_t s);
 cudaError_t launch_own_rhs(const float *Hs, const float *W, const uint8_t *Q, const int32_t *Z,
                            double *own, int p, int d, int g, cudaStream_t s);
-cudaError_t launch_scale_fit(const double *gram, const double *rhs, const double *own,
+cudaError_t launch_scale_fit(const float2 *gram, const double *rhs, const double *own,
                              const double *wHw, float *S, double *F_before, double *F_after, int p,
                              int G, int method, int passes, cudaStream_t s);
 cudaError_t launch_probe(const float *Phi, const float *Plo, const float *t_hi, const float *t_lo,
@@ -180,7 +180,7 @@ cudaError_t launch_grad(const uint8_t *Q, const int32_t *Z, const float *r, cons
 cudaError_t launch_slices(const float *Hs, int *expo, __nv_bfloat16 *dig8, __half *dig10, int d,
                           int d_pad, int g, cudaStream_t s);
 cudaError_t launch_tc_gram(const CUtensorMap &mapC, const CUtensorMap &mapS, const uint8_t *Q,
-                           const int32_t *Z, const int *expo, const int *active, double *gram,
+                           const int32_t *Z, const int *expo, const int *active, float2 *gram,
                            int p, int p_pad, int d, int d_pad, int g, int bits, int *status,
                            cudaStream_t s);
 cudaError_t launch_slices8(const float *M, int *expo, __nv_bfloat16 *dig8, int d, int d_pad,
@@ -197,7 +197,7 @@ cudaError_t launch_whw(const float *W, const float *Phi, const float *Plo, doubl
                        int d, cudaStream_t s);
 cudaError_t launch_rhs(const uint8_t *Q, const int32_t *Z, const float *Phi, const float *Plo,
                        const int *active, double *rhs, int p, int d, int g, cudaStream_t s);
-cudaError_t launch_scale_solve(const double *gram, const double *rhs, const double *wHw, float *S,
+cudaError_t launch_scale_solve(const float2 *gram, const double *rhs, const double *wHw, float *S,
                                double *L_prev, double *L_out, int *active,
                                int *iters, int *ridge, int *rstat, int *status, int p, int d,
                                int g, int k, bool eval_only, const jarq_options &o,

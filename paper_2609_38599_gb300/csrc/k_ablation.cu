@@ -85,14 +85,25 @@ __global__ void own_rhs_kernel(const float *__restrict__ Hs, const float *__rest
 }
 
 struct FitArgs {
-    const double *gram, *rhs, *own, *wHw;
+    const float2 *gram;   // [p][G][G] float pairs (hi, lo)
+    const double *rhs, *own, *wHw;
     float *S;
     double *F_before, *F_after;
     int p, G, method, passes;
 };
 
+// A row's Gram matrix read as float64: each entry is stored as a float
+// pair (hi, lo), whose sum is exact in float64.
+struct PairRow {
+    const float2 *p;
+    __device__ double operator[](size_t i) const {
+        const float2 e = p[i];
+        return (double)e.x + (double)e.y;
+    }
+};
+
 // F(s) = wHw - 2 s^T rhs + s^T Gram s for the scales in s (shared memory).
-__device__ double row_objective(const double *gj, const double *rj, double wHw, const double *s,
+__device__ double row_objective(PairRow gj, const double *rj, double wHw, const double *s,
                                 int G) {
     const int lane = threadIdx.x & 31;
     double t = 0.0;
@@ -112,7 +123,8 @@ __global__ void scale_fit_kernel(FitArgs a) {
     if (j >= a.p) return;                                    // warp-uniform
     const int G = a.G;
     double *s = sm + (size_t)warp * 2 * G, *grad = s + G;
-    const double *gj = a.gram + (size_t)j * G * G, *rj = a.rhs + (size_t)j * G;
+    const PairRow gj{a.gram + (size_t)j * G * G};
+    const double *rj = a.rhs + (size_t)j * G;
     for (int t = lane; t < G; t += 32) s[t] = (double)a.S[(size_t)j * G + t];
     __syncwarp();
     const double Fb = row_objective(gj, rj, a.wHw[j], s, G);
@@ -327,7 +339,7 @@ cudaError_t launch_own_rhs(const float *Hs, const float *W, const uint8_t *Q, co
     return cudaGetLastError();
 }
 
-cudaError_t launch_scale_fit(const double *gram, const double *rhs, const double *own,
+cudaError_t launch_scale_fit(const float2 *gram, const double *rhs, const double *own,
                              const double *wHw, float *S, double *F_before, double *F_after, int p,
                              int G, int method, int passes, cudaStream_t s) {
     const int wpb = 8;

@@ -26,6 +26,7 @@
 // row.
 #include <float.h>
 
+#include "df.cuh"
 #include "jarq_internal.cuh"
 
 namespace jarq {
@@ -52,11 +53,21 @@ __device__ bool warp_cholesky(float *A, int G, float thr) {
         for (int a = k + 1 + lane; a < G; a += 32) {
             float *Aa = A + tri(a);
             const float lak = Aa[k];
-            const float *Abk = A + tri(k + 1) + k;   // A[b][k], b = k + 1
-            for (int b = k + 1; b <= a; ++b) {
-                Aa[b] = fmaf(-lak, *Abk, Aa[b]);
-                Abk += b + 1;
+            // A[b][k] (rows b > k, column k) and A[a][b] (row a, columns
+            // b > k) never overlap: four of each are loaded before the
+            // four updates are stored
+            int b = k + 1;
+            for (; b + 3 <= a; b += 4) {
+                const int t0 = tri(b) + k;
+                const float c0 = A[t0], c1 = A[t0 + b + 1], c2 = A[t0 + 2 * b + 3],
+                            c3 = A[t0 + 3 * b + 6];
+                const float x0 = Aa[b], x1 = Aa[b + 1], x2 = Aa[b + 2], x3 = Aa[b + 3];
+                Aa[b] = fmaf(-lak, c0, x0);
+                Aa[b + 1] = fmaf(-lak, c1, x1);
+                Aa[b + 2] = fmaf(-lak, c2, x2);
+                Aa[b + 3] = fmaf(-lak, c3, x3);
             }
+            for (; b <= a; ++b) Aa[b] = fmaf(-lak, A[tri(b) + k], Aa[b]);
         }
     }
     __syncwarp();
@@ -73,96 +84,9 @@ __device__ __forceinline__ float warp_max(float v) {
     return v;
 }
 
-// ---------------------------------------------------------------------------
-// Double-float arithmetic (pairs of float32 with error-free products and
-// sums, about 48 significant bits): GB300 runs float64 at about 1/64 of the
-// float32 rate, so neither solve does float64 arithmetic in bulk.  The
-// Gram matrices arrive as float64 and are split into such pairs by integer
-// operations.
-// ---------------------------------------------------------------------------
-
-struct DF {
-    float h, l;
-};
-
-__device__ __forceinline__ DF df_two_sum(float a, float b) {
-    const float s = __fadd_rn(a, b);
-    const float bb = __fsub_rn(s, a);
-    const float e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
-    return {s, e};
-}
-
-// (h, l) += x * y: the exact product x y = p + pe, p added by two_sum
-__device__ __forceinline__ void df_add_prod(DF &a, float x, float y) {
-    const float p = __fmul_rn(x, y);
-    const float pe = __fmaf_rn(x, y, -p);
-    const DF s = df_two_sum(a.h, p);
-    a.h = s.h;
-    a.l = __fadd_rn(a.l, __fadd_rn(s.l, pe));
-}
-
-__device__ __forceinline__ DF df_add(DF a, DF b) {
-    const DF s = df_two_sum(a.h, b.h);
-    return {s.h, __fadd_rn(s.l, __fadd_rn(a.l, b.l))};
-}
-
-__device__ __forceinline__ DF df_neg(DF a) { return {-a.h, -a.l}; }
-
-__device__ __forceinline__ DF df_warp_sum(DF a) {
-    // two_sum is exact, so both lanes of a butterfly pair form the same value
-    for (int o = 16; o; o >>= 1) {
-        const DF b{__shfl_xor_sync(0xffffffffu, a.h, o), __shfl_xor_sync(0xffffffffu, a.l, o)};
-        a = df_add(a, b);
-    }
-    return a;
-}
-
-__device__ __forceinline__ double df_to_double(DF a) { return (double)a.h + (double)a.l; }
-
-// x = hi + lo with hi = x rounded to float32 (nearest, ties to even) and
-// lo = x - hi rounded to float32, by integer operations on the bits of x.
-// Branch-free for zero and for 2^-74 <= |x| < 2^126; any other value
-// (tiny, huge, non-finite) sets `rare` and must be split by split_slow.
-__device__ __forceinline__ DF split_fast(double x, bool &rare) {
-    const unsigned long long bits = (unsigned long long)__double_as_longlong(x);
-    const unsigned long long u = bits & 0x7FFFFFFFFFFFFFFFull;
-    const int ex = (int)(u >> 52);
-    rare = (u != 0) && (ex < 949 || ex > 1148);
-    // keep the top 24 significant bits, round to nearest even; a carry out
-    // of the mantissa moves into the exponent field, which is still exact
-    unsigned long long keep = u >> 29;
-    const unsigned long long rem = u & ((1ull << 29) - 1);
-    keep += (rem > (1ull << 28)) || (rem == (1ull << 28) && (keep & 1ull));
-    // float32 bits: re-bias the exponent from 1023 to 127
-    const uint32_t hb = (uint32_t)(keep - (896ull << 23));
-    // x - hi in units of x's last place (|r| <= 2^28), times 2^(ex - 1075)
-    const int r = (int)(long long)(u - (keep << 29));
-    const float unit = __uint_as_float((uint32_t)((ex - 948) & 0xFF) << 23);
-    float h = __uint_as_float(hb), l = __fmul_rn(__int2float_rn(r), unit);
-    if (u == 0) {
-        h = 0.f;
-        l = 0.f;
-    }
-    if (bits >> 63) {
-        h = -h;
-        l = -l;
-    }
-    return {h, l};
-}
-
-__device__ __noinline__ DF split_slow(double x) {
-    const float h = __double2float_rn(x);
-    return {h, __double2float_rn(x - (double)h)};
-}
-
-__device__ __forceinline__ DF split_double(double x) {
-    bool rare;
-    const DF v = split_fast(x, rare);
-    return rare ? split_slow(x) : v;
-}
-
 struct SolveArgs {
-    const double *gram, *rhs, *wHw;
+    const float2 *gram;  // [p][G][G] Gram matrices as float pairs (hi, lo)
+    const double *rhs, *wHw;
     float *S;
     double *L_prev;
     double *L_out;       // optional: F(s_old) of every processed row
@@ -179,23 +103,53 @@ __host__ __device__ inline size_t solve_warp_bytes(int G) {
     return ((size_t)G * (G + 1) / 2 + 6 * (size_t)G) * sizeof(float);
 }
 
-// Forward and back substitution with the packed float32 factor in A:
-// y <- (L L^T)^{-1} y.
+// Forward and back substitution with the packed float32 factor in A,
+// y <- (L L^T)^{-1} y, for G <= 128: lane l keeps y[l + 32 m] in a
+// register, multiplies by the pivots' reciprocals, and each solved value
+// reaches the other lanes by a shuffle.  y is read and written in shared
+// memory.
 __device__ void warp_chol_solve(const float *A, int G, float *y) {
     const int lane = threadIdx.x & 31;
-    for (int k = 0; k < G; ++k) {
-        __syncwarp();
-        const float yk = y[k] / A[tri(k) + k];
-        __syncwarp();
-        if (lane == 0) y[k] = yk;
-        for (int t = k + 1 + lane; t < G; t += 32) y[t] = fmaf(-A[tri(t) + k], yk, y[t]);
+    float v[4], rd[4];
+#pragma unroll
+    for (int m = 0; m < 4; ++m) {
+        const int t = lane + 32 * m;
+        v[m] = t < G ? y[t] : 0.f;
+        rd[m] = t < G ? 1.0f / A[tri(t) + t] : 0.f;
     }
-    for (int k = G - 1; k >= 0; --k) {
-        __syncwarp();
-        const float sk = y[k] / A[tri(k) + k];
-        __syncwarp();
-        if (lane == 0) y[k] = sk;
-        for (int t = lane; t < k; t += 32) y[t] = fmaf(-A[tri(k) + t], sk, y[t]);
+#pragma unroll
+    for (int m = 0; m < 4; ++m) {
+        for (int kk = 0; kk < 32; ++kk) {
+            const int k = 32 * m + kk;
+            if (k >= G) break;   // warp-uniform
+            const float yk = __shfl_sync(0xffffffffu, v[m] * rd[m], kk);
+            if (lane == kk) v[m] = yk;
+#pragma unroll
+            for (int mm = m; mm < 4; ++mm) {
+                const int t = lane + 32 * mm;
+                if (t > k && t < G) v[mm] = fmaf(-A[tri(t) + k], yk, v[mm]);
+            }
+        }
+    }
+#pragma unroll
+    for (int m = 3; m >= 0; --m) {
+        for (int kk = 31; kk >= 0; --kk) {
+            const int k = 32 * m + kk;
+            if (k >= G) continue;   // warp-uniform
+            const float sk = __shfl_sync(0xffffffffu, v[m] * rd[m], kk);
+            if (lane == kk) v[m] = sk;
+#pragma unroll
+            for (int mm = 0; mm <= m; ++mm) {
+                const int t = lane + 32 * mm;
+                if (t < k) v[mm] = fmaf(-A[tri(k) + t], sk, v[mm]);
+            }
+        }
+    }
+    __syncwarp();
+#pragma unroll
+    for (int m = 0; m < 4; ++m) {
+        const int t = lane + 32 * m;
+        if (t < G) y[t] = v[m];
     }
     __syncwarp();
 }
@@ -204,18 +158,17 @@ __device__ void warp_chol_solve(const float *A, int G, float *y) {
 // double-float.  Entry (r0, c) is read as (c, r0), so that lanes with
 // consecutive r0 read consecutive addresses, eight loads at a time.
 template <bool kPair>
-__device__ __forceinline__ DF gram_dot(const double *gj, int G, int r0, const float *xh,
+__device__ __forceinline__ DF gram_dot(const float2 *gj, int G, int r0, const float *xh,
                                        const float *xl) {
     DF acc{0.f, 0.f};
-    auto term = [&](double v, int c) {
-        const DF e = split_double(v);
-        df_add_prod(acc, e.h, xh[c]);
-        acc.l = fmaf(e.l, xh[c], acc.l);
-        if (kPair) acc.l = fmaf(e.h, xl[c], acc.l);
+    auto term = [&](float2 e, int c) {
+        df_add_prod(acc, e.x, xh[c]);
+        acc.l = fmaf(e.y, xh[c], acc.l);
+        if (kPair) acc.l = fmaf(e.x, xl[c], acc.l);
     };
     int c = 0;
     for (; c + 8 <= G; c += 8) {
-        double v[8];
+        float2 v[8];
 #pragma unroll
         for (int u = 0; u < 8; ++u) v[u] = __ldg(gj + (size_t)(c + u) * G + r0);
 #pragma unroll
@@ -241,7 +194,7 @@ __global__ void scale_solve_kernel(SolveArgs a) {
     float *y = so + G;              // float work vector
     float *bh = y + G, *bl = bh + G;    // gradient g (double-float)
     float *ih = bl + G, *il = ih + G;   // increment of the scales (double-float)
-    const double *gj = a.gram + (size_t)j * G * G;
+    const float2 *gj = a.gram + (size_t)j * G * G;
     const double *rj = a.rhs + (size_t)j * G;
     // the row's Gram matrix (8 G^2 bytes) is read by five or six passes:
     // bring it into L2 once, all lines at a time
@@ -293,7 +246,7 @@ __global__ void scale_solve_kernel(SolveArgs a) {
 #pragma unroll 4
         for (int r0 = 0; r0 < G; ++r0)
             for (int c0 = lane; c0 <= r0; c0 += 32) {
-                float v = split_double(__ldg(gj + (size_t)r0 * G + c0)).h;
+                float v = __ldg(gj + (size_t)r0 * G + c0).x;
                 if (r0 == c0) v += shift;
                 if (!isfinite(v)) finite = false;
                 A[tri(r0) + c0] = v;
@@ -471,27 +424,17 @@ __global__ void __launch_bounds__(32 * kSmallWarps, 4) scale_solve_small_kernel(
     const int j = blockIdx.x * kSmallWarps + w;
     if (j >= a.p || (!a.eval_only && !a.active[j])) return;  // warp-uniform
     const bool own = lane < G;
-    const double *gj = a.gram + (size_t)j * G * G;
+    const float2 *gj = a.gram + (size_t)j * G * G;
     // row `lane` of the Gram matrix, read column-wise (coalesced) by
     // symmetry: every load is issued before the first is used
-    double gx[32];
-#pragma unroll
-    for (int c = 0; c < 32; ++c) gx[c] = (own && c < G) ? gj[(size_t)c * G + lane] : 0.0;
-    const float so = own ? a.S[(size_t)j * G + lane] : 0.f;
-    const double rhs_d = own ? a.rhs[(size_t)j * G + lane] : 0.0;
     DF gr[32];
-    uint32_t rare = 0;
 #pragma unroll
     for (int c = 0; c < 32; ++c) {
-        bool rc;
-        gr[c] = split_fast(gx[c], rc);
-        rare |= (uint32_t)rc << c;
+        const float2 e = (own && c < G) ? gj[(size_t)c * G + lane] : make_float2(0.f, 0.f);
+        gr[c] = DF{e.x, e.y};
     }
-    if (__any_sync(0xffffffffu, rare != 0)) {
-#pragma unroll
-        for (int c = 0; c < 32; ++c)
-            if ((rare >> c) & 1u) gr[c] = split_slow(gj[(size_t)c * G + lane]);
-    }
+    const float so = own ? a.S[(size_t)j * G + lane] : 0.f;
+    const double rhs_d = own ? a.rhs[(size_t)j * G + lane] : 0.0;
     const DF rh = split_double(rhs_d);
 
     // gradient g = rhs - Gram s_old and F(s_old) = wHw - s_old^T (rhs + g)
@@ -654,7 +597,7 @@ __global__ void __launch_bounds__(32 * kSmallWarps, 4) scale_solve_small_kernel(
 
 }  // namespace
 
-cudaError_t launch_scale_solve(const double *gram, const double *rhs, const double *wHw, float *S,
+cudaError_t launch_scale_solve(const float2 *gram, const double *rhs, const double *wHw, float *S,
                                double *L_prev, double *L_out, int *active,
                                int *iters, int *ridge, int *rstat, int *status, int p, int d,
                                int g, int k, bool eval_only, const jarq_options &o,

@@ -25,6 +25,7 @@
 // plane), double-buffered in 512 TMEM columns.
 #include <type_traits>
 
+#include "df.cuh"
 #include "tc_common.cuh"
 
 namespace jarq {
@@ -57,7 +58,7 @@ struct GramArgs {
     const int32_t *Z;
     const int *expo;     // [G][G] block exponents E_ih
     const int *active;   // optional: rows whose Gram matrix is needed
-    double *gram;        // [p][G][G]
+    float2 *gram;        // [p][G][G] as float pairs (hi, lo) of the float64 value
     int *status;
     int p, d, g, G, d_pad;
     int nparts;          // block ranges per (row tile, group pair): blockIdx.z
@@ -327,9 +328,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                                       ldexp((double)acc[2], -20) + ldexp((double)acc[3], -30),
                                   E - 9);
                     }
-                    double *gr = a.gram + (size_t)row * G * G;
-                    gr[(size_t)gi * G + h] = v;
-                    gr[(size_t)h * G + gi] = v;
+                    // stored once as the float pair the scale solve works on
+                    const DF vp = split_double(v);
+                    const float2 v2 = make_float2(vp.h, vp.l);
+                    float2 *gr = a.gram + (size_t)row * G * G;
+                    gr[(size_t)gi * G + h] = v2;
+                    gr[(size_t)h * G + gi] = v2;
                 }
 #pragma unroll
                 for (int t = 0; t < 4; ++t) acc[t] = 0;
@@ -479,7 +483,7 @@ cudaError_t launch_slices8(const float *M, int *expo, __nv_bfloat16 *dig8, int d
 }
 
 cudaError_t launch_tc_gram(const CUtensorMap &mapC, const CUtensorMap &mapS, const uint8_t *Q,
-                           const int32_t *Z, const int *expo, const int *active, double *gram,
+                           const int32_t *Z, const int *expo, const int *active, float2 *gram,
                            int p, int p_pad, int d, int d_pad, int g, int bits, int *status,
                            cudaStream_t s) {
     static std::atomic<unsigned long long> attr_narrow{0}, attr_wide{0};

@@ -69,6 +69,11 @@ CONFIGS = {
         din=4096, dout=4096, g=128, bits=3, K=10, rank=64, n_out=16,
         out_scale=30.0, tokens=262144, w_std=0.015, w_out_frac=0.001,
         w_out_mul=10.0, law="normal", clip=1.0, D_lo=0.05, seed=2),
+    # the q_proj layer at group size 64 (App. "Group size"): 64 groups per row
+    "llama2_7b_q_proj_4096x4096_g64_w3": dict(
+        din=4096, dout=4096, g=64, bits=3, K=10, rank=64, n_out=16,
+        out_scale=30.0, tokens=262144, w_std=0.015, w_out_frac=0.001,
+        w_out_mul=10.0, law="normal", clip=1.0, D_lo=0.05, seed=2),
     "llama2_7b_down_proj_4096x11008_g128_w4": dict(
         din=11008, dout=4096, g=128, bits=4, K=10, rank=64, n_out=32,
         out_scale=30.0, tokens=131072, w_std=0.015, w_out_frac=0.001,
