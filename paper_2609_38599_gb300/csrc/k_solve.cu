@@ -4,8 +4,8 @@
 //  1. reads its G x G Gram matrix -- symmetric by construction, since the
 //     Gram kernel computes each block once and writes it to both triangles,
 //     so the symmetrisation of App. E "Solving for scales" is the identity
-//     on it -- and forms, in float64 (double-float in the G <= 32 kernel
-//     below), the gradient g = rhs - Gram s_old of the current scales
+//     on it -- and forms, in double-float (the Gram entries arrive as
+//     float pairs), the gradient g = rhs - Gram s_old of the current scales
 //     (rhs_i = c_i^T P_i from the target projection) and the objective
 //     F(s_old) = wHw - s_old^T (rhs + g);
 //  2. factors the Gram matrix by Cholesky in float32 (the paper solves this
@@ -16,7 +16,7 @@
 //     increment of the scales: Gram s_new = rhs <=> Gram (s_new - s_old) = g,
 //     and with the ridge (Gram + lambda I) delta = g - lambda s_old (float32
 //     Cholesky, then two refinement steps whose residuals are formed in
-//     float64 or double-float), and stores s_new rounded to float32;
+//     double-float), and stores s_new rounded to float32;
 //  4. evaluates L^{(k)} = F(s_new) = wHw - 2 s_new^T rhs + s_new^T Gram s_new
 //     at the stored float32 scales and applies the early stop of Eq.
 //     strict_stopping against L^{(k-1)}; with the ridge-acceptance option a
@@ -182,7 +182,7 @@ __device__ __forceinline__ DF gram_dot(const float2 *gj, int G, int r0, const fl
 // matrix stays in global memory (L2) and is read row by row; the float32
 // factor lives in shared memory.  Every dot product with the Gram matrix --
 // the gradient, the two refinement residuals, the objective -- is summed in
-// double-float, each float64 entry split into a float pair first.
+// double-float on the entries' float pairs.
 __global__ void scale_solve_kernel(SolveArgs a) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int G = a.d / a.g;
@@ -239,8 +239,9 @@ __global__ void scale_solve_kernel(SolveArgs a) {
         }
         return;
     }
-    // float32 copy of the Gram matrix (the float of a split is the correctly
-    // rounded float32 of the entry), plus a ridge shift of the diagonal
+    // float32 copy of the Gram matrix (the high part of a pair is the
+    // correctly rounded float32 of the entry), plus a ridge shift of the
+    // diagonal
     auto load_sym = [&](float shift) -> bool {
         bool finite = true;
 #pragma unroll 4
@@ -360,8 +361,8 @@ __global__ void scale_solve_kernel(SolveArgs a) {
 // refinement residuals and the objective are done in double-float (pairs of
 // float32 with error-free products and sums, about 48 significant bits).
 // Lane l owns row l of the Gram matrix (= column l: it is exactly
-// symmetric) as a double-float pair per entry, split from the float64 with
-// integer operations.  The float32 Cholesky keeps row l in registers and
+// symmetric) as the double-float pair per entry that the Gram kernel
+// stores.  The float32 Cholesky keeps row l in registers and
 // broadcasts the column of each step with shuffles: the same operations in
 // the same order as warp_cholesky, so the factor (and the ridge decision)
 // is bit-identical.  The triangular solves multiply by the reciprocal of

@@ -34,6 +34,7 @@ def sub_layer(lay_np, rows):
 
 @pytest.mark.parametrize("name", [
     "llama2_7b_q_proj_4096x4096_g128_w3",
+    "llama2_7b_q_proj_4096x4096_g64_w3",      # 64 groups per row
     "llama2_7b_down_proj_4096x11008_g128_w4",
     "llama3_8b_gate_proj_14336x4096_g128_w3",
 ])
