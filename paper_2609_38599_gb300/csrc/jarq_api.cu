@@ -77,14 +77,16 @@ jarq_status cuda_fail(cudaError_t e) {
         }                                      \
     } while (0)
 
-// Launch `call` (which enqueues `n` kernels) under the profiling scope `name`.
-#define RUN(name, n, call)              \
+// Launch `call` (which enqueues `n` kernels on stream `strm`) under the
+// profiling scope `name`.
+#define RUN_ON(name, n, strm, call)     \
     do {                                \
-        ProfScope ps_(name, st);        \
+        ProfScope ps_(name, strm);      \
         CK(call);                       \
         ps_.done();                     \
         count_launches(n);              \
     } while (0)
+#define RUN(name, n, call) RUN_ON(name, n, st, call)
 
 template <class T>
 cudaError_t dalloc(T **p, size_t n) {
@@ -408,6 +410,9 @@ void jarq_hessian_destroy(jarq_hessian *h) {
     cudaFree(h->qstage);
     cudaFree(h->dstatus);
     cudaFreeHost(h->hstatus);
+    if (h->ev_fork) cudaEventDestroy(h->ev_fork);
+    if (h->ev_join) cudaEventDestroy(h->ev_join);
+    if (h->aux) cudaStreamDestroy(h->aux);
     (void)cudaGetLastError();
     delete h;
 }
@@ -609,8 +614,8 @@ jarq_status jarq_multicode_probe(jarq_hessian *h, const float *W, const float *S
                                   h->d_pad, g, h->dstatus, st));
     // T = sum_h s_h H_ih c_h: the phase product with H's own digits
     RUN("target", 1, launch_tc_target(w.mapC, h->mapD10, w.t_hi, w.t_lo, la.S, h->expo, nullptr, p,
-                                      w.p_pad, h->d_pad, g, G, group, nsplit, (1 << bits) - 1, h->dstatus,
-                                      st));
+                                      w.p_pad, h->d_pad, g, G, group, nsplit, 0, p, (1 << bits) - 1,
+                                      h->dstatus, st));
     uint8_t *qo = reinterpret_cast<uint8_t *>(w.Hr);
     RUN("probe", 1, launch_probe(w.Phi, w.Plo, w.t_hi, w.t_lo, h->Hs, h->L64, la.S, la.Q, la.Z, qo,
                                  w.iters, w.accepted, w.ridge, w.L_final, p, w.p_pad, d, g, group,
@@ -659,6 +664,18 @@ jarq_status refine_impl(jarq_hessian *h, const float *W, float *S, uint8_t *Q, c
     RUN("init_rows", 1, launch_init_rows(w.active, w.iters, w.accepted, w.ridge, w.rstat, p, st));
     const ResidualView rv = rview(h);
     const int nsplit = target_splits(w.p_pad, g, G);
+    // rows of the first half of the sweep: the rows split into two halves
+    // only when one phase product needs more than one wave of CTAs (the
+    // halves then fill each other's last wave); otherwise a single chain
+    // with programmatic launches is faster
+    const int tiles = (p + 127) / 128;
+    const bool two_chains = tiles >= kSweepSplitTiles && tiles * (g / 64) * nsplit > num_sms();
+    const int rows_a = two_chains ? (tiles / 2) * 128 : p;
+    if (rows_a < p && !h->aux) {
+        CK(cudaStreamCreateWithFlags(&h->aux, cudaStreamNonBlocking));
+        CK(cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming));
+        CK(cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming));
+    }
     // target projection P = W H, w^T H w and the folded Pt, once per call
     RUN("slice_rows", 1, launch_slice_rows(la.W, w.wdig, w.wexp, p, d, h->d_pad, w.p_pad, g, st));
     RUN("proj", 1, launch_tc_proj(w.mapWd, h->mapD8, w.Phi, w.Plo, w.wexp, h->expo, p, w.p_pad, d,
@@ -681,13 +698,41 @@ jarq_status refine_impl(jarq_hessian *h, const float *W, float *S, uint8_t *Q, c
         RUN("scale_solve", 1, launch_scale_solve(w.gram, w.rhs, w.wHw, la.S, w.L_prev, L_out,
                                                  w.active, w.iters, w.ridge, w.rstat, h->dstatus,
                                                  p, d, g, k, false, o, st));
+        // The sweep.  Rows are independent, so the row tiles form two halves,
+        // each with its own chain of phase products and Babai steps on its
+        // own stream: one half's Babai step runs on the SMs that the other
+        // half's phase product leaves free, and each chain's launch gaps are
+        // filled by the other's work.
+        // Programmatic launch only for a single chain: an early-launched
+        // grid waits on its SMs, which the other half's kernels need.
+        const bool pdl = rows_a == p;
+        cudaStream_t sb = st;
+        if (rows_a < p) {
+            CK(cudaEventRecord(h->ev_fork, st));
+            CK(cudaStreamWaitEvent(h->aux, h->ev_fork, 0));
+            sb = h->aux;
+        }
         for (int i = 0; i < G; ++i) {
             RUN("target", 1, launch_tc_target(w.mapC, h->mapHt, w.t_hi, w.t_lo, la.S, h->expoT,
-                                              w.active, p, w.p_pad, h->d_pad, g, G, i, nsplit,
-                                              qmax, h->dstatus, st));
+                                              w.active, p, w.p_pad, h->d_pad, g, G, i, nsplit, 0,
+                                              rows_a, qmax, h->dstatus, st, pdl));
             RUN("babai", 1, launch_babai(w.t_hi, w.t_lo, w.Pt_hi, w.Pt_lo, nsplit, h->Lf, la.S, la.Q,
                                          la.Z, rv, w.active, w.accepted, h->dstatus, p, g, i, qmax,
-                                         o.eps, st));
+                                         o.eps, 0, rows_a, st, pdl));
+            if (rows_a < p) {
+                RUN_ON("target", 1, sb,
+                       launch_tc_target(w.mapC, h->mapHt, w.t_hi, w.t_lo, la.S, h->expoT,
+                                        w.active, p, w.p_pad, h->d_pad, g, G, i, nsplit, rows_a,
+                                        p - rows_a, qmax, h->dstatus, sb, pdl));
+                RUN_ON("babai", 1, sb,
+                       launch_babai(w.t_hi, w.t_lo, w.Pt_hi, w.Pt_lo, nsplit, h->Lf, la.S, la.Q,
+                                    la.Z, rv, w.active, w.accepted, h->dstatus, p, g, i, qmax,
+                                    o.eps, rows_a, p, sb, pdl));
+            }
+        }
+        if (rows_a < p) {
+            CK(cudaEventRecord(h->ev_join, h->aux));
+            CK(cudaStreamWaitEvent(st, h->ev_join, 0));
         }
     }
     // objective of the returned state (and of the input state when K = 0)

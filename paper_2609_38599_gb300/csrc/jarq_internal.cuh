@@ -23,6 +23,7 @@ enum : int {
 };
 
 constexpr int kMaxGroups = 128;    // largest supported G for the scale solve
+constexpr int kSweepSplitTiles = 8;   // row tiles from which the sweep runs as two halves
 constexpr int kMaxSplit = 16;      // largest split-K factor of the phase product
 
 __host__ __device__ inline int round_up(int x, int m) { return (x + m - 1) / m * m; }
@@ -139,6 +140,9 @@ struct jarq_hessian {
     CUtensorMap mapQ;                  // tensor map of qdig, 64 x 64 boxes
     int *dstatus = nullptr;       // device status word
     int *hstatus = nullptr;       // pinned host mirror
+    // second stream of the sweep and its fork / join events (made on first use)
+    cudaStream_t aux = nullptr;
+    cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
     jarq::Workspace ws;
 };
 
@@ -205,8 +209,8 @@ cudaError_t launch_scale_solve(const float2 *gram, const double *rhs, const doub
 cudaError_t launch_babai(const float *t_hi, const float *t_lo, const float *pt_hi,
                          const float *pt_lo, int nsplit, const float *Lf, const float *S,
                          uint8_t *Q, const int32_t *Z, ResidualView rv, const int *active,
-                         int *accepted, int *status, int p, int g, int i, int qmax, float eps,
-                         cudaStream_t s);
+                         int *accepted, int *status, int p, int g, int i, int qmax, float eps, int row0, int row1,
+                         cudaStream_t s, bool pdl = true);
 cudaError_t launch_slice_rinv(const double *Rinv, __nv_bfloat16 *rdig, int *rexp, int d, int g,
                               cudaStream_t s);
 cudaError_t launch_ptilde(const CUtensorMap &mapPd, const CUtensorMap &mapR, const float *Phi,
@@ -216,15 +220,16 @@ cudaError_t launch_ptilde(const CUtensorMap &mapPd, const CUtensorMap &mapR, con
 int target_splits(int p_pad, int g, int G);
 cudaError_t launch_tc_target(const CUtensorMap &mapC, const CUtensorMap &mapT, float *out_hi,
                              float *out_lo, const float *S, const int *expoT, const int *active,
-                             int p, int p_pad, int d_pad, int g, int G, int i, int nsplit, int qmax,
-                             int *status, cudaStream_t s);
+                             int p, int p_pad, int d_pad, int g, int G, int i, int nsplit,
+                             int row0, int nrows, int qmax, int *status, cudaStream_t s,
+                             bool pdl = true);
 
 // Launch with programmatic stream serialization: the kernel may start while
 // the previous kernel in the stream finishes; it must call griddepcontrol.wait
 // before touching that kernel's inputs or outputs.
 template <class... KArgs, class... Args>
-cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
-                       cudaStream_t s, Args &&...args) {
+cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                     bool pdl, Args &&...args) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = grid;
     cfg.blockDim = block;
@@ -234,28 +239,13 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = pdl ? 1 : 0;
     return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
 }
-// The same with a thread-block cluster of cluster_x CTAs along x.
 template <class... KArgs, class... Args>
-cudaError_t launch_pdl_cluster(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
-                               cudaStream_t s, int cluster_x, Args &&...args) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = grid;
-    cfg.blockDim = block;
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = s;
-    cudaLaunchAttribute attr[2];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    attr[1].id = cudaLaunchAttributeClusterDimension;
-    attr[1].val.clusterDim.x = cluster_x;
-    attr[1].val.clusterDim.y = 1;
-    attr[1].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 2;
-    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t s, Args &&...args) {
+    return launch_k(kernel, grid, block, smem, s, true, static_cast<Args &&>(args)...);
 }
 cudaError_t launch_init_rows(int *active, int *iters, int *accepted, int *ridge, int *rstat,
                              int p, cudaStream_t s);

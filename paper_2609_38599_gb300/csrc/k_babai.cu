@@ -48,6 +48,7 @@ struct BabaiArgs {
     int *status;
     int p, g, i, qmax;
     float eps;
+    int row0, row1;              // rows [row0, row1) of this launch
 };
 
 template <int NT>
@@ -100,7 +101,7 @@ __global__ void __launch_bounds__(32 * kMaxWarps) babai_kernel(BabaiArgs a) {
     const int col0 = a.i * g;
     float rd[NT];
     load_vec<NT>(rdiag + l0, rd);
-    for (int j = blockIdx.x * nwarps + wid; j < a.p; j += gridDim.x * nwarps) {
+    for (int j = a.row0 + blockIdx.x * nwarps + wid; j < a.row1; j += gridDim.x * nwarps) {
         if (!a.active[j]) continue;
         const float s = a.S[(size_t)j * G + a.i];
         if (!(fabsf(s) > a.eps)) continue;  // small-scale skip (also NaN)
@@ -216,26 +217,29 @@ cudaError_t launch_babai(const float *t_hi, const float *t_lo, const float *pt_h
                          const float *pt_lo, int nsplit, const float *Lf, const float *S,
                          uint8_t *Q, const int32_t *Z, ResidualView rv, const int *active,
                          int *accepted, int *status, int p, int g, int i, int qmax, float eps,
-                         cudaStream_t s) {
+                         int row0, int row1, cudaStream_t s, bool pdl) {
+    if (row0 < 0 || row1 > p || row0 > row1) return cudaErrorInvalidValue;
+    if (row0 == row1) return cudaSuccess;
     BabaiArgs a{t_hi, t_lo, pt_hi, pt_lo, nsplit, Lf, S, Q, Z, rv, active, accepted, status,
-                p, g, i, qmax, eps};
+                p, g, i, qmax, eps, row0, row1};
     // one block per SM, one warp per row: spread the rows evenly over the SMs
+    const int rows = row1 - row0;
     const int nsm = num_sms();
-    int warps = (p + nsm - 1) / nsm;
+    int warps = (rows + nsm - 1) / nsm;
     if (warps > kMaxWarps) warps = kMaxWarps;
     if (warps < 1) warps = 1;
-    int blocks = (p + warps - 1) / warps;
+    int blocks = (rows + warps - 1) / warps;
     if (blocks > nsm) blocks = nsm;
     const size_t smem = ((size_t)g * g + g) * sizeof(float);
     cudaError_t e = cudaSuccess;
     if (g == 128) {
         e = cudaFuncSetAttribute(babai_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
-        e = launch_pdl(babai_kernel<4>, dim3(blocks), dim3(32 * warps), smem, s, a);
+        e = launch_k(babai_kernel<4>, dim3(blocks), dim3(32 * warps), smem, s, pdl, a);
     } else if (g == 64) {
         e = cudaFuncSetAttribute(babai_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
-        e = launch_pdl(babai_kernel<2>, dim3(blocks), dim3(32 * warps), smem, s, a);
+        e = launch_k(babai_kernel<2>, dim3(blocks), dim3(32 * warps), smem, s, pdl, a);
     } else {
         return cudaErrorInvalidValue;
     }

@@ -52,6 +52,7 @@ struct TargetArgs {
     const int *active;        // optional: rows still refined
     int *status;
     int p, p_pad, d_pad, g, G, i, seg_per_split;
+    int row0;                 // first row of this launch's tiles (a multiple of 128)
     float round_c;            // 1.5 * 2^(23 - k): rounds to multiples of 2^-k
 };
 
@@ -70,7 +71,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t *tmem_slot = (uint32_t *)(bars + 2 * kStages + 4);
     volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int j0 = blockIdx.x * 128;
+    const int j0 = a.row0 + blockIdx.x * 128;
     const int m0 = a.i * a.g + blockIdx.y * 64;          // first row of Ht (output column)
     const int h0 = blockIdx.z * a.seg_per_split;
     const int h1 = min(a.G, h0 + a.seg_per_split);
@@ -275,12 +276,15 @@ int target_splits(int p_pad, int g, int G) {
 cudaError_t launch_tc_target(const CUtensorMap &mapC, const CUtensorMap &mapT, float *out_hi,
                              float *out_lo, const float *S, const int *expoT, const int *active,
                              int p, int p_pad, int d_pad, int g, int G, int i, int nsplit,
-                             int qmax, int *status, cudaStream_t s) {
+                             int row0, int nrows, int qmax, int *status, cudaStream_t s,
+                             bool pdl) {
     static std::atomic<unsigned long long> attr_done{0};
     const cudaError_t e = set_max_dynamic_smem((const void *)tc_target_kernel, kSmem, attr_done);
     if (e != cudaSuccess) return e;
     const int per = (G + nsplit - 1) / nsplit;
-    const int tiles = p_pad / 128;
+    if (row0 % 128 != 0 || nrows < 0 || row0 + nrows > p_pad) return cudaErrorInvalidValue;
+    const int tiles = (nrows + 127) / 128;
+    if (tiles == 0) return cudaSuccess;
     // quantum 2^-k of the exact digit split: the largest k with
     // 128 qmax 512 + 2^14 <= 2^(24-k)
     if (qmax < 1 || qmax > 255 || g > 128) return cudaErrorInvalidValue;
@@ -289,9 +293,9 @@ cudaError_t launch_tc_target(const CUtensorMap &mapC, const CUtensorMap &mapT, f
     while (kq < 7 && bound <= std::ldexp(1.0, 24 - (kq + 1))) ++kq;
     const float round_c = (float)std::ldexp(1.5, 23 - kq);
     TargetArgs a{out_hi, out_lo, S, expoT, active, status, p, p_pad, d_pad, g, G, i, per,
-                 round_c};
+                 row0, round_c};
     dim3 grid(tiles, g / 64, nsplit);
-    return launch_pdl(tc_target_kernel, grid, dim3(kThreads), (size_t)kSmem, s, mapC, mapT, a);
+    return launch_k(tc_target_kernel, grid, dim3(kThreads), (size_t)kSmem, s, pdl, mapC, mapT, a);
 }
 
 }  // namespace jarq
