@@ -411,8 +411,10 @@ void jarq_hessian_destroy(jarq_hessian *h) {
     cudaFree(h->dstatus);
     cudaFreeHost(h->hstatus);
     if (h->ev_fork) cudaEventDestroy(h->ev_fork);
-    if (h->ev_join) cudaEventDestroy(h->ev_join);
-    if (h->aux) cudaStreamDestroy(h->aux);
+    for (int c = 0; c < kMaxChains - 1; ++c) {
+        if (h->ev_join[c]) cudaEventDestroy(h->ev_join[c]);
+        if (h->aux[c]) cudaStreamDestroy(h->aux[c]);
+    }
     (void)cudaGetLastError();
     delete h;
 }
@@ -664,17 +666,25 @@ jarq_status refine_impl(jarq_hessian *h, const float *W, float *S, uint8_t *Q, c
     RUN("init_rows", 1, launch_init_rows(w.active, w.iters, w.accepted, w.ridge, w.rstat, p, st));
     const ResidualView rv = rview(h);
     const int nsplit = target_splits(w.p_pad, g, G);
-    // rows of the first half of the sweep: the rows split into two halves
+    // chains of the sweep: the row tiles split into nchain contiguous ranges
     // only when one phase product needs more than one wave of CTAs (the
-    // halves then fill each other's last wave); otherwise a single chain
-    // with programmatic launches is faster
+    // chains then fill each other's last wave); otherwise a single chain
+    // with programmatic launches is faster.  Two chains: on the 14336-row
+    // layer three were 2 % faster and four slower.
     const int tiles = (p + 127) / 128;
-    const bool two_chains = tiles >= kSweepSplitTiles && tiles * (g / 64) * nsplit > num_sms();
-    const int rows_a = two_chains ? (tiles / 2) * 128 : p;
-    if (rows_a < p && !h->aux) {
-        CK(cudaStreamCreateWithFlags(&h->aux, cudaStreamNonBlocking));
-        CK(cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming));
-        CK(cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming));
+    const int waves = (tiles * (g / 64) * nsplit + num_sms() - 1) / num_sms();
+    int nchain = (tiles >= kSweepSplitTiles && waves > 1) ? 2 : 1;
+    if (nchain > kMaxChains) nchain = kMaxChains;
+    if (nchain > tiles) nchain = tiles;
+    if (nchain < 1) nchain = 1;
+    int chain_row[kMaxChains + 1];
+    for (int c = 0; c <= nchain; ++c) chain_row[c] = c == nchain ? p : (tiles * c / nchain) * 128;
+    for (int c = 0; c < nchain - 1; ++c) {
+        if (!h->aux[c]) {
+            CK(cudaStreamCreateWithFlags(&h->aux[c], cudaStreamNonBlocking));
+            CK(cudaEventCreateWithFlags(&h->ev_join[c], cudaEventDisableTiming));
+        }
+        if (!h->ev_fork) CK(cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming));
     }
     // target projection P = W H, w^T H w and the folded Pt, once per call
     RUN("slice_rows", 1, launch_slice_rows(la.W, w.wdig, w.wexp, p, d, h->d_pad, w.p_pad, g, st));
@@ -698,41 +708,35 @@ jarq_status refine_impl(jarq_hessian *h, const float *W, float *S, uint8_t *Q, c
         RUN("scale_solve", 1, launch_scale_solve(w.gram, w.rhs, w.wHw, la.S, w.L_prev, L_out,
                                                  w.active, w.iters, w.ridge, w.rstat, h->dstatus,
                                                  p, d, g, k, false, o, st));
-        // The sweep.  Rows are independent, so the row tiles form two halves,
-        // each with its own chain of phase products and Babai steps on its
-        // own stream: one half's Babai step runs on the SMs that the other
-        // half's phase product leaves free, and each chain's launch gaps are
-        // filled by the other's work.
-        // Programmatic launch only for a single chain: an early-launched
-        // grid waits on its SMs, which the other half's kernels need.
-        const bool pdl = rows_a == p;
-        cudaStream_t sb = st;
-        if (rows_a < p) {
+        // The sweep.  Rows are independent, so the row tiles may form several
+        // ranges, each with its own chain of phase products and Babai steps
+        // on its own stream: one chain's Babai step runs on the SMs that
+        // another chain's phase product leaves free, and each chain's launch
+        // gaps are filled by the others' work.  Programmatic launch only for
+        // a single chain: an early-launched grid waits on its SMs, which the
+        // other chains' kernels need.
+        const bool pdl = nchain == 1;
+        if (nchain > 1) {
             CK(cudaEventRecord(h->ev_fork, st));
-            CK(cudaStreamWaitEvent(h->aux, h->ev_fork, 0));
-            sb = h->aux;
+            for (int c = 0; c < nchain - 1; ++c) CK(cudaStreamWaitEvent(h->aux[c], h->ev_fork, 0));
         }
         for (int i = 0; i < G; ++i) {
-            RUN("target", 1, launch_tc_target(w.mapC, h->mapHt, w.t_hi, w.t_lo, la.S, h->expoT,
-                                              w.active, p, w.p_pad, h->d_pad, g, G, i, nsplit, 0,
-                                              rows_a, qmax, h->dstatus, st, pdl));
-            RUN("babai", 1, launch_babai(w.t_hi, w.t_lo, w.Pt_hi, w.Pt_lo, nsplit, h->Lf, la.S, la.Q,
-                                         la.Z, rv, w.active, w.accepted, h->dstatus, p, g, i, qmax,
-                                         o.eps, 0, rows_a, st, pdl));
-            if (rows_a < p) {
-                RUN_ON("target", 1, sb,
+            for (int c = 0; c < nchain; ++c) {
+                cudaStream_t sc = c == 0 ? st : h->aux[c - 1];
+                const int r0 = chain_row[c], r1 = chain_row[c + 1];
+                RUN_ON("target", 1, sc,
                        launch_tc_target(w.mapC, h->mapHt, w.t_hi, w.t_lo, la.S, h->expoT,
-                                        w.active, p, w.p_pad, h->d_pad, g, G, i, nsplit, rows_a,
-                                        p - rows_a, qmax, h->dstatus, sb, pdl));
-                RUN_ON("babai", 1, sb,
+                                        w.active, p, w.p_pad, h->d_pad, g, G, i, nsplit, r0,
+                                        r1 - r0, qmax, h->dstatus, sc, pdl));
+                RUN_ON("babai", 1, sc,
                        launch_babai(w.t_hi, w.t_lo, w.Pt_hi, w.Pt_lo, nsplit, h->Lf, la.S, la.Q,
                                     la.Z, rv, w.active, w.accepted, h->dstatus, p, g, i, qmax,
-                                    o.eps, rows_a, p, sb, pdl));
+                                    o.eps, r0, r1, sc, pdl));
             }
         }
-        if (rows_a < p) {
-            CK(cudaEventRecord(h->ev_join, h->aux));
-            CK(cudaStreamWaitEvent(st, h->ev_join, 0));
+        for (int c = 0; c < nchain - 1; ++c) {
+            CK(cudaEventRecord(h->ev_join[c], h->aux[c]));
+            CK(cudaStreamWaitEvent(st, h->ev_join[c], 0));
         }
     }
     // objective of the returned state (and of the input state when K = 0)

@@ -23,7 +23,8 @@ enum : int {
 };
 
 constexpr int kMaxGroups = 128;    // largest supported G for the scale solve
-constexpr int kSweepSplitTiles = 8;   // row tiles from which the sweep runs as two halves
+constexpr int kSweepSplitTiles = 8;   // row tiles from which the sweep may run as several chains
+constexpr int kMaxChains = 4;         // chains of the sweep at most
 constexpr int kMaxSplit = 16;      // largest split-K factor of the phase product
 
 __host__ __device__ inline int round_up(int x, int m) { return (x + m - 1) / m * m; }
@@ -140,9 +141,10 @@ struct jarq_hessian {
     CUtensorMap mapQ;                  // tensor map of qdig, 64 x 64 boxes
     int *dstatus = nullptr;       // device status word
     int *hstatus = nullptr;       // pinned host mirror
-    // second stream of the sweep and its fork / join events (made on first use)
-    cudaStream_t aux = nullptr;
-    cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+    // extra streams of the sweep's chains and their fork / join events
+    // (made on first use)
+    cudaStream_t aux[jarq::kMaxChains - 1] = {};
+    cudaEvent_t ev_fork = nullptr, ev_join[jarq::kMaxChains - 1] = {};
     jarq::Workspace ws;
 };
 
