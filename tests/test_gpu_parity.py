@@ -105,6 +105,22 @@ def test_many_groups_parity(jarq, din, dout, g, bits, K):
     assert m["gpu_no_worse_than_host"], m
 
 
+def test_two_chain_sweep_parity(jarq):
+    """10200 rows, din 256, g = 128: one phase product needs 80 x 2 = 160 CTAs,
+    more than one wave, so the sweep runs as two chains over the row halves
+    (5120 and 5080 rows, the second ending in a ragged tile).  Every row is
+    compared."""
+    lay = small_layer(256, 10200, 128, 3, K=2, seed=77)
+    prep, res = oracle_run(lay, 2, False)
+    S, Q, st = gpu_refine(lay, 2)
+    assert st["status"] == 0
+    m = compare_final(lay, prep, res, S, Q, st)
+    assert m["codes_same"] >= CODES_SAME, m
+    assert m["S_rel_max_same_rows"] <= REL_S and m["F_rel_max_same_rows"] <= REL_F, m
+    assert m["F_rel_all"] <= REL_F, m
+    assert m["gpu_no_worse_than_host"], m
+
+
 def test_lockstep_tiny_every_difference_is_a_near_tie(jarq):
     lay = tiny_layer()
 
