@@ -55,7 +55,7 @@ TRAFFIC = {
     "rhs": ("k_tc_proj.cu", "6cf1b3d8cc4f", 151.550e6 + 0.264e6),
     "whw": ("k_tc_proj.cu", "6cf1b3d8cc4f", 201.371e6 + 0.190e6),
     "slice_rows": ("k_tc_proj.cu", "6cf1b3d8cc4f", 67.122e6 + 81.168e6),
-    "scale_solve": ("k_solve.cu", "b17a40c3fe33", 35.291e6 + 0.0),
+    "scale_solve": ("k_solve.cu", "e42b89126e93", 35.291e6 + 0.0),
     # captured at 32768 tokens, scaled to 262144
     "syrk": ("k_syrk.cu", "3896afedc783", 8 * 537.171e6 + 40.712e6),
 }

@@ -95,16 +95,6 @@ cudaError_t dalloc(T **p, size_t n) {
     return cudaMalloc((void **)p, n * sizeof(T));
 }
 
-// Split-K factor of the phase product: enough CTAs to cover the SMs.
-int phase_splits(int p_pad, int d_pad) {
-    const int tiles = p_pad / 128, chunks = d_pad / 64;
-    int n = num_sms() / tiles;
-    if (n < 1) n = 1;
-    if (n > kMaxSplit) n = kMaxSplit;
-    if (n > chunks) n = chunks;
-    return n;
-}
-
 bool is_device_ptr(const void *ptr) {
     cudaPointerAttributes at;
     if (cudaPointerGetAttributes(&at, ptr) != cudaSuccess) {
