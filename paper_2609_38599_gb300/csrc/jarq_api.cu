@@ -185,6 +185,23 @@ cudaError_t ensure_ws(jarq_hessian *h, int p) {
     return cudaSuccess;
 }
 
+// Joins the first n extra streams of the sweep to `st` when it goes out of
+// scope: an error return in the middle of a sweep leaves no work of this
+// call running unordered with the caller's stream (best effort: the errors
+// of the join itself are dropped).
+struct ChainJoin {
+    jarq_hessian *h;
+    cudaStream_t st;
+    int n;
+    ~ChainJoin() {
+        if (n == 0) return;
+        for (int c = 0; c < n; ++c)
+            if (cudaEventRecord(h->ev_join[c], h->aux[c]) == cudaSuccess)
+                (void)cudaStreamWaitEvent(st, h->ev_join[c], 0);
+        (void)cudaGetLastError();
+    }
+};
+
 // Device views of the four layer arguments, staging host buffers.
 struct LayerArgs {
     const float *W;
@@ -706,9 +723,13 @@ jarq_status refine_impl(jarq_hessian *h, const float *W, float *S, uint8_t *Q, c
         // a single chain: an early-launched grid waits on its SMs, which the
         // other chains' kernels need.
         const bool pdl = nchain == 1;
+        ChainJoin join{h, st, 0};
         if (nchain > 1) {
             CK(cudaEventRecord(h->ev_fork, st));
-            for (int c = 0; c < nchain - 1; ++c) CK(cudaStreamWaitEvent(h->aux[c], h->ev_fork, 0));
+            for (int c = 0; c < nchain - 1; ++c) {
+                CK(cudaStreamWaitEvent(h->aux[c], h->ev_fork, 0));
+                join.n = c + 1;
+            }
         }
         for (int i = 0; i < G; ++i) {
             for (int c = 0; c < nchain; ++c) {
@@ -724,6 +745,7 @@ jarq_status refine_impl(jarq_hessian *h, const float *W, float *S, uint8_t *Q, c
                                     o.eps, r0, r1, sc, pdl));
             }
         }
+        join.n = 0;
         for (int c = 0; c < nchain - 1; ++c) {
             CK(cudaEventRecord(h->ev_join[c], h->aux[c]));
             CK(cudaStreamWaitEvent(st, h->ev_join[c], 0));
