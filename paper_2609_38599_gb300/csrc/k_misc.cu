@@ -22,6 +22,31 @@ __global__ void validate_kernel(const uint8_t *__restrict__ Q, const int32_t *__
     if (threadIdx.x == 0 && flag) atomicOr(status, flag);
 }
 
+// The same check, sixteen codes per thread (Q 16-byte aligned, nq a
+// multiple of 16).
+__global__ void validate16_kernel(const uint4 *__restrict__ Q16, const int32_t *__restrict__ Z,
+                                  size_t nq16, size_t nz, int qmax, int *status) {
+    __shared__ int flag;
+    if (threadIdx.x == 0) flag = 0;
+    __syncthreads();
+    int local = 0;
+    const size_t stride = (size_t)gridDim.x * blockDim.x;
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < nq16; i += stride) {
+        const uint4 v = Q16[i];
+        const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+#pragma unroll
+            for (int b = 0; b < 4; ++b)
+                if ((int)((w4[k] >> (8 * b)) & 0xFFu) > qmax) local |= ST_BAD_CODE;
+    }
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < nz; i += stride)
+        if (Z[i] < 0 || Z[i] > qmax) local |= ST_BAD_ZERO;
+    if (local) atomicOr(&flag, local);
+    __syncthreads();
+    if (threadIdx.x == 0 && flag) atomicOr(status, flag);
+}
+
 // r = w - s (q - z), one rounding (fma) per element (Eq. quantized_group),
 // and the code plane c = q - z; with rv.r == nullptr only the code plane.
 __global__ void residual_kernel(const float *__restrict__ W, const float *__restrict__ S,
@@ -36,6 +61,27 @@ __global__ void residual_kernel(const float *__restrict__ W, const float *__rest
         const int ci = (int)Q[idx] - Z[j * G + grp];
         if (rv.r) store_residual(rv, j, (int)(idx - j * d), fmaf(-S[j * G + grp], (float)ci, W[idx]));
         store_code(rv, j, (int)(idx - j * d), ci);
+    }
+}
+
+// Only the code plane c = q - z, eight codes per thread (one group: g is a
+// multiple of 8; Q 8-byte aligned; 16-byte stores into the plane).
+__global__ void codes_kernel(const uint8_t *__restrict__ Q, const int32_t *__restrict__ Z,
+                             ResidualView rv, int p, int g) {
+    const int d = rv.d, G = d / g;
+    const size_t n8 = (size_t)p * d / 8;
+    const size_t stride = (size_t)gridDim.x * blockDim.x;
+    for (size_t i8 = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i8 < n8; i8 += stride) {
+        const size_t idx = i8 * 8;
+        const size_t j = idx / d;
+        const int col = (int)(idx - j * d);
+        const int z = Z[j * G + col / g];
+        const uint2 q8 = *reinterpret_cast<const uint2 *>(Q + idx);
+        const uint32_t w2[2] = {q8.x, q8.y};
+        __align__(16) __half h[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) h[k] = __int2half_rn((int)((w2[k >> 2] >> (8 * (k & 3))) & 0xFFu) - z);
+        *reinterpret_cast<uint4 *>(rv.cplane + j * rv.d_pad + col) = *reinterpret_cast<const uint4 *>(h);
     }
 }
 
@@ -91,7 +137,11 @@ cudaError_t launch_validate(const uint8_t *Q, const int32_t *Z, int p, int d, in
     int blocks = (int)((nq + 255) / 256);
     if (blocks > 4 * num_sms()) blocks = 4 * num_sms();
     if (blocks < 1) blocks = 1;
-    validate_kernel<<<blocks, 256, 0, s>>>(Q, Z, nq, nz, qmax, status);
+    if (nq % 16 == 0 && (uintptr_t)Q % 16 == 0)
+        validate16_kernel<<<blocks, 256, 0, s>>>(reinterpret_cast<const uint4 *>(Q), Z, nq / 16, nz,
+                                                 qmax, status);
+    else
+        validate_kernel<<<blocks, 256, 0, s>>>(Q, Z, nq, nz, qmax, status);
     return cudaGetLastError();
 }
 
@@ -101,7 +151,10 @@ cudaError_t launch_residual(const float *W, const float *S, const uint8_t *Q, co
     int blocks = (int)((n + 255) / 256);
     if (blocks > 8 * num_sms()) blocks = 8 * num_sms();
     if (blocks < 1) blocks = 1;
-    residual_kernel<<<blocks, 256, 0, s>>>(W, S, Q, Z, rv, p, g);
+    if (!rv.r && g % 8 == 0 && (uintptr_t)Q % 8 == 0 && rv.d_pad % 8 == 0)
+        codes_kernel<<<blocks, 256, 0, s>>>(Q, Z, rv, p, g);
+    else
+        residual_kernel<<<blocks, 256, 0, s>>>(W, S, Q, Z, rv, p, g);
     return cudaGetLastError();
 }
 
