@@ -715,6 +715,9 @@ jarq_status refine_impl(jarq_hessian *h, const float *W, float *S, uint8_t *Q, c
         RUN("scale_solve", 1, launch_scale_solve(w.gram, w.rhs, w.wHw, la.S, w.L_prev, L_out,
                                                  w.active, w.iters, w.ridge, w.rstat, h->dstatus,
                                                  p, d, g, k, false, o, st));
+        // The phase product reads the active flags only with the early stop
+        // on (to skip tiles whose rows all stopped); a row marked numerical
+        // by the scale solve is skipped by Babai, and its partials go unread.
         // The sweep.  Rows are independent, so the row tiles may form several
         // ranges, each with its own chain of phase products and Babai steps
         // on its own stream: one chain's Babai step runs on the SMs that
@@ -737,8 +740,9 @@ jarq_status refine_impl(jarq_hessian *h, const float *W, float *S, uint8_t *Q, c
                 const int r0 = chain_row[c], r1 = chain_row[c + 1];
                 RUN_ON("target", 1, sc,
                        launch_tc_target(w.mapC, h->mapHt, w.t_hi, w.t_lo, la.S, h->expoT,
-                                        w.active, p, w.p_pad, h->d_pad, g, G, i, nsplit, r0,
-                                        r1 - r0, qmax, h->dstatus, sc, pdl));
+                                        o.early_stop ? w.active : nullptr, p, w.p_pad,
+                                        h->d_pad, g, G, i, nsplit, r0, r1 - r0, qmax,
+                                        h->dstatus, sc, pdl));
                 RUN_ON("babai", 1, sc,
                        launch_babai(w.t_hi, w.t_lo, w.Pt_hi, w.Pt_lo, nsplit, h->Lf, la.S, la.Q,
                                     la.Z, rv, w.active, w.accepted, h->dstatus, p, g, i, qmax,

@@ -102,10 +102,12 @@ __global__ void __launch_bounds__(32 * kMaxWarps) babai_kernel(BabaiArgs a) {
     float rd[NT];
     load_vec<NT>(rdiag + l0, rd);
     for (int j = a.row0 + blockIdx.x * nwarps + wid; j < a.row1; j += gridDim.x * nwarps) {
-        if (!a.active[j]) continue;
+        // the row's flag, scale and zero point are loaded together
+        const int act = a.active[j];
         const float s = a.S[(size_t)j * G + a.i];
-        if (!(fabsf(s) > a.eps)) continue;  // small-scale skip (also NaN)
         const int z = a.Z[(size_t)j * G + a.i];
+        if (!act) continue;
+        if (!(fabsf(s) > a.eps)) continue;  // small-scale skip (also NaN)
         const size_t off = (size_t)j * d + col0;
         // s y = Pt_i - sum_sp T_sp, in double-float
         float y[NT], yl[NT];
