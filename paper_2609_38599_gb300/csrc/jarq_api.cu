@@ -708,9 +708,13 @@ jarq_status refine_impl(jarq_hessian *h, const float *W, float *S, uint8_t *Q, c
     RUN("ptilde", 2, launch_ptilde(w.mapPd, h->mapRi, w.Phi, w.Plo, w.wdig, w.wexp, h->rexp, w.Pt_hi,
                                    w.Pt_lo, p, w.p_pad, d, h->d_pad, g, h->dstatus, st));
     for (int k = 1; k <= o.max_iters; ++k) {
-        RUN("gram", 1, launch_tc_gram(w.mapC, h->mapD10, la.Q, la.Z, h->expo, w.active, w.gram, p,
+        // with the early stop off every row is refined (a row marked numerical
+        // is skipped by the solve and Babai), so the Gram and the right-hand
+        // side need not read the active flags
+        const int *act_es = o.early_stop ? w.active : nullptr;
+        RUN("gram", 1, launch_tc_gram(w.mapC, h->mapD10, la.Q, la.Z, h->expo, act_es, w.gram, p,
                                       w.p_pad, d, h->d_pad, g, bits, h->dstatus, st));
-        RUN("rhs", 1, launch_rhs(la.Q, la.Z, w.Phi, w.Plo, w.active, w.rhs, p, d, g, st));
+        RUN("rhs", 1, launch_rhs(la.Q, la.Z, w.Phi, w.Plo, act_es, w.rhs, p, d, g, st));
         double *L_out = (k == 1 && stats && stats->L_host) ? w.L_host : nullptr;
         RUN("scale_solve", 1, launch_scale_solve(w.gram, w.rhs, w.wHw, la.S, w.L_prev, L_out,
                                                  w.active, w.iters, w.ridge, w.rstat, h->dstatus,

@@ -418,11 +418,13 @@ __global__ void __launch_bounds__(32 * kSmallWarps, 4) scale_solve_small_kernel(
     const int G = a.d / a.g;
     const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int j = blockIdx.x * kSmallWarps + w;
-    if (j >= a.p || (!a.eval_only && !a.active[j])) return;  // warp-uniform
+    if (j >= a.p) return;  // warp-uniform
     const bool own = lane < G;
     const float2 *gj = a.gram + (size_t)j * G * G;
     // row `lane` of the Gram matrix, read column-wise (coalesced) by
-    // symmetry: every load is issued before the first is used
+    // symmetry: every load (and the row's active flag) is issued before the
+    // first is used
+    const int act = a.eval_only ? 1 : a.active[j];
     DF gr[32];
 #pragma unroll
     for (int c = 0; c < 32; ++c) {
@@ -431,6 +433,7 @@ __global__ void __launch_bounds__(32 * kSmallWarps, 4) scale_solve_small_kernel(
     }
     const float so = own ? a.S[(size_t)j * G + lane] : 0.f;
     const double rhs_d = own ? a.rhs[(size_t)j * G + lane] : 0.0;
+    if (!act) return;  // warp-uniform
     const DF rh = split_double(rhs_d);
 
     // gradient g = rhs - Gram s_old and F(s_old) = wHw - s_old^T (rhs + g)
