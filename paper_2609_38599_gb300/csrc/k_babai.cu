@@ -102,17 +102,18 @@ __global__ void __launch_bounds__(32 * kMaxWarps) babai_kernel(BabaiArgs a) {
     float rd[NT];
     load_vec<NT>(rdiag + l0, rd);
     for (int j = a.row0 + blockIdx.x * nwarps + wid; j < a.row1; j += gridDim.x * nwarps) {
-        // the row's flag, scale and zero point are loaded together
+        // the row's flag, scale and zero point, and this lane's slice of the
+        // folded projection Pt_i, are loaded together
+        const size_t off = (size_t)j * d + col0;
         const int act = a.active[j];
         const float s = a.S[(size_t)j * G + a.i];
         const int z = a.Z[(size_t)j * G + a.i];
-        if (!act) continue;
-        if (!(fabsf(s) > a.eps)) continue;  // small-scale skip (also NaN)
-        const size_t off = (size_t)j * d + col0;
-        // s y = Pt_i - sum_sp T_sp, in double-float
         float y[NT], yl[NT];
         load_vec<NT>(a.pt_hi + off + l0, y);
         load_vec<NT>(a.pt_lo + off + l0, yl);
+        if (!act) continue;
+        if (!(fabsf(s) > a.eps)) continue;  // small-scale skip (also NaN)
+        // s y = Pt_i - sum_sp T_sp, in double-float
         for (int sp = 0; sp < a.nsplit; ++sp) {
             float th[NT], tl[NT];
             const size_t o = ((size_t)sp * a.rv.p_pad + j) * g + l0;
