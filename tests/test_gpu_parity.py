@@ -105,14 +105,18 @@ def test_many_groups_parity(jarq, din, dout, g, bits, K):
     assert m["gpu_no_worse_than_host"], m
 
 
-def test_two_chain_sweep_parity(jarq):
+@pytest.mark.parametrize("early_stop", [False, True])
+def test_two_chain_sweep_parity(jarq, early_stop):
     """10200 rows, din 256, g = 128: one phase product needs 80 x 2 = 160 CTAs,
     more than one wave, so the sweep runs as two chains over the row halves
     (5120 and 5080 rows, the second ending in a ragged tile).  Every row is
-    compared."""
-    lay = small_layer(256, 10200, 128, 3, K=2, seed=77)
-    prep, res = oracle_run(lay, 2, False)
-    S, Q, st = gpu_refine(lay, 2)
+    compared; with the early stop on, also the stopping iterations."""
+    K = 4 if early_stop else 2
+    lay = small_layer(256, 10200, 128, 3, K=K, seed=77)
+    prep, res = oracle_run(lay, K, early_stop)
+    S, Q, st = gpu_refine(lay, K, early_stop=early_stop)
+    if early_stop:
+        assert np.mean(st["iters"] == res.iters) >= 0.99
     assert st["status"] == 0
     m = compare_final(lay, prep, res, S, Q, st)
     assert m["codes_same"] >= CODES_SAME, m
