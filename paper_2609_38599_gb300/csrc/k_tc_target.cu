@@ -108,6 +108,22 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc::tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    // Before the wait on the previous grid: without the early stop (no
+    // active flags to read) the tile's work is known, and the Ht digit tiles
+    // of the first stages -- constant during the refinement -- are requested
+    // already; only the code tiles, which the previous Babai step rewrites,
+    // wait.
+    int npre = 0;
+    if (!a.active && warp == 0 && lane == 0) {
+        npre = min(kStages, (j0 < a.p ? max(0, h1 - h0) : 0) * nkc);
+        for (int c = 0; c < npre; ++c) {
+            const int kx = h0 * a.g + c * 64;
+            tc::mbar_add_tx(full(c), 4 * kTileB);
+#pragma unroll
+            for (int t = 0; t < 4; ++t)
+                tc::tma_load_2d(tileB(c, t), &mapT, full(c), kx, t * a.d_pad + m0);
+        }
+    }
     // the codes are rewritten by the previous Babai phase
     tc::pdl_wait();
     tc::pdl_launch_dependents();
@@ -128,17 +144,29 @@ __global__ void __launch_bounds__(kThreads, 1)
                 break;
             }
             const int kx = h0 * a.g + c * 64;
-            tc::mbar_expect_tx(full(s), kStage);
-            tc::tma_load_2d(tileA(s), &mapC, full(s), kx, j0);
+            if (c < npre) {
+                // the digit tiles of this stage are already in flight
+                tc::mbar_expect_tx(full(s), kTileA);
+                tc::tma_load_2d(tileA(s), &mapC, full(s), kx, j0);
+            } else {
+                tc::mbar_expect_tx(full(s), kStage);
+                tc::tma_load_2d(tileA(s), &mapC, full(s), kx, j0);
 #pragma unroll
-            for (int t = 0; t < 4; ++t)
-                tc::tma_load_2d(tileB(s, t), &mapT, full(s), kx, t * a.d_pad + m0);
+                for (int t = 0; t < 4; ++t)
+                    tc::tma_load_2d(tileB(s, t), &mapT, full(s), kx, t * a.d_pad + m0);
+            }
             issued = c + 1;
         }
         // do not leave before the MMAs have consumed the stages filled here:
         // no copy or commit is in flight afterwards
         for (int c = issued > kStages ? issued - kStages : 0; c < issued; ++c)
             if (!tc::mbar_wait(empty(c % kStages), (c / kStages) & 1)) *abort_flag = 1;
+        // after an abort: digit tiles requested before the wait for stages
+        // never issued must land before the CTA leaves
+        for (int c = issued; c < npre; ++c) {
+            tc::mbar_arrive(full(c));
+            if (!tc::mbar_wait(full(c), 0)) *abort_flag = 1;
+        }
     } else if (warp == 1 && lane == 0) {
         // ---------------- MMA issuer: one unit per group h
         for (int u = 0; u < nseg && !*abort_flag; ++u) {
