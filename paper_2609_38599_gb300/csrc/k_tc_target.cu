@@ -109,16 +109,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::tc_fence_after();
     const uint32_t tmem = *tmem_slot;
     // Before the wait on the previous grid: without the early stop (no
-    // active flags to read) the tile's work is known, and the Ht digit tiles
-    // of the first stages -- constant during the refinement -- are requested
-    // already; only the code tiles, which the previous Babai step rewrites,
-    // wait.
+    // active flags to read) the tile's work is known, and the first stages
+    // are requested already.  Their Ht digit tiles are constant during the
+    // refinement; their code tiles too, except those of group i - 1, which
+    // the previous Babai step rewrites: a stage of that group requests its
+    // code tile after the wait.
     int npre = 0;
+    uint32_t pre_full = 0;   // stages whose code tile is requested too
     if (!a.active && warp == 0 && lane == 0) {
         npre = min(kStages, (j0 < a.p ? max(0, h1 - h0) : 0) * nkc);
         for (int c = 0; c < npre; ++c) {
             const int kx = h0 * a.g + c * 64;
-            tc::mbar_add_tx(full(c), 4 * kTileB);
+            if (h0 + c / nkc != a.i - 1) {
+                pre_full |= 1u << c;
+                tc::mbar_expect_tx(full(c), kStage);
+                tc::tma_load_2d(tileA(c), &mapC, full(c), kx, j0);
+            } else {
+                tc::mbar_add_tx(full(c), 4 * kTileB);
+            }
 #pragma unroll
             for (int t = 0; t < 4; ++t)
                 tc::tma_load_2d(tileB(c, t), &mapT, full(c), kx, t * a.d_pad + m0);
@@ -145,9 +153,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             const int kx = h0 * a.g + c * 64;
             if (c < npre) {
-                // the digit tiles of this stage are already in flight
-                tc::mbar_expect_tx(full(s), kTileA);
-                tc::tma_load_2d(tileA(s), &mapC, full(s), kx, j0);
+                // the digit tiles of this stage (and maybe its code tile)
+                // are already in flight
+                if (!((pre_full >> c) & 1u)) {
+                    tc::mbar_expect_tx(full(s), kTileA);
+                    tc::tma_load_2d(tileA(s), &mapC, full(s), kx, j0);
+                }
             } else {
                 tc::mbar_expect_tx(full(s), kStage);
                 tc::tma_load_2d(tileA(s), &mapC, full(s), kx, j0);
@@ -164,7 +175,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // after an abort: digit tiles requested before the wait for stages
         // never issued must land before the CTA leaves
         for (int c = issued; c < npre; ++c) {
-            tc::mbar_arrive(full(c));
+            if (!((pre_full >> c) & 1u)) tc::mbar_arrive(full(c));
             if (!tc::mbar_wait(full(c), 0)) *abort_flag = 1;
         }
     } else if (warp == 1 && lane == 0) {
