@@ -108,43 +108,31 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc::tc_fence_after();
     const uint32_t tmem = *tmem_slot;
-    // Before the wait on the previous grid: without the early stop (no
-    // active flags to read) the tile's work is known, and the first stages
-    // are requested already.  Their Ht digit tiles are constant during the
-    // refinement; their code tiles too, except those of group i - 1, which
-    // the previous Babai step rewrites: a stage of that group requests its
-    // code tile after the wait.
-    int npre = 0;
-    uint32_t pre_full = 0;   // stages whose code tile is requested too
-    if (!a.active && warp == 0 && lane == 0) {
-        npre = min(kStages, (j0 < a.p ? max(0, h1 - h0) : 0) * nkc);
-        for (int c = 0; c < npre; ++c) {
-            const int kx = h0 * a.g + c * 64;
-            if (h0 + c / nkc != a.i - 1) {
-                pre_full |= 1u << c;
-                tc::mbar_expect_tx(full(c), kStage);
-                tc::tma_load_2d(tileA(c), &mapC, full(c), kx, j0);
-            } else {
-                tc::mbar_add_tx(full(c), 4 * kTileB);
-            }
-#pragma unroll
-            for (int t = 0; t < 4; ++t)
-                tc::tma_load_2d(tileB(c, t), &mapT, full(c), kx, t * a.d_pad + m0);
-        }
-    }
-    // the codes are rewritten by the previous Babai phase
-    tc::pdl_wait();
+    // The previous grid (the Babai step of group i - 1) rewrites only the
+    // codes of group i - 1, and reads the phase partials this grid writes.
+    // Without the early stop (no active flags to read) each role therefore
+    // waits for it only where it must: the producer before the code tile of
+    // a chunk of group i - 1, the drain before writing the partials.  The
+    // Ht digit tiles, the other code tiles and the scales do not change
+    // during the sweep, so the products of the other groups can run while
+    // the previous grid finishes.  With the early stop every thread waits
+    // here, before reading the flags; so it does in the first phase, whose
+    // previous grid is the scale solve that writes the scales.
+    const bool early = !a.active && a.i > 0;
+    if (!early) tc::pdl_wait();
     tc::pdl_launch_dependents();
     // a tile none of whose rows is still active (early stop, App. E) does
     // no work: the Babai step reads the partials of active rows only
-    const bool live = __syncthreads_or(threadIdx.x < 128 && j0 + (int)threadIdx.x < a.p &&
-                                       (!a.active || a.active[j0 + threadIdx.x] != 0));
+    const bool live = early ? j0 < a.p
+                            : __syncthreads_or(threadIdx.x < 128 && j0 + (int)threadIdx.x < a.p &&
+                                               (!a.active || a.active[j0 + threadIdx.x] != 0));
     const int nseg = live ? max(0, h1 - h0) : 0;
     const int nchunks = nseg * nkc;
 
     if (warp == 0 && lane == 0) {
         // ---------------- producer
         int issued = 0;
+        bool waited = !early;
         for (int c = 0; c < nchunks; ++c) {
             const int s = c % kStages;
             if (!tc::mbar_wait(empty(s), ((c / kStages) & 1) ^ 1) || *abort_flag) {
@@ -152,32 +140,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                 break;
             }
             const int kx = h0 * a.g + c * 64;
-            if (c < npre) {
-                // the digit tiles of this stage (and maybe its code tile)
-                // are already in flight
-                if (!((pre_full >> c) & 1u)) {
-                    tc::mbar_expect_tx(full(s), kTileA);
-                    tc::tma_load_2d(tileA(s), &mapC, full(s), kx, j0);
-                }
-            } else {
-                tc::mbar_expect_tx(full(s), kStage);
-                tc::tma_load_2d(tileA(s), &mapC, full(s), kx, j0);
-#pragma unroll
-                for (int t = 0; t < 4; ++t)
-                    tc::tma_load_2d(tileB(s, t), &mapT, full(s), kx, t * a.d_pad + m0);
+            if (!waited && h0 + c / nkc == a.i - 1) {
+                tc::pdl_wait();   // the codes of group i - 1
+                waited = true;
             }
+            tc::mbar_expect_tx(full(s), kStage);
+            tc::tma_load_2d(tileA(s), &mapC, full(s), kx, j0);
+#pragma unroll
+            for (int t = 0; t < 4; ++t)
+                tc::tma_load_2d(tileB(s, t), &mapT, full(s), kx, t * a.d_pad + m0);
             issued = c + 1;
         }
         // do not leave before the MMAs have consumed the stages filled here:
         // no copy or commit is in flight afterwards
         for (int c = issued > kStages ? issued - kStages : 0; c < issued; ++c)
             if (!tc::mbar_wait(empty(c % kStages), (c / kStages) & 1)) *abort_flag = 1;
-        // after an abort: digit tiles requested before the wait for stages
-        // never issued must land before the CTA leaves
-        for (int c = issued; c < npre; ++c) {
-            if (!((pre_full >> c) & 1u)) tc::mbar_arrive(full(c));
-            if (!tc::mbar_wait(full(c), 0)) *abort_flag = 1;
-        }
     } else if (warp == 1 && lane == 0) {
         // ---------------- MMA issuer: one unit per group h
         for (int u = 0; u < nseg && !*abort_flag; ++u) {
@@ -278,6 +255,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
         }
+        // the previous grid reads the partials this drain overwrites
+        if (early) tc::pdl_wait();
         if (ok && row < a.p) {
             const size_t o = (size_t)blockIdx.z * a.p_pad * a.g + (size_t)row * a.g + blockIdx.y * 64 + cq * 16;
 #pragma unroll
