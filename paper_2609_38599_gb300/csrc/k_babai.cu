@@ -32,7 +32,7 @@
 namespace jarq {
 namespace {
 
-constexpr int kMaxWarps = 32;   // warps per block (one row each) at most
+constexpr int kMaxWarps = 28;   // warps per block (one row each) at most
 
 struct BabaiArgs {
     const float *t_hi, *t_lo;    // [nsplit][p_pad][g] split-K partials of T_i
@@ -93,9 +93,14 @@ __global__ void __launch_bounds__(32 * kMaxWarps) babai_kernel(BabaiArgs a) {
     for (int l = threadIdx.x; l < g; l += blockDim.x) rdiag[l] = 1.0f / Lg[l * g + l];
     __syncthreads();
     // the phase product (previous kernel) must be complete before its
-    // partials are read and before the residual it reads is rewritten
-    tc::pdl_wait();
-    tc::pdl_launch_dependents();
+    // partials are read and before the codes it reads are rewritten: each
+    // thread waits for it just before reading the partials (the loads of a
+    // row's flag, scale, zero point and Pt slice, which the phase product
+    // does not write, come first).  The next grid is released only after
+    // the wait: by then every grid before this one has completed, so the
+    // next phase product may read the codes of the groups this step leaves
+    // alone before its own wait.
+    bool waited = false;
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
     const int l0 = NT * lane;
     const int col0 = a.i * g;
@@ -114,6 +119,11 @@ __global__ void __launch_bounds__(32 * kMaxWarps) babai_kernel(BabaiArgs a) {
         if (!act) continue;
         if (!(fabsf(s) > a.eps)) continue;  // small-scale skip (also NaN)
         // s y = Pt_i - sum_sp T_sp, in double-float
+        if (!waited) {
+            tc::pdl_wait();
+            tc::pdl_launch_dependents();
+            waited = true;
+        }
         for (int sp = 0; sp < a.nsplit; ++sp) {
             float th[NT], tl[NT];
             const size_t o = ((size_t)sp * a.rv.p_pad + j) * g + l0;

@@ -120,6 +120,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     // previous grid is the scale solve that writes the scales.
     const bool early = !a.active && a.i > 0;
     if (!early) tc::pdl_wait();
+    // The next grid (Babai of group i) is released at once: before its own
+    // wait it reads nothing that this grid or the previous one writes.
     tc::pdl_launch_dependents();
     // a tile none of whose rows is still active (early stop, App. E) does
     // no work: the Babai step reads the partials of active rows only
