@@ -32,7 +32,7 @@
 namespace jarq {
 namespace {
 
-constexpr int kMaxWarps = 28;   // warps per block (one row each) at most
+constexpr int kMaxWarps = 32;   // warps per block (one row each) at most
 
 struct BabaiArgs {
     const float *t_hi, *t_lo;    // [nsplit][p_pad][g] split-K partials of T_i
