@@ -323,7 +323,9 @@ def run_ours(args, rank, world):
     if world > 1:
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
-    lay = config_layer(args.workload, device=dev)
+    # each rank refines its own layer of the same shape (rank 0: the named
+    # layer): independent problems, weak scaling, no collective on the path
+    lay = config_layer(args.workload, device=dev, seed_offset=rank)
     hess = jarq.prepare(lay.H, lay.g)
     opts = jarq.default_options(max_iters=lay.K, early_stop=0)
     S = lay.S0.clone()

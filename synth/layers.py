@@ -253,14 +253,17 @@ def weights_torch(dout, din, w_std, w_out_frac, w_out_mul, law, seed, device):
     return W.float().contiguous()
 
 
-def config_layer(name, device="cuda", H=None):
-    """Build one named full-size layer on ``device`` (torch tensors)."""
+def config_layer(name, device="cuda", H=None, seed_offset=0):
+    """Build one named full-size layer on ``device`` (torch tensors).
+    ``seed_offset`` draws another instance of the same shape and statistics
+    (0: the named layer itself)."""
     c = CONFIGS[name]
+    seed = c["seed"] + 7919 * seed_offset
     if H is None:
         H = hessian_torch(c["din"], c["rank"], c["n_out"], c["out_scale"], c["tokens"],
-                          c["D_lo"], c["seed"], device)
+                          c["D_lo"], seed, device)
     W = weights_torch(c["dout"], c["din"], c["w_std"], c["w_out_frac"], c["w_out_mul"],
-                      c["law"], 1000 + c["seed"], device)
+                      c["law"], 1000 + seed, device)
     S0, Q0, Z = rtn_host_torch(W, c["bits"], c["g"], c["clip"])
     return Layer(name, W, H, S0, Q0, Z, c["bits"], c["g"], c["K"])
 

@@ -112,3 +112,16 @@ def test_token_sharded_hessian_equals_single_process():
     from synth import integer_activations_np
     X = integer_activations_np(1001, 24, amax=8, seed=5)
     np.testing.assert_array_equal(H, accumulate_hessian(X))
+
+
+def test_rank_layer_instances():
+    """Under torchrun each rank refines its own instance of the named layer
+    (independent problems, weak scaling): offset 0 is the named layer itself,
+    another offset draws different data of the same shape."""
+    from synth import config_layer
+    a = config_layer("tiny_256x256_g64_w3", device="cpu")
+    b = config_layer("tiny_256x256_g64_w3", device="cpu", seed_offset=0)
+    c = config_layer("tiny_256x256_g64_w3", device="cpu", seed_offset=1)
+    assert torch.equal(a.W, b.W) and torch.equal(a.H, b.H) and torch.equal(a.Q0, b.Q0)
+    assert a.W.shape == c.W.shape and a.H.shape == c.H.shape
+    assert not torch.equal(a.W, c.W) and not torch.equal(a.H, c.H)
