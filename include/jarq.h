@@ -52,7 +52,7 @@ typedef enum jarq_status {
     JARQ_ERR_NOT_SPD = 2,    /* a diagonal block H_ii is not positive definite */
     JARQ_ERR_NUMERICAL = 3,  /* a scale system failed even with the ridge      */
     JARQ_ERR_CUDA = 4,       /* a CUDA runtime or driver call failed           */
-    JARQ_ERR_TIMEOUT = 5,    /* reserved: a bounded device wait gave up        */
+    JARQ_ERR_TIMEOUT = 5,    /* a bounded device wait gave up; outputs invalid  */
     JARQ_ERR_NOMEM = 6       /* device allocation failed                       */
 } jarq_status;
 
@@ -339,6 +339,16 @@ void jarq_profile_reset(void);
 int jarq_profile_read(const char *kernel, long long *launches, double *total_ms);
 /* Number of kernels this library has launched since it was loaded. */
 long long jarq_launch_count(void);
+
+/* Test hook for the bounded device waits (no counterpart in the paper).
+ * Every wait of the library's kernels on a barrier gives up after a fixed
+ * number of polls; the kernel then records the timeout, finishes its copies
+ * in flight and returns, and the call reports JARQ_ERR_TIMEOUT.  This call
+ * launches one thread that waits on a barrier nothing completes, with a
+ * short poll limit, and returns the status the same path produces:
+ * JARQ_ERR_TIMEOUT when it works.  The CUDA context stays usable.  `stream`
+ * as for every entry point; returns after the stream work has finished. */
+jarq_status jarq_selftest_wait_timeout(void *stream);
 
 #ifdef __cplusplus
 }

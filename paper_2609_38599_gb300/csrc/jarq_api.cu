@@ -379,6 +379,26 @@ jarq_options jarq_default_options(void) {
     return o;
 }
 
+jarq_status jarq_selftest_wait_timeout(void *stream) {
+    cudaStream_t st = (cudaStream_t)stream;
+    int *d = nullptr;
+    int bits = 0;
+    if (cudaMalloc(&d, sizeof(int)) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return JARQ_ERR_NOMEM;
+    }
+    cudaError_t e = cudaMemsetAsync(d, 0, sizeof(int), st);
+    if (e == cudaSuccess) e = launch_wait_timeout(d, 256, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&bits, d, sizeof(int), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    cudaFree(d);
+    if (e != cudaSuccess) {
+        (void)cudaGetLastError();
+        return JARQ_ERR_CUDA;
+    }
+    return status_from_bits(bits);
+}
+
 const char *jarq_status_string(jarq_status s) {
     switch (s) {
         case JARQ_OK: return "ok";

@@ -220,6 +220,7 @@ cudaError_t launch_ptilde(const CUtensorMap &mapPd, const CUtensorMap &mapR, con
                           float *out_hi, float *out_lo, int p, int p_pad, int d, int d_pad, int g,
                           int *status, cudaStream_t s);
 int target_splits(int p_pad, int g, int G);
+cudaError_t launch_wait_timeout(int *status, uint32_t polls, cudaStream_t s);
 cudaError_t launch_tc_target(const CUtensorMap &mapC, const CUtensorMap &mapT, float *out_hi,
                              float *out_lo, const float *S, const int *expoT, const int *active,
                              int p, int p_pad, int d_pad, int g, int G, int i, int nsplit,

@@ -1,5 +1,5 @@
 // Elementwise and bookkeeping kernels of the refinement path.
-#include "jarq_internal.cuh"
+#include "tc_common.cuh"
 
 namespace jarq {
 namespace {
@@ -161,6 +161,25 @@ cudaError_t launch_residual(const float *W, const float *S, const uint8_t *Q, co
 cudaError_t launch_init_rows(int *active, int *iters, int *accepted, int *ridge, int *rstat,
                              int p, cudaStream_t s) {
     init_rows_kernel<<<(p + 255) / 256, 256, 0, s>>>(active, iters, accepted, ridge, rstat, p);
+    return cudaGetLastError();
+}
+
+// A wait that nothing completes: one thread polls a fresh mbarrier (count 1,
+// no arrival), gives up after `polls` polls and records ST_TIMEOUT, as every
+// kernel of the library does when one of its bounded waits runs out.
+__global__ void wait_timeout_kernel(int *status, uint32_t polls) {
+    __shared__ uint64_t bar;
+    if (threadIdx.x != 0) return;
+    const uint32_t b = tc::smem_u32(&bar);
+    tc::mbar_init(b, 1);
+    tc::fence_barrier_init();
+    bool done = false;
+    for (uint32_t i = 0; i < polls && !done; ++i) done = tc::mbar_try_wait(b, 0);
+    if (!done) atomicOr(status, ST_TIMEOUT);
+}
+
+cudaError_t launch_wait_timeout(int *status, uint32_t polls, cudaStream_t s) {
+    wait_timeout_kernel<<<1, 32, 0, s>>>(status, polls);
     return cudaGetLastError();
 }
 

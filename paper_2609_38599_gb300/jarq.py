@@ -32,7 +32,8 @@ EXPORTS = ("jarq_default_options", "jarq_prepare_hessian", "jarq_refine_layer",
            "jarq_profile_reset", "jarq_profile_read", "jarq_launch_count",
            "jarq_objective_noalloc", "jarq_residual_product", "jarq_canonicalize",
            "jarq_dequantize", "jarq_pack_codes", "jarq_accumulate_hessian",
-           "jarq_refine_layer_mu", "jarq_fit_scales", "jarq_multicode_probe")
+           "jarq_refine_layer_mu", "jarq_fit_scales", "jarq_multicode_probe",
+           "jarq_selftest_wait_timeout")
 
 
 class JarqError(RuntimeError):
@@ -106,6 +107,8 @@ def _load():
                                       ctypes.POINTER(ctypes.c_double)]
     lib.jarq_launch_count.restype = ctypes.c_longlong
     lib.jarq_launch_count.argtypes = []
+    lib.jarq_selftest_wait_timeout.restype = ci
+    lib.jarq_selftest_wait_timeout.argtypes = [vp]
     return lib
 
 
@@ -143,6 +146,13 @@ def profile_read(kernel: str):
 def launch_count() -> int:
     """Kernels launched by the library since it was loaded."""
     return int(_lib.jarq_launch_count())
+
+
+def selftest_wait_timeout() -> int:
+    """Status of a device wait that nothing completes (JARQ_ERR_TIMEOUT when
+    the bounded-wait path works), on the current torch stream."""
+    import torch
+    return int(_lib.jarq_selftest_wait_timeout(ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)))
 
 
 def status_string(status: int) -> str:

@@ -297,3 +297,18 @@ def test_small_scale_group_keeps_codes(jarq):
     S, Qg, st = gpu_refine(lay2, 1)
     assert np.all(np.abs(S[:, 1]) <= 1e-6)
     assert np.array_equal(Qg[:, 64:128], Q[:, 64:128])
+
+
+def test_bounded_wait_reports_timeout_and_context_survives(jarq):
+    """A device wait that nothing completes gives up after its poll limit and
+    the call reports JARQ_ERR_TIMEOUT, through the status word and mapping
+    every kernel's bounded waits use; the context stays usable afterwards:
+    the tiny layer still refines as the oracle does."""
+    assert jarq.selftest_wait_timeout() == jarq.JARQ_ERR_TIMEOUT
+    lay = tiny_layer()
+    prep, res = oracle_run(lay, 2, False)
+    S, Q, st = gpu_refine(lay, 2, early_stop=False)
+    assert st["status"] == 0
+    m = compare_final(lay, prep, res, S, Q, st)
+    assert m["codes_same"] >= CODES_SAME, m
+    assert m["F_rel_all"] <= REL_F, m
